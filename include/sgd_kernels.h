@@ -1,0 +1,98 @@
+/*
+ * sgd_kernels.h — kernel-level entry points of libsgd, one per hot-path kernel of
+ * the scheduled denoiser step.  They exist so that every kernel can be checked
+ * against the CPU oracle on its own; sgd_step launches the same kernels with the
+ * same launch configurations.
+ *
+ * Paper passages (Algorithm 2, "Jagged-Stream Execution"):
+ *   - an active unit computes Delta_{l,s} = F_l(h_{l-1,s}; c_s), refreshes its cache
+ *     and sets h_{l,s} = h_{l-1,s} + Delta   -> sgd_kernel_gemm with SGD_EPI_DELTA
+ *     (the branch's last projection, its epilogue stores the cache and adds to h);
+ *   - the branch body F_l (norm, projections, attention, MLP activation)
+ *                                          -> sgd_kernel_norm, sgd_kernel_gemm,
+ *                                             sgd_kernel_attention;
+ *   - a frozen unit reads its cached Delta_{l, r_l(s)} and adds it to the current
+ *     residual stream                        -> sgd_kernel_frozen_run (one pass over h
+ *     for a run of consecutive frozen units).
+ *
+ * All pointers are device pointers; all calls are asynchronous on `stream`
+ * (a cudaStream_t) and return an sgd_status (sgd.h).  Arguments are validated on
+ * the host (SGD_ERR_ARG / SGD_ERR_SHAPE); nothing is launched on a validation error.
+ */
+#ifndef SGD_KERNELS_H
+#define SGD_KERNELS_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Epilogue applied to the fp32 accumulator tile of C = A B^T. */
+typedef enum {
+  SGD_EPI_BF16 = 0,   /* out bf16 [M, N] = acc                                          */
+  SGD_EPI_F32 = 1,    /* out fp32 [M, N] = acc                                          */
+  SGD_EPI_DELTA = 2,  /* Delta = gate * acc; h fp32 [M, N] += Delta; cache bf16 = Delta   */
+  SGD_EPI_GATED = 3,  /* B has 2f rows; out bf16 [M, f] = act(acc[:, :f], acc[:, f:])   */
+  SGD_EPI_GELU = 4,   /* out bf16 [M, N] = gelu(acc)                                    */
+  SGD_EPI_ROPE = 5    /* out bf16 [M, N] = acc with rotate-half RoPE on columns < rope_cols */
+} sgd_epilogue_kind;
+
+typedef struct {
+  int kind;                      /* sgd_epilogue_kind                                        */
+  void* out; int ldo;            /* output (elements); unused by SGD_EPI_DELTA               */
+  float* h; int ldh;             /* DELTA: fp32 residual updated in place                   */
+  void* cache; int ld_cache;     /* DELTA: optional bf16 copy of Delta (NULL: not stored)    */
+  const float* gate;             /* DELTA: optional fp32 gate [B, ld_gate], row r uses sample r / rows_per_batch */
+  int ld_gate, rows_per_batch;
+  int act;                       /* GATED: 0 = silu(a) * b (SwiGLU), 1 = a * gelu_erf(b) (GEGLU);
+                                    GELU: 0 = tanh form, 1 = erf form                           */
+  const float* rope_cos;         /* ROPE: fp32 [rope_tokens, d_head / 2] tables, row = token % rope_tokens */
+  const float* rope_sin;
+  int rope_tokens, d_head, rope_cols;
+} sgd_epilogue_args;
+
+/*
+ * C = A B^T.  A bf16 [M, K] (row stride lda elements), B bf16 [N or 2N, K] (row
+ * stride ldb).  K, lda, ldb multiples of 8; N multiple of 8; pointers 16-byte
+ * aligned.  use_simt = 1 runs the plain SIMT kernel (reference / debugging), 0 the
+ * tcgen05 + TMA kernel.
+ */
+int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
+                    const sgd_epilogue_args* epi, int use_simt, void* stream);
+
+/*
+ * O = softmax(Q K^T / sqrt(d_head)) V per (sample, head), non-causal, keys beyond n_kv
+ * masked.  Row r = b * n_q + i of q / o, row b * n_kv + j of k / v; head h occupies
+ * columns [h d_head, (h+1) d_head).  bf16 in and out; d_head in {64, 72, 128};
+ * leading dimensions in elements, multiples of 8.
+ */
+int sgd_kernel_attention(const void* q, int ldq, const void* k, const void* v, int ldkv,
+                         void* o, int ldo, int batch, int n_q, int n_kv, int n_heads,
+                         int d_head, void* stream);
+
+/*
+ * out bf16 [rows, d] = norm(h fp32 [rows, d]); kind = sgd_norm_kind.  g, b: bf16 [d]
+ * (NULL allowed for LN_PLAIN).  shift/scale: optional fp32 AdaLN modulation
+ * [B, ld_mod]: out = norm(h) * (1 + scale[r / rows_per_batch]) + shift[...].
+ */
+int sgd_kernel_norm(const float* h, void* out, int rows, int d, int kind, const void* g,
+                    const void* b, const float* shift, const float* scale, int ld_mod,
+                    int rows_per_batch, float eps, void* stream);
+
+/*
+ * h fp32 [n] += sum_{i < n_caches} caches[i] (bf16 [n]), summed in order i = 0, 1, ...
+ * in fp32.  caches_host: host array of n_caches (<= 96) device pointers.  n multiple
+ * of 8, pointers 16-byte aligned.
+ */
+int sgd_kernel_frozen_run(float* h, const void* const* caches_host, int n_caches, int64_t n,
+                          void* stream);
+
+/* Device status word shared by all kernels (bounded-wait expiry); returns and clears it. */
+int sgd_kernel_status(int* status_host);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SGD_KERNELS_H */

@@ -1,0 +1,1065 @@
+// C ABI of libsgd (include/sgd.h, include/sgd_kernels.h).
+//
+// sgd_create       borrows the weights, allocates the residual stream and workspaces.
+// sgd_set_schedule compiles per-unit lifetimes (Sec. 4.1, Eq. schedule) into the per-step
+//                  active/frozen patterns of Sec. 4.2 and captures one CUDA graph per
+//                  pattern (plus one per step at which some unit stores its final
+//                  update), so that replay has no host branching per layer.
+// sgd_step         writes the per-step I/O slot and replays the step's graph
+//                  (Algorithm 2).  Inside a graph: stem, conditioning, then for every
+//                  unit in graph order either the active branch (norm -> projections
+//                  -> attention/MLP -> projection whose epilogue adds Delta to h and,
+//                  on the unit's last active step, stores it) or, for a maximal run of
+//                  consecutive frozen units, one frozen-run kernel; then the head.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <functional>
+#include <map>
+#include <memory>
+#include <string>
+#include <vector>
+
+#include "../../include/sgd.h"
+#include "kernels.h"
+
+using namespace sgd;
+
+namespace {
+
+thread_local std::string g_err;
+
+int fail(int code, const std::string& msg) {
+  g_err = msg;
+  return code;
+}
+
+#define CUDA_TRY(expr)                                                                   \
+  do {                                                                                   \
+    cudaError_t e_ = (expr);                                                             \
+    if (e_ != cudaSuccess)                                                               \
+      return fail(SGD_ERR_CUDA, std::string(#expr) + ": " + cudaGetErrorString(e_));     \
+  } while (0)
+
+struct Op {
+  std::string name;
+  int kernel;
+  double flops;
+  double bytes;
+  std::function<cudaError_t(cudaStream_t)> run;
+};
+
+bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int validate_schedule(int T, int n_units, const int32_t* S, const int32_t* groups,
+                      int expected_units) {
+  if (T < 1) return fail(SGD_ERR_SCHEDULE, "T must be >= 1");
+  if (!S || !groups) return fail(SGD_ERR_ARG, "null lifetimes or groups");
+  if (expected_units >= 0 && n_units != expected_units)
+    return fail(SGD_ERR_SCHEDULE, "n_units " + std::to_string(n_units) + " != model units " +
+                                      std::to_string(expected_units));
+  if (n_units < 1) return fail(SGD_ERR_SCHEDULE, "n_units must be >= 1");
+  std::map<int32_t, int32_t> life_of_group;
+  for (int u = 0; u < n_units; ++u) {
+    if (S[u] < 1 || S[u] > T)
+      return fail(SGD_ERR_SCHEDULE, "lifetime of unit " + std::to_string(u) + " = " +
+                                        std::to_string(S[u]) + " outside [1, T]");
+    auto it = life_of_group.find(groups[u]);
+    if (it == life_of_group.end())
+      life_of_group[groups[u]] = S[u];
+    else if (it->second != S[u])
+      return fail(SGD_ERR_SCHEDULE, "atomic group " + std::to_string(groups[u]) +
+                                        " is split: its members have different lifetimes");
+  }
+  return SGD_OK;
+}
+
+// pattern ids in order of first appearance; writes = units whose lifetime ends at s < T
+void compile_patterns(int T, int n_units, const int32_t* S, std::vector<int>& pattern_of_step,
+                      std::vector<int>& writes, std::vector<std::vector<uint8_t>>& patterns) {
+  pattern_of_step.assign(T, 0);
+  writes.assign(T, 0);
+  patterns.clear();
+  std::map<std::vector<uint8_t>, int> ids;
+  for (int s = 1; s <= T; ++s) {
+    std::vector<uint8_t> m(n_units);
+    for (int u = 0; u < n_units; ++u) {
+      m[u] = S[u] >= s ? 1 : 0;
+      if (S[u] == s && s < T) writes[s - 1]++;
+    }
+    auto it = ids.find(m);
+    if (it == ids.end()) {
+      const int id = static_cast<int>(patterns.size());
+      ids[m] = id;
+      patterns.push_back(m);
+      pattern_of_step[s - 1] = id;
+    } else {
+      pattern_of_step[s - 1] = it->second;
+    }
+  }
+}
+
+}  // namespace
+
+struct sgd_ctx {
+  sgd_model_desc d{};
+  std::vector<sgd_block_weights> blk;
+  std::vector<const bf16*> skip_w;
+  sgd_weights w{};
+  int device = 0;
+  int M = 0, U = 0, nbr = 0;
+  // buffers
+  float* h = nullptr;
+  bf16* xn = nullptr;
+  bf16* qkv = nullptr;
+  bf16* attn = nullptr;
+  bf16* act = nullptr;
+  float* t_hidden = nullptr;
+  float* cond_c = nullptr;
+  float* mod = nullptr;
+  float* modf = nullptr;
+  float* rope_cos = nullptr;
+  float* rope_sin = nullptr;
+  IoSlot* slot = nullptr;
+  std::vector<bf16*> cache;
+  std::vector<bf16*> ctxkv;
+  std::vector<bf16*> skipcat;
+  std::vector<void*> allocs;
+  size_t cache_bytes = 0, ws_bytes = 0;
+  // schedule
+  int T = 0;
+  std::vector<int32_t> S, groups;
+  std::vector<int> pattern_of_step, writes;
+  std::vector<std::vector<uint8_t>> patterns;
+  std::vector<int> graph_of_step;
+  std::vector<std::vector<Op>> programs;
+  std::vector<cudaGraph_t> graphs;
+  std::vector<cudaGraphExec_t> execs;
+  cudaStream_t cap_stream = nullptr;
+  int last_step = 0;
+  bool scheduled = false;
+  // host-buffer step staging
+  void* st_in = nullptr;
+  void* st_out = nullptr;
+  int32_t* st_cls = nullptr;
+  void* st_ctx = nullptr;
+
+  ~sgd_ctx() {
+    for (auto e : execs) cudaGraphExecDestroy(e);
+    for (auto g : graphs) cudaGraphDestroy(g);
+    if (cap_stream) cudaStreamDestroy(cap_stream);
+    for (void* p : allocs) cudaFree(p);
+  }
+
+  template <typename T_>
+  int alloc(T_** p, size_t count, size_t* acct) {
+    void* q = nullptr;
+    const size_t bytes = std::max<size_t>(count * sizeof(T_), 16);
+    cudaError_t e = cudaMalloc(&q, bytes);
+    if (e != cudaSuccess)
+      return fail(e == cudaErrorMemoryAllocation ? SGD_ERR_OOM : SGD_ERR_CUDA,
+                  std::string("cudaMalloc: ") + cudaGetErrorString(e));
+    allocs.push_back(q);
+    if (acct) *acct += bytes;
+    *p = static_cast<T_*>(q);
+    return SGD_OK;
+  }
+
+  size_t in_bytes() const {
+    if (d.stem == SGD_STEM_EMBED) return static_cast<size_t>(M) * 4;
+    return static_cast<size_t>(d.batch) * (d.n_tokens - d.n_prefix) * d.d_in * 4;
+  }
+  size_t out_bytes() const {
+    if (d.head == SGD_HEAD_LOGITS) return static_cast<size_t>(M) * d.d_out * 2;
+    if (d.head == SGD_HEAD_IDENTITY) return static_cast<size_t>(M) * d.d * 4;
+    return static_cast<size_t>(d.batch) * (d.n_tokens - d.n_prefix) * d.out_channels * 4;
+  }
+};
+
+namespace {
+
+const bf16* B16(const void* p) { return static_cast<const bf16*>(p); }
+
+// ---------------------------------------------------------------------------
+// op builders
+// ---------------------------------------------------------------------------
+
+int make_gemm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, const bf16* A,
+                 int lda, const bf16* B, int ldb, int M, int N, int K, const EpiParams& epi) {
+  auto plan = std::make_shared<GemmPlan>();
+  plan->A = A;
+  plan->lda = lda;
+  plan->B = B;
+  plan->ldb = ldb;
+  plan->M = M;
+  plan->N = N;
+  plan->K = K;
+  plan->epi = epi;
+  plan->simt = (c->d.flags & SGD_FLAG_SIMT_GEMM) != 0;
+  const char* why = "";
+  if (gemm_plan(*plan, &why) != 0) return fail(SGD_ERR_SHAPE, std::string(name) + ": " + why);
+  const bool gated = epi.kind == SGD_EPI_GATED;
+  const double nb = gated ? 2.0 * N : N;
+  double out_b;
+  switch (epi.kind) {
+    case SGD_EPI_F32: out_b = 4.0 * M * N; break;
+    case SGD_EPI_DELTA: out_b = 8.0 * M * N + (epi.cache ? 2.0 * M * N : 0.0); break;
+    default: out_b = 2.0 * M * N; break;
+  }
+  Op op;
+  op.name = name;
+  op.kernel = plan->simt ? SGD_KERNEL_GEMM_SIMT : SGD_KERNEL_GEMM_TC;
+  op.flops = 2.0 * M * nb * K;
+  op.bytes = 2.0 * M * K + 2.0 * nb * K + out_b;
+  op.run = [plan](cudaStream_t s) { return gemm_launch(*plan, s); };
+  ops.push_back(std::move(op));
+  return SGD_OK;
+}
+
+EpiParams epi_base(int kind) {
+  EpiParams e{};
+  e.kind = kind;
+  e.rows_per_batch = 1;
+  return e;
+}
+
+void make_norm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, int kind,
+                  const void* g, const void* b, const float* shift, const float* scale, int ld_mod) {
+  NormParams p{};
+  p.h = c->h;
+  p.out = c->xn;
+  p.rows = c->M;
+  p.d = c->d.d;
+  p.kind = kind;
+  p.g = B16(g);
+  p.b = B16(b);
+  p.shift = shift;
+  p.scale = scale;
+  p.ld_mod = ld_mod;
+  p.rows_per_batch = c->d.n_tokens;
+  p.eps = c->d.eps;
+  Op op;
+  op.name = name;
+  op.kernel = SGD_KERNEL_NORM;
+  op.flops = 0;
+  op.bytes = 6.0 * c->M * c->d.d;
+  op.run = [p](cudaStream_t s) { return norm_launch(p, s); };
+  ops.push_back(std::move(op));
+}
+
+int make_attn_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, const AttnParams& p) {
+  const char* why = "";
+  if (attn_check(p, &why) != 0) return fail(SGD_ERR_SHAPE, name + ": " + why);
+  Op op;
+  op.name = name;
+  op.kernel = SGD_KERNEL_ATTENTION;
+  const double dm = static_cast<double>(p.n_heads) * p.d_head;
+  op.flops = 4.0 * p.batch * p.n_heads * static_cast<double>(p.n_q) * p.n_kv * p.d_head;
+  op.bytes = 2.0 * p.batch * (2.0 * p.n_q * dm + 2.0 * p.n_kv * dm);
+  op.run = [p](cudaStream_t s) { return attn_launch(p, s); };
+  ops.push_back(std::move(op));
+  return SGD_OK;
+}
+
+void make_gemv_op(std::vector<Op>& ops, const std::string& name, const GemvParams& p) {
+  Op op;
+  op.name = name;
+  op.kernel = SGD_KERNEL_SMALL;
+  op.flops = 2.0 * p.rows * p.N * p.K;
+  op.bytes = 2.0 * p.N * p.K + 4.0 * p.rows * (p.N + p.K);
+  op.run = [p](cudaStream_t s) { return gemv_launch(p, s); };
+  ops.push_back(std::move(op));
+}
+
+void flush_run(sgd_ctx* c, std::vector<Op>& ops, std::vector<const bf16*>& run, int first_unit) {
+  size_t i = 0;
+  while (i < run.size()) {
+    FrozenParams p{};
+    p.h = c->h;
+    p.n = static_cast<int64_t>(c->M) * c->d.d;
+    p.n_caches = 0;
+    while (i < run.size() && p.n_caches < kMaxRun) p.caches[p.n_caches++] = run[i++];
+    Op op;
+    op.name = "frozen_run(u" + std::to_string(first_unit) + "+" + std::to_string(p.n_caches) + ")";
+    op.kernel = SGD_KERNEL_FROZEN_RUN;
+    op.flops = static_cast<double>(p.n) * p.n_caches;
+    op.bytes = static_cast<double>(p.n) * (8.0 + 2.0 * p.n_caches);
+    op.run = [p](cudaStream_t s) { return frozen_launch(p, s); };
+    ops.push_back(std::move(op));
+  }
+  run.clear();
+}
+
+int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_cache, int u) {
+  const sgd_model_desc& d = c->d;
+  const sgd_block_weights& W = c->blk[b];
+  const int M = c->M, D = d.d, F = d.d_ff;
+  const std::string pre = "b" + std::to_string(b) + ".";
+  const bool adaln = d.block == SGD_BLOCK_ADALN;
+  float* mod = adaln ? c->mod + static_cast<size_t>(b) * d.batch * 6 * D : nullptr;
+  bf16* cache = write_cache ? c->cache[u] : nullptr;
+  EpiParams delta = epi_base(SGD_EPI_DELTA);
+  delta.h = c->h;
+  delta.ldh = D;
+  delta.cache = cache;
+  delta.ld_cache = D;
+  int rc;
+  if (kind == 0) {  // self-attention
+    make_norm_op(c, ops, pre + "attn.norm", d.norm, W.norm1_w, W.norm1_b, adaln ? mod : nullptr,
+                 adaln ? mod + D : nullptr, 6 * D);
+    EpiParams e = epi_base(d.rope ? SGD_EPI_ROPE : SGD_EPI_BF16);
+    e.out = c->qkv;
+    e.ldo = 3 * D;
+    if (d.rope) {
+      e.rope_cos = c->rope_cos;
+      e.rope_sin = c->rope_sin;
+      e.rope_tokens = d.n_tokens;
+      e.d_head = d.d_head;
+      e.rope_cols = 2 * D;
+    }
+    if ((rc = make_gemm_op(c, ops, pre + "attn.qkv", c->xn, D, B16(W.w_qkv), D, M, 3 * D, D, e)))
+      return rc;
+    AttnParams ap{c->qkv, 3 * D, c->qkv + D, c->qkv + 2 * D, 3 * D, c->attn, D,
+                  d.batch, d.n_tokens, d.n_tokens, d.n_heads, d.d_head};
+    if ((rc = make_attn_op(c, ops, pre + "attn.sdpa", ap))) return rc;
+    if (adaln) {
+      delta.gate = mod + 2 * D;
+      delta.ld_gate = 6 * D;
+      delta.rows_per_batch = d.n_tokens;
+    }
+    return make_gemm_op(c, ops, pre + "attn.out", c->attn, D, B16(W.w_o), D, M, D, D, delta);
+  }
+  if (kind == 1) {  // cross-attention
+    make_norm_op(c, ops, pre + "xattn.norm", SGD_NORM_LN, W.normx_w, W.normx_b, nullptr, nullptr, 0);
+    EpiParams e = epi_base(SGD_EPI_BF16);
+    e.out = c->qkv;
+    e.ldo = D;
+    if ((rc = make_gemm_op(c, ops, pre + "xattn.q", c->xn, D, B16(W.wx_q), D, M, D, D, e))) return rc;
+    AttnParams ap{c->qkv, D, c->ctxkv[b], c->ctxkv[b] + D, 2 * D, c->attn, D,
+                  d.batch, d.n_tokens, d.ctx_len, d.n_heads, d.d_head};
+    if ((rc = make_attn_op(c, ops, pre + "xattn.sdpa", ap))) return rc;
+    return make_gemm_op(c, ops, pre + "xattn.out", c->attn, D, B16(W.wx_o), D, M, D, D, delta);
+  }
+  // MLP
+  make_norm_op(c, ops, pre + "mlp.norm", d.norm, W.norm2_w, W.norm2_b, adaln ? mod + 3 * D : nullptr,
+               adaln ? mod + 4 * D : nullptr, 6 * D);
+  const bool gated = d.mlp == SGD_MLP_SWIGLU || d.mlp == SGD_MLP_GEGLU;
+  EpiParams e = epi_base(gated ? SGD_EPI_GATED : SGD_EPI_GELU);
+  e.out = c->act;
+  e.ldo = F;
+  e.act = (d.mlp == SGD_MLP_GEGLU || d.mlp == SGD_MLP_GELU_ERF) ? 1 : 0;
+  if ((rc = make_gemm_op(c, ops, pre + "mlp.up", c->xn, D, B16(W.w_1), D, M, F, D, e))) return rc;
+  if (adaln) {
+    delta.gate = mod + 5 * D;
+    delta.ld_gate = 6 * D;
+    delta.rows_per_batch = d.n_tokens;
+  }
+  return make_gemm_op(c, ops, pre + "mlp.down", c->act, F, B16(W.w_2), F, M, D, F, delta);
+}
+
+int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vector<uint8_t>& write,
+                  std::vector<Op>& ops) {
+  const sgd_model_desc& d = c->d;
+  const int M = c->M, D = d.d;
+  ops.clear();
+  int rc;
+  {  // stem
+    StemParams p{};
+    p.kind = d.stem;
+    p.slot = c->slot;
+    p.h = c->h;
+    p.batch = d.batch;
+    p.n_tokens = d.n_tokens;
+    p.n_prefix = d.n_prefix;
+    p.d = D;
+    p.d_in = d.d_in;
+    p.w_stem = B16(c->w.w_stem);
+    p.pos = B16(c->w.pos_emb);
+    p.class_emb = B16(c->w.class_emb);
+    p.embed = B16(c->w.embed);
+    Op op;
+    op.name = "stem";
+    op.kernel = SGD_KERNEL_SMALL;
+    op.flops = 2.0 * M * D * std::max(d.d_in, 1);
+    op.bytes = 4.0 * M * D + static_cast<double>(c->in_bytes()) +
+               (d.stem == SGD_STEM_EMBED ? 2.0 * M * D : 0.0);
+    op.run = [p](cudaStream_t s) { return stem_launch(p, s); };
+    ops.push_back(std::move(op));
+  }
+  if (d.block == SGD_BLOCK_ADALN) {  // conditioning: c = W_t2 silu(W_t1 sin(t)) + class_emb[y]
+    GemvParams g{};
+    g.out = c->t_hidden;
+    g.ldo = D;
+    g.x_sinusoid = 1;
+    g.slot = c->slot;
+    g.W = B16(c->w.w_t1);
+    g.N = D;
+    g.K = d.t_freq;
+    g.rows = 1;
+    make_gemv_op(ops, "cond.t1", g);
+    GemvParams g2{};
+    g2.out = c->cond_c;
+    g2.ldo = D;
+    g2.x = c->t_hidden;
+    g2.ldx = 0;
+    g2.slot = c->slot;
+    g2.in_silu = 1;
+    g2.W = B16(c->w.w_t2);
+    g2.N = D;
+    g2.K = D;
+    g2.rows = d.batch;
+    g2.add_class = B16(c->w.class_emb);
+    make_gemv_op(ops, "cond.t2", g2);
+    for (int b = 0; b < d.n_blocks; ++b) {
+      bool any = false;
+      for (int k = 0; k < c->nbr; ++k) any = any || active[b * c->nbr + k];
+      if (!any) continue;  // modulation only for active blocks
+      GemvParams gm{};
+      gm.out = c->mod + static_cast<size_t>(b) * d.batch * 6 * D;
+      gm.ldo = 6 * D;
+      gm.x = c->cond_c;
+      gm.ldx = D;
+      gm.slot = c->slot;
+      gm.in_silu = 1;
+      gm.W = B16(c->blk[b].w_mod);
+      gm.N = 6 * D;
+      gm.K = D;
+      gm.rows = d.batch;
+      make_gemv_op(ops, "b" + std::to_string(b) + ".mod", gm);
+    }
+  }
+  std::vector<const bf16*> run;
+  int run_first = 0;
+  int u = 0;
+  for (int b = 0; b < d.n_blocks; ++b) {
+    if (d.n_skips && b > d.n_skips) {  // U-ViT deep block: h = W_skip [h; skip]
+      flush_run(c, ops, run, run_first);
+      const int j = b - d.n_skips - 1;
+      bf16* cat = c->skipcat[j];
+      const float* hh = c->h;
+      const int Mr = M;
+      Op op;
+      op.name = "b" + std::to_string(b) + ".skip_pack";
+      op.kernel = SGD_KERNEL_SMALL;
+      op.flops = 0;
+      op.bytes = 6.0 * M * D;
+      op.run = [cat, hh, Mr, D](cudaStream_t s) { return pack_bf16_launch(cat, 2 * D, 0, hh, Mr, D, s); };
+      ops.push_back(std::move(op));
+      EpiParams e = epi_base(SGD_EPI_F32);
+      e.out = c->h;
+      e.ldo = D;
+      if ((rc = make_gemm_op(c, ops, "b" + std::to_string(b) + ".skip_linear", cat, 2 * D,
+                             c->skip_w[j], 2 * D, M, D, 2 * D, e)))
+        return rc;
+    }
+    for (int k = 0; k < c->nbr; ++k, ++u) {
+      const int kind = d.block == SGD_BLOCK_XATTN ? k : (k == 0 ? 0 : 2);
+      if (active[u]) {
+        flush_run(c, ops, run, run_first);
+        if ((rc = build_branch(c, ops, b, kind, write[u] != 0, u))) return rc;
+      } else {
+        if (run.empty()) run_first = u;
+        run.push_back(c->cache[u]);
+      }
+    }
+    if (d.n_skips && b < d.n_skips) {  // U-ViT shallow block: push the current h
+      flush_run(c, ops, run, run_first);
+      bf16* cat = c->skipcat[d.n_skips - 1 - b];
+      const float* hh = c->h;
+      const int Mr = M;
+      Op op;
+      op.name = "b" + std::to_string(b) + ".skip_push";
+      op.kernel = SGD_KERNEL_SMALL;
+      op.flops = 0;
+      op.bytes = 6.0 * M * D;
+      op.run = [cat, hh, Mr, D](cudaStream_t s) { return pack_bf16_launch(cat, 2 * D, D, hh, Mr, D, s); };
+      ops.push_back(std::move(op));
+    }
+  }
+  flush_run(c, ops, run, run_first);
+  // head
+  void* const* out_slot = reinterpret_cast<void* const*>(&c->slot->out);
+  if (d.head == SGD_HEAD_IDENTITY) {
+    const IoSlot* slot = c->slot;
+    const float* hh = c->h;
+    const int64_t n = static_cast<int64_t>(M) * D;
+    Op op;
+    op.name = "head.copy";
+    op.kernel = SGD_KERNEL_SMALL;
+    op.flops = 0;
+    op.bytes = 8.0 * n;
+    op.run = [slot, hh, n](cudaStream_t s) { return copy_out_launch(slot, hh, n, s); };
+    ops.push_back(std::move(op));
+    return SGD_OK;
+  }
+  if (d.head == SGD_HEAD_ADALN_LINEAR) {
+    GemvParams g{};
+    g.out = c->modf;
+    g.ldo = 2 * D;
+    g.x = c->cond_c;
+    g.ldx = D;
+    g.slot = c->slot;
+    g.in_silu = 1;
+    g.W = B16(c->w.w_modf);
+    g.N = 2 * D;
+    g.K = D;
+    g.rows = d.batch;
+    make_gemv_op(ops, "head.mod", g);
+    make_norm_op(c, ops, "head.norm", SGD_NORM_LN_PLAIN, nullptr, nullptr, c->modf, c->modf + D, 2 * D);
+  } else {
+    make_norm_op(c, ops, "head.norm", d.norm == SGD_NORM_RMS ? SGD_NORM_RMS : SGD_NORM_LN,
+                 c->w.normf_w, c->w.normf_b, nullptr, nullptr, 0);
+  }
+  if (d.d_out <= 64 && d.head != SGD_HEAD_LOGITS) {
+    HeadParams hp{};
+    hp.x = c->xn;
+    hp.ldx = D;
+    hp.W = B16(c->w.w_head);
+    hp.N = d.d_out;
+    hp.K = D;
+    hp.batch = d.batch;
+    hp.n_tokens = d.n_tokens;
+    hp.n_prefix = d.n_prefix;
+    hp.out_channels = d.out_channels;
+    hp.slot = c->slot;
+    Op op;
+    op.name = "head.linear";
+    op.kernel = SGD_KERNEL_SMALL;
+    op.flops = 2.0 * M * d.out_channels * D;
+    op.bytes = 2.0 * M * D + 4.0 * M * d.out_channels;
+    op.run = [hp](cudaStream_t s) { return head_small_launch(hp, s); };
+    ops.push_back(std::move(op));
+    return SGD_OK;
+  }
+  EpiParams e = epi_base(d.head == SGD_HEAD_LOGITS ? SGD_EPI_BF16 : SGD_EPI_F32);
+  e.out_slot = out_slot;
+  e.ldo = d.head == SGD_HEAD_LOGITS ? d.d_out : d.out_channels;
+  return make_gemm_op(c, ops, "head.linear", c->xn, D, B16(c->w.w_head), D, M, d.d_out, D, e);
+}
+
+int run_ops(const std::vector<Op>& ops, cudaStream_t s) {
+  for (const Op& op : ops) {
+    cudaError_t e = op.run(s);
+    if (e != cudaSuccess) return fail(SGD_ERR_CUDA, op.name + ": " + cudaGetErrorString(e));
+  }
+  return SGD_OK;
+}
+
+int check_shape(const sgd_model_desc& d, const sgd_weights& w) {
+  auto bad = [](const std::string& m) { return fail(SGD_ERR_SHAPE, m); };
+  if (d.n_blocks < 1 || d.n_blocks > 64) return bad("n_blocks must be in [1, 64]");
+  if (d.d_head != 64 && d.d_head != 72 && d.d_head != 128) return bad("d_head must be 64, 72 or 128");
+  if (d.n_heads * d.d_head != d.d) return bad("d must equal n_heads * d_head");
+  if (d.d % 8 || d.d > 4096) return bad("d must be a multiple of 8 and at most 4096");
+  if (d.d_ff < 8 || d.d_ff % 8) return bad("d_ff must be a positive multiple of 8");
+  if (d.batch < 1 || d.n_tokens < 1 || d.batch * d.n_heads > 65535) return bad("bad batch / tokens");
+  if (d.rope && d.d_head == 72) return bad("RoPE needs d_head 64 or 128");
+  if (d.eps <= 0.f) return bad("eps must be > 0");
+  if (d.stem < 0 || d.stem > 4 || d.block < 0 || d.block > 2 || d.norm < 0 || d.norm > 2 ||
+      d.mlp < 0 || d.mlp > 3 || d.head < 0 || d.head > 3)
+    return fail(SGD_ERR_ARG, "enum out of range");
+  switch (d.stem) {
+    case SGD_STEM_TIME_ADD:
+    case SGD_STEM_IDENTITY:
+      if (d.d_in != d.d || d.n_prefix) return bad("time_add / identity stems need d_in == d, no prefix");
+      break;
+    case SGD_STEM_PATCH:
+      if (d.d_in < 1 || d.n_prefix || !w.w_stem || !w.pos_emb) return bad("patch stem needs w_stem, pos_emb");
+      break;
+    case SGD_STEM_PATCH_TOKENS:
+      if (d.d_in < 1 || d.n_prefix != 2 || !w.w_stem || !w.pos_emb || !w.class_emb || d.n_classes < 1)
+        return bad("patch-token stem needs n_prefix 2, w_stem, pos_emb, class_emb");
+      break;
+    case SGD_STEM_EMBED:
+      if (d.vocab < 1 || !w.embed || d.n_prefix) return bad("embed stem needs vocab and embed");
+      break;
+  }
+  if (d.block == SGD_BLOCK_ADALN) {
+    if (!w.w_t1 || !w.w_t2 || !w.class_emb || d.t_freq < 8 || d.t_freq % 8 || d.batch > 16 ||
+        d.norm != SGD_NORM_LN_PLAIN)
+      return bad("AdaLN blocks need w_t1, w_t2, class_emb, t_freq % 8 == 0, batch <= 16, LN_PLAIN");
+  }
+  if (d.block == SGD_BLOCK_XATTN && (d.ctx_len < 1 || d.d_ctx < 8 || d.d_ctx % 8))
+    return bad("cross-attention needs ctx_len >= 1 and d_ctx a multiple of 8");
+  if (d.n_skips && (d.n_blocks != 2 * d.n_skips + 1 || !w.skip_w))
+    return bad("long skips need n_blocks = 2 n_skips + 1 and skip weights");
+  switch (d.head) {
+    case SGD_HEAD_LINEAR:
+      if (!w.w_head || !w.normf_w) return bad("linear head needs normf_w and w_head");
+      if (d.d_out > 64 && (d.n_prefix || d.out_channels != d.d_out || d.d_out % 8))
+        return bad("wide linear head needs out_channels == d_out (multiple of 8) and no prefix");
+      if (d.out_channels > d.d_out) return bad("out_channels > d_out");
+      break;
+    case SGD_HEAD_ADALN_LINEAR:
+      if (d.block != SGD_BLOCK_ADALN || !w.w_modf || !w.w_head || d.d_out > 64 ||
+          d.out_channels > d.d_out)
+        return bad("AdaLN head needs AdaLN blocks, w_modf, w_head, d_out <= 64");
+      break;
+    case SGD_HEAD_IDENTITY:
+      if (d.n_prefix || d.out_channels != d.d) return bad("identity head needs out_channels == d");
+      break;
+    case SGD_HEAD_LOGITS:
+      if (!w.w_head || !w.normf_w || d.d_out % 8 || d.d_out < 8) return bad("logits head needs normf_w, w_head, d_out % 8 == 0");
+      break;
+  }
+  if (!w.blocks) return fail(SGD_ERR_ARG, "null block weights");
+  for (int b = 0; b < d.n_blocks; ++b) {
+    const sgd_block_weights& W = w.blocks[b];
+    const void* need[] = {W.w_qkv, W.w_o, W.w_1, W.w_2};
+    for (const void* p : need)
+      if (!p || !al16(p)) return fail(SGD_ERR_ARG, "block " + std::to_string(b) + ": missing or misaligned weight");
+    if (d.norm != SGD_NORM_LN_PLAIN && (!W.norm1_w || !W.norm2_w))
+      return fail(SGD_ERR_ARG, "block " + std::to_string(b) + ": missing norm gains");
+    if (d.norm == SGD_NORM_LN && (!W.norm1_b || !W.norm2_b))
+      return fail(SGD_ERR_ARG, "block " + std::to_string(b) + ": missing norm shifts");
+    if (d.block == SGD_BLOCK_ADALN && (!W.w_mod || !al16(W.w_mod)))
+      return fail(SGD_ERR_ARG, "block " + std::to_string(b) + ": missing w_mod");
+    if (d.block == SGD_BLOCK_XATTN &&
+        (!W.wx_q || !W.wx_kv || !W.wx_o || !W.normx_w || !W.normx_b || !al16(W.wx_kv)))
+      return fail(SGD_ERR_ARG, "block " + std::to_string(b) + ": missing cross-attention weights");
+  }
+  return SGD_OK;
+}
+
+int ensure_alloc(sgd_ctx* c) {
+  const sgd_model_desc& d = c->d;
+  const size_t M = c->M, D = d.d, F = d.d_ff;
+  int rc;
+  if ((rc = c->alloc(&c->h, M * D, &c->ws_bytes))) return rc;
+  if ((rc = c->alloc(&c->xn, M * D, &c->ws_bytes))) return rc;
+  if ((rc = c->alloc(&c->qkv, M * 3 * D, &c->ws_bytes))) return rc;
+  if ((rc = c->alloc(&c->attn, M * D, &c->ws_bytes))) return rc;
+  if ((rc = c->alloc(&c->act, M * F, &c->ws_bytes))) return rc;
+  if ((rc = c->alloc(&c->slot, 1, &c->ws_bytes))) return rc;
+  CUDA_TRY(cudaMemset(c->slot, 0, sizeof(IoSlot)));
+  if (d.block == SGD_BLOCK_ADALN) {
+    if ((rc = c->alloc(&c->t_hidden, D, &c->ws_bytes))) return rc;
+    if ((rc = c->alloc(&c->cond_c, d.batch * D, &c->ws_bytes))) return rc;
+    if ((rc = c->alloc(&c->mod, static_cast<size_t>(d.n_blocks) * d.batch * 6 * D, &c->ws_bytes))) return rc;
+    if ((rc = c->alloc(&c->modf, d.batch * 2 * D, &c->ws_bytes))) return rc;
+  }
+  if (d.block == SGD_BLOCK_XATTN) {
+    c->ctxkv.assign(d.n_blocks, nullptr);
+    for (int b = 0; b < d.n_blocks; ++b)
+      if ((rc = c->alloc(&c->ctxkv[b], static_cast<size_t>(d.batch) * d.ctx_len * 2 * D, &c->ws_bytes))) return rc;
+  }
+  if (d.n_skips) {
+    c->skipcat.assign(d.n_skips, nullptr);
+    for (int j = 0; j < d.n_skips; ++j)
+      if ((rc = c->alloc(&c->skipcat[j], M * 2 * D, &c->ws_bytes))) return rc;
+  }
+  if (d.rope) {
+    const int half = d.d_head / 2;
+    std::vector<float> cs(static_cast<size_t>(d.n_tokens) * half), sn(cs.size());
+    for (int p = 0; p < d.n_tokens; ++p)
+      for (int i = 0; i < half; ++i) {
+        const double f = std::pow(static_cast<double>(d.rope_theta), -2.0 * i / d.d_head);
+        cs[static_cast<size_t>(p) * half + i] = static_cast<float>(std::cos(p * f));
+        sn[static_cast<size_t>(p) * half + i] = static_cast<float>(std::sin(p * f));
+      }
+    if ((rc = c->alloc(&c->rope_cos, cs.size(), &c->ws_bytes))) return rc;
+    if ((rc = c->alloc(&c->rope_sin, sn.size(), &c->ws_bytes))) return rc;
+    CUDA_TRY(cudaMemcpy(c->rope_cos, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice));
+    CUDA_TRY(cudaMemcpy(c->rope_sin, sn.data(), sn.size() * 4, cudaMemcpyHostToDevice));
+  }
+  c->cache.assign(c->U, nullptr);
+  return SGD_OK;
+}
+
+void drop_graphs(sgd_ctx* c) {
+  for (auto e : c->execs) cudaGraphExecDestroy(e);
+  for (auto g : c->graphs) cudaGraphDestroy(g);
+  c->execs.clear();
+  c->graphs.clear();
+  c->programs.clear();
+  c->scheduled = false;
+}
+
+// Cross-attention K/V of the (constant) context, projected at step 1 of a trajectory.
+int ctx_kv_ops(sgd_ctx* c, const void* ctx_dev, std::vector<Op>& ops) {
+  const sgd_model_desc& d = c->d;
+  ops.clear();
+  for (int b = 0; b < d.n_blocks; ++b) {
+    EpiParams e = epi_base(SGD_EPI_BF16);
+    e.out = c->ctxkv[b];
+    e.ldo = 2 * d.d;
+    int rc = make_gemm_op(c, ops, "b" + std::to_string(b) + ".xattn.ctx_kv", B16(ctx_dev), d.d_ctx,
+                          B16(c->blk[b].wx_kv), d.d_ctx, d.batch * d.ctx_len, 2 * d.d, d.d_ctx, e);
+    if (rc) return rc;
+  }
+  return SGD_OK;
+}
+
+int check_step_args(sgd_ctx* c, const void* in, void* out, const sgd_cond* cond, int step) {
+  if (!c) return fail(SGD_ERR_ARG, "null context");
+  if (!c->scheduled) return fail(SGD_ERR_STATE, "no schedule installed");
+  if (!in || !out) return fail(SGD_ERR_ARG, "null state or output");
+  if (step < 1 || step > c->T) return fail(SGD_ERR_ARG, "step outside [1, T]");
+  if (step != 1 && step != c->last_step + 1)
+    return fail(SGD_ERR_CACHE_INVALID, "step " + std::to_string(step) + " after step " +
+                                           std::to_string(c->last_step) +
+                                           ": caches need steps 1..s-1 since the last reset");
+  if ((c->d.n_classes && c->d.block == SGD_BLOCK_ADALN) || c->d.stem == SGD_STEM_PATCH_TOKENS) {
+    if (!cond || !cond->class_ids) return fail(SGD_ERR_ARG, "model needs class ids");
+  }
+  if (c->d.block == SGD_BLOCK_XATTN && step == 1 && (!cond || !cond->ctx))
+    return fail(SGD_ERR_ARG, "cross-attention model needs a context at step 1");
+  if (!al16(in) || !al16(out)) return fail(SGD_ERR_ARG, "state/output must be 16-byte aligned");
+  return SGD_OK;
+}
+
+int prepare_step(sgd_ctx* c, const void* in, void* out, float t, const sgd_cond* cond, int step,
+                 cudaStream_t s) {
+  IoSlot v{};
+  v.state = in;
+  v.out = out;
+  v.class_ids = cond ? cond->class_ids : nullptr;
+  v.ctx = cond ? cond->ctx : nullptr;
+  v.t = t;
+  v.step = step;
+  CUDA_TRY(io_set_launch(c->slot, v, s));
+  if (step == 1 && c->d.block == SGD_BLOCK_XATTN) {
+    std::vector<Op> ops;
+    int rc = ctx_kv_ops(c, cond->ctx, ops);
+    if (rc) return rc;
+    if ((rc = run_ops(ops, s))) return rc;
+  }
+  return SGD_OK;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// C ABI
+// ---------------------------------------------------------------------------
+
+extern "C" {
+
+const char* sgd_last_error(void) { return g_err.c_str(); }
+
+int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out) {
+  if (!desc || !w || !out) return fail(SGD_ERR_ARG, "null argument");
+  *out = nullptr;
+  int rc = check_shape(*desc, *w);
+  if (rc) return rc;
+  auto* c = new (std::nothrow) sgd_ctx();
+  if (!c) return fail(SGD_ERR_OOM, "host allocation failed");
+  c->d = *desc;
+  c->blk.assign(w->blocks, w->blocks + desc->n_blocks);
+  c->w = *w;
+  c->w.blocks = c->blk.data();
+  for (int j = 0; j < desc->n_skips; ++j) c->skip_w.push_back(B16(w->skip_w[j]));
+  c->w.skip_w = nullptr;
+  if (cudaGetDevice(&c->device) != cudaSuccess) {
+    delete c;
+    return fail(SGD_ERR_CUDA, "no CUDA device");
+  }
+  c->M = desc->batch * desc->n_tokens;
+  c->nbr = desc->block == SGD_BLOCK_XATTN ? 3 : 2;
+  c->U = desc->n_blocks * c->nbr;
+  if ((rc = ensure_alloc(c))) {
+    delete c;
+    return rc;
+  }
+  if (cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking) != cudaSuccess) {
+    delete c;
+    return fail(SGD_ERR_CUDA, "stream creation failed");
+  }
+  *out = c;
+  g_err.clear();
+  return SGD_OK;
+}
+
+int sgd_compile_schedule(int T, int n_units, const int32_t* lifetimes, const int32_t* groups,
+                         int32_t* pattern_of_step, int32_t* writes_at_step, int32_t* n_patterns) {
+  int rc = validate_schedule(T, n_units, lifetimes, groups, -1);
+  if (rc) return rc;
+  std::vector<int> pos, wr;
+  std::vector<std::vector<uint8_t>> pats;
+  compile_patterns(T, n_units, lifetimes, pos, wr, pats);
+  for (int s = 0; s < T; ++s) {
+    if (pattern_of_step) pattern_of_step[s] = pos[s];
+    if (writes_at_step) writes_at_step[s] = wr[s];
+  }
+  if (n_patterns) *n_patterns = static_cast<int32_t>(pats.size());
+  return SGD_OK;
+}
+
+int sgd_set_schedule(sgd_ctx* c, int T, int n_units, const int32_t* lifetimes, const int32_t* groups) {
+  if (!c) return fail(SGD_ERR_ARG, "null context");
+  int rc = validate_schedule(T, n_units, lifetimes, groups, c->U);
+  if (rc) return rc;
+  CUDA_TRY(cudaSetDevice(c->device));
+  drop_graphs(c);
+  c->T = T;
+  c->S.assign(lifetimes, lifetimes + n_units);
+  c->groups.assign(groups, groups + n_units);
+  compile_patterns(T, n_units, lifetimes, c->pattern_of_step, c->writes, c->patterns);
+  // caches only for units that are ever frozen
+  for (int u = 0; u < c->U; ++u)
+    if (c->S[u] < T && !c->cache[u]) {
+      if ((rc = c->alloc(&c->cache[u], static_cast<size_t>(c->M) * c->d.d, &c->cache_bytes))) return rc;
+    }
+  // graph variants: (pattern, cache-store set); the store set is non-empty only at steps
+  // s = S_u < T, so each such step gets its own variant.
+  std::map<std::pair<int, int>, int> key_to_graph;
+  c->graph_of_step.assign(T + 1, -1);
+  for (int s = 1; s <= T; ++s) {
+    const int pid = c->pattern_of_step[s - 1];
+    const int key2 = c->writes[s - 1] ? s : -1;
+    auto it = key_to_graph.find({pid, key2});
+    if (it != key_to_graph.end()) {
+      c->graph_of_step[s] = it->second;
+      continue;
+    }
+    std::vector<uint8_t> write(c->U, 0);
+    for (int u = 0; u < c->U; ++u) write[u] = (c->S[u] == s && s < T) ? 1 : 0;
+    std::vector<Op> ops;
+    if ((rc = build_program(c, c->patterns[pid], write, ops))) return rc;
+    cudaGraph_t g = nullptr;
+    CUDA_TRY(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeRelaxed));
+    rc = run_ops(ops, c->cap_stream);
+    cudaError_t ce = cudaStreamEndCapture(c->cap_stream, &g);
+    if (rc) {
+      if (g) cudaGraphDestroy(g);
+      return rc;
+    }
+    if (ce != cudaSuccess) return fail(SGD_ERR_CUDA, std::string("graph capture: ") + cudaGetErrorString(ce));
+    cudaGraphExec_t ex = nullptr;
+    ce = cudaGraphInstantiate(&ex, g, 0);
+    if (ce != cudaSuccess) {
+      cudaGraphDestroy(g);
+      return fail(SGD_ERR_CUDA, std::string("graph instantiate: ") + cudaGetErrorString(ce));
+    }
+    const int gid = static_cast<int>(c->graphs.size());
+    c->graphs.push_back(g);
+    c->execs.push_back(ex);
+    c->programs.push_back(std::move(ops));
+    key_to_graph[{pid, key2}] = gid;
+    c->graph_of_step[s] = gid;
+  }
+  c->last_step = 0;
+  c->scheduled = true;
+  g_err.clear();
+  return SGD_OK;
+}
+
+int sgd_step(sgd_ctx* c, const void* in, void* out, float t, const sgd_cond* cond, int step,
+             void* stream) {
+  int rc = check_step_args(c, in, out, cond, step);
+  if (rc) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((rc = prepare_step(c, in, out, t, cond, step, s))) return rc;
+  CUDA_TRY(cudaGraphLaunch(c->execs[c->graph_of_step[step]], s));
+  c->last_step = step == c->T ? 0 : step;
+  return SGD_OK;
+}
+
+int sgd_step_profile(sgd_ctx* c, const void* in, void* out, float t, const sgd_cond* cond, int step,
+                     void* stream, sgd_op_record* rec, int max_rec, int* n_rec) {
+  int rc = check_step_args(c, in, out, cond, step);
+  if (rc) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((rc = prepare_step(c, in, out, t, cond, step, s))) return rc;
+  const std::vector<Op>& ops = c->programs[c->graph_of_step[step]];
+  std::vector<cudaEvent_t> ev(2 * ops.size());
+  for (auto& e : ev) CUDA_TRY(cudaEventCreate(&e));
+  for (size_t i = 0; i < ops.size(); ++i) {
+    cudaEventRecord(ev[2 * i], s);
+    cudaError_t e = ops[i].run(s);
+    cudaEventRecord(ev[2 * i + 1], s);
+    if (e != cudaSuccess) {
+      for (auto& x : ev) cudaEventDestroy(x);
+      return fail(SGD_ERR_CUDA, ops[i].name + ": " + cudaGetErrorString(e));
+    }
+  }
+  cudaError_t se = cudaStreamSynchronize(s);
+  int n = 0;
+  for (size_t i = 0; i < ops.size() && static_cast<int>(i) < max_rec; ++i, ++n) {
+    float ms = 0.f;
+    cudaEventElapsedTime(&ms, ev[2 * i], ev[2 * i + 1]);
+    if (rec) {
+      memset(&rec[i], 0, sizeof(sgd_op_record));
+      strncpy(rec[i].name, ops[i].name.c_str(), sizeof(rec[i].name) - 1);
+      rec[i].kernel = ops[i].kernel;
+      rec[i].ms = ms;
+      rec[i].flops = ops[i].flops;
+      rec[i].bytes = ops[i].bytes;
+    }
+  }
+  for (auto& x : ev) cudaEventDestroy(x);
+  if (n_rec) *n_rec = n;
+  if (se != cudaSuccess) return fail(SGD_ERR_CUDA, std::string("profile sync: ") + cudaGetErrorString(se));
+  c->last_step = step == c->T ? 0 : step;
+  return SGD_OK;
+}
+
+int sgd_step_host(sgd_ctx* c, const void* in_host, void* out_host, float t, const int32_t* cls_host,
+                  const void* ctx_host, int step, void* stream) {
+  if (!c) return fail(SGD_ERR_ARG, "null context");
+  if (!in_host || !out_host) return fail(SGD_ERR_ARG, "null host buffer");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int rc;
+  if (!c->st_in && (rc = c->alloc(reinterpret_cast<uint8_t**>(&c->st_in), c->in_bytes(), &c->ws_bytes))) return rc;
+  if (!c->st_out && (rc = c->alloc(reinterpret_cast<uint8_t**>(&c->st_out), c->out_bytes(), &c->ws_bytes))) return rc;
+  sgd_cond cond{};
+  if (cls_host) {
+    if (!c->st_cls && (rc = c->alloc(&c->st_cls, c->d.batch, &c->ws_bytes))) return rc;
+    CUDA_TRY(cudaMemcpyAsync(c->st_cls, cls_host, c->d.batch * 4, cudaMemcpyHostToDevice, s));
+    cond.class_ids = c->st_cls;
+  }
+  if (ctx_host && step == 1) {
+    const size_t cb = static_cast<size_t>(c->d.batch) * c->d.ctx_len * c->d.d_ctx * 2;
+    if (!c->st_ctx && (rc = c->alloc(reinterpret_cast<uint8_t**>(&c->st_ctx), cb, &c->ws_bytes))) return rc;
+    CUDA_TRY(cudaMemcpyAsync(c->st_ctx, ctx_host, cb, cudaMemcpyHostToDevice, s));
+  }
+  if (ctx_host) cond.ctx = c->st_ctx;
+  CUDA_TRY(cudaMemcpyAsync(c->st_in, in_host, c->in_bytes(), cudaMemcpyHostToDevice, s));
+  if ((rc = sgd_step(c, c->st_in, c->st_out, t, &cond, step, stream))) return rc;
+  CUDA_TRY(cudaMemcpyAsync(out_host, c->st_out, c->out_bytes(), cudaMemcpyDeviceToHost, s));
+  CUDA_TRY(cudaStreamSynchronize(s));
+  return SGD_OK;
+}
+
+int sgd_get_active_mask(const sgd_ctx* c, int step, uint8_t* mask, int n_units) {
+  if (!c || !mask) return fail(SGD_ERR_ARG, "null argument");
+  if (!c->scheduled) return fail(SGD_ERR_STATE, "no schedule installed");
+  if (step < 1 || step > c->T) return fail(SGD_ERR_ARG, "step outside [1, T]");
+  if (n_units != c->U) return fail(SGD_ERR_ARG, "n_units mismatch");
+  const auto& m = c->patterns[c->pattern_of_step[step - 1]];
+  for (int u = 0; u < n_units; ++u) mask[u] = m[u];
+  return SGD_OK;
+}
+
+int sgd_get_info(const sgd_ctx* c, sgd_info* info) {
+  if (!c || !info) return fail(SGD_ERR_ARG, "null argument");
+  memset(info, 0, sizeof(*info));
+  info->n_units = c->U;
+  info->n_patterns = static_cast<int>(c->patterns.size());
+  info->n_graphs = static_cast<int>(c->graphs.size());
+  info->T = c->scheduled ? c->T : 0;
+  int64_t ls = 0;
+  if (c->scheduled)
+    for (int u = 0; u < c->U; ++u) ls += c->S[u];
+  info->layer_steps = ls;
+  info->cache_bytes = c->cache_bytes;
+  info->workspace_bytes = c->ws_bytes;
+  return SGD_OK;
+}
+
+int sgd_reset(sgd_ctx* c) {
+  if (!c) return fail(SGD_ERR_ARG, "null context");
+  c->last_step = 0;
+  return SGD_OK;
+}
+
+int sgd_check_device(sgd_ctx* c, void* stream) {
+  (void)c;
+  CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+  int st = 0;
+  int rc = sgd_kernel_status(&st);
+  if (rc) return rc;
+  if (st) return fail(SGD_ERR_DEVICE_TIMEOUT, "a kernel's bounded wait expired (code " + std::to_string(st) + ")");
+  return SGD_OK;
+}
+
+void sgd_destroy(sgd_ctx* c) { delete c; }
+
+int sgd_sampler_update(float* z, const float* eps, float alpha, float beta, int64_t n, void* stream) {
+  if (!z || !eps || n < 0) return fail(SGD_ERR_ARG, "bad sampler arguments");
+  CUDA_TRY(sampler_launch(z, eps, alpha, beta, n, static_cast<cudaStream_t>(stream)));
+  return SGD_OK;
+}
+
+// ----- kernel-level entry points (include/sgd_kernels.h) -----
+
+int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
+                    const sgd_epilogue_args* ea, int use_simt, void* stream) {
+  if (!ea) return fail(SGD_ERR_ARG, "null epilogue");
+  if (ea->kind < 0 || ea->kind > SGD_EPI_ROPE) return fail(SGD_ERR_ARG, "bad epilogue kind");
+  GemmPlan p;
+  p.A = B16(A);
+  p.lda = lda;
+  p.B = B16(B);
+  p.ldb = ldb;
+  p.M = M;
+  p.N = N;
+  p.K = K;
+  p.simt = use_simt != 0;
+  EpiParams& e = p.epi;
+  e = EpiParams{};
+  e.kind = ea->kind;
+  e.out = ea->out;
+  e.ldo = ea->ldo;
+  e.h = ea->h;
+  e.ldh = ea->ldh;
+  e.cache = static_cast<bf16*>(ea->cache);
+  e.ld_cache = ea->ld_cache;
+  e.gate = ea->gate;
+  e.ld_gate = ea->ld_gate;
+  e.rows_per_batch = ea->rows_per_batch > 0 ? ea->rows_per_batch : 1;
+  e.act = ea->act;
+  e.rope_cos = ea->rope_cos;
+  e.rope_sin = ea->rope_sin;
+  e.rope_tokens = ea->rope_tokens;
+  e.d_head = ea->d_head;
+  e.rope_cols = ea->rope_cols;
+  e.M = M;
+  e.N = N;
+  const char* why = "";
+  const int rc = gemm_plan(p, &why);
+  if (rc) return fail(rc == -5 ? SGD_ERR_CUDA : (rc == -1 ? SGD_ERR_ARG : SGD_ERR_SHAPE), why);
+  CUDA_TRY(gemm_launch(p, static_cast<cudaStream_t>(stream)));
+  return SGD_OK;
+}
+
+int sgd_kernel_attention(const void* q, int ldq, const void* k, const void* v, int ldkv, void* o,
+                         int ldo, int batch, int n_q, int n_kv, int n_heads, int d_head, void* stream) {
+  AttnParams p{B16(q), ldq, B16(k), B16(v), ldkv, static_cast<bf16*>(o), ldo,
+               batch, n_q, n_kv, n_heads, d_head};
+  const char* why = "";
+  const int rc = attn_check(p, &why);
+  if (rc) return fail(rc == -1 ? SGD_ERR_ARG : SGD_ERR_SHAPE, why);
+  CUDA_TRY(attn_launch(p, static_cast<cudaStream_t>(stream)));
+  return SGD_OK;
+}
+
+int sgd_kernel_norm(const float* h, void* out, int rows, int d, int kind, const void* g, const void* b,
+                    const float* shift, const float* scale, int ld_mod, int rows_per_batch, float eps,
+                    void* stream) {
+  if (!h || !out || rows < 1 || d < 4 || d % 4 || d > 4096 || kind < 0 || kind > 2)
+    return fail(SGD_ERR_ARG, "norm: bad arguments (d must be a multiple of 4, <= 4096)");
+  if ((shift == nullptr) != (scale == nullptr) || (shift && rows_per_batch < 1))
+    return fail(SGD_ERR_ARG, "norm: shift and scale go together, rows_per_batch >= 1");
+  NormParams p{h, static_cast<bf16*>(out), rows, d, kind, B16(g), B16(b), shift, scale, ld_mod,
+               rows_per_batch > 0 ? rows_per_batch : 1, eps};
+  CUDA_TRY(norm_launch(p, static_cast<cudaStream_t>(stream)));
+  return SGD_OK;
+}
+
+int sgd_kernel_frozen_run(float* h, const void* const* caches, int n_caches, int64_t n, void* stream) {
+  if (!h || !caches || n_caches < 1 || n_caches > kMaxRun || n < 0 || n % 8 || !al16(h))
+    return fail(SGD_ERR_ARG, "frozen_run: bad arguments");
+  FrozenParams p{};
+  p.h = h;
+  p.n = n;
+  p.n_caches = n_caches;
+  for (int i = 0; i < n_caches; ++i) {
+    if (!caches[i] || !al16(caches[i])) return fail(SGD_ERR_ARG, "frozen_run: null or misaligned cache");
+    p.caches[i] = B16(caches[i]);
+  }
+  CUDA_TRY(frozen_launch(p, static_cast<cudaStream_t>(stream)));
+  return SGD_OK;
+}
+
+int sgd_kernel_status(int* status_host) {
+  if (!status_host) return fail(SGD_ERR_ARG, "null argument");
+  int* p = device_status_ptr();
+  if (!p) return fail(SGD_ERR_CUDA, "status word unavailable");
+  CUDA_TRY(cudaMemcpy(status_host, p, sizeof(int), cudaMemcpyDeviceToHost));
+  if (*status_host) CUDA_TRY(cudaMemset(p, 0, sizeof(int)));
+  return SGD_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,362 @@
+// Bandwidth-bound kernels of the scheduled step:
+//   frozen_run   — Algorithm 2, frozen branch: h_{l,s} = h_{l-1,s} + Delta_{l, r_l(s)}
+//                  for a run of consecutive frozen units in one read-modify-write of h
+//                  (16-byte vectors: 8 fp32 of h, 8 bf16 of each cached update).
+//   norm         — pre-norm of an active branch (RMSNorm / LayerNorm / AdaLN modulate),
+//                  fp32 residual in, bf16 GEMM operand out.
+//   stem, gemv, head_small, copy_out, pack_bf16 — the always-on parts around the
+//                  scheduled units (input stage, conditioning, output head, U-ViT skip
+//                  operands), Sec. 4.2: conditioning and skip features stay current.
+#include <cmath>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace sgd {
+
+namespace {
+
+constexpr int kNormThreads = 128;
+constexpr int kNormMaxVec = 8;  // float4 per thread: d <= 4096
+
+__device__ __forceinline__ float block_sum(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float s = 0.f;
+  const int nw = blockDim.x >> 5;
+  for (int i = 0; i < nw; ++i) s += red[i];
+  return s;
+}
+
+__device__ __forceinline__ void load_bf16x4(const bf16* p, float* f) {
+  const uint2 u = *reinterpret_cast<const uint2*>(p);
+  const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&u);
+  float2 a = __bfloat1622float2(b[0]), c = __bfloat1622float2(b[1]);
+  f[0] = a.x; f[1] = a.y; f[2] = c.x; f[3] = c.y;
+}
+
+__global__ void __launch_bounds__(kNormThreads) norm_kernel(const NormParams p) {
+  __shared__ float red[kNormThreads / 32];
+  const int row = blockIdx.x;
+  const int nv = p.d >> 2;
+  const float4* hr = reinterpret_cast<const float4*>(p.h + static_cast<int64_t>(row) * p.d);
+  float4 v[kNormMaxVec];
+  float sum = 0.f;
+#pragma unroll
+  for (int j = 0; j < kNormMaxVec; ++j) {
+    const int i = threadIdx.x + j * kNormThreads;
+    if (i < nv) {
+      v[j] = hr[i];
+      sum += (v[j].x + v[j].y) + (v[j].z + v[j].w);
+    }
+  }
+  float mean = 0.f, rstd;
+  if (p.kind == SGD_NORM_RMS) {
+    float sq = 0.f;
+#pragma unroll
+    for (int j = 0; j < kNormMaxVec; ++j) {
+      const int i = threadIdx.x + j * kNormThreads;
+      if (i < nv) sq += (v[j].x * v[j].x + v[j].y * v[j].y) + (v[j].z * v[j].z + v[j].w * v[j].w);
+    }
+    sq = block_sum(sq, red);
+    rstd = rsqrtf(sq / p.d + p.eps);
+  } else {
+    mean = block_sum(sum, red) / p.d;
+    float sq = 0.f;
+#pragma unroll
+    for (int j = 0; j < kNormMaxVec; ++j) {
+      const int i = threadIdx.x + j * kNormThreads;
+      if (i < nv) {
+        const float a = v[j].x - mean, b = v[j].y - mean, c = v[j].z - mean, d = v[j].w - mean;
+        sq += (a * a + b * b) + (c * c + d * d);
+      }
+    }
+    sq = block_sum(sq, red);
+    rstd = rsqrtf(sq / p.d + p.eps);
+  }
+  const float* sh = p.shift ? p.shift + static_cast<int64_t>(row / p.rows_per_batch) * p.ld_mod : nullptr;
+  const float* sc = p.scale ? p.scale + static_cast<int64_t>(row / p.rows_per_batch) * p.ld_mod : nullptr;
+  bf16* orow = p.out + static_cast<int64_t>(row) * p.d;
+#pragma unroll
+  for (int j = 0; j < kNormMaxVec; ++j) {
+    const int i = threadIdx.x + j * kNormThreads;
+    if (i < nv) {
+      float y[4] = {(v[j].x - mean) * rstd, (v[j].y - mean) * rstd, (v[j].z - mean) * rstd,
+                    (v[j].w - mean) * rstd};
+      if (p.g) {
+        float g[4];
+        load_bf16x4(p.g + 4 * i, g);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) y[k] *= g[k];
+      }
+      if (p.b) {
+        float b[4];
+        load_bf16x4(p.b + 4 * i, b);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) y[k] += b[k];
+      }
+      if (sc) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) y[k] = y[k] * (1.f + sc[4 * i + k]) + sh[4 * i + k];
+      }
+      uint2 u;
+      u.x = pack_bf16x2(y[0], y[1]);
+      u.y = pack_bf16x2(y[2], y[3]);
+      *reinterpret_cast<uint2*>(orow + 4 * i) = u;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(256) frozen_kernel(const __grid_constant__ FrozenParams p) {
+  const int64_t n8 = p.n >> 3;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n8; i += stride) {
+    float4* hp = reinterpret_cast<float4*>(p.h) + 2 * i;
+    const float4 a = hp[0], b = hp[1];
+    float acc[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+    for (int c = 0; c < p.n_caches; ++c) {
+      const uint4 u = __ldcs(reinterpret_cast<const uint4*>(p.caches[c]) + i);
+      float f[8];
+      unpack_bf16x8(u, f);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) acc[k] += f[k];
+    }
+    hp[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+    hp[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+  }
+}
+
+__global__ void io_set_kernel(IoSlot* slot, const IoSlot v) { *slot = v; }
+
+// sinusoid(t, dim)[c] = cos(t w_i) for c < half, sin(t w_{c-half}) otherwise,
+// w_i = 10000^(-i / half), evaluated in double precision.
+__device__ __forceinline__ float sinusoid_at(double t, int dim, int c) {
+  const int half = dim >> 1;
+  const int i = c < half ? c : c - half;
+  const double w = exp(-9.210340371976184 * static_cast<double>(i) / half);  // ln(10000)
+  return static_cast<float>(c < half ? cos(t * w) : sin(t * w));
+}
+
+__global__ void stem_kernel(const StemParams p) {
+  const int64_t total = static_cast<int64_t>(p.batch) * p.n_tokens * p.d;
+  const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (idx >= total) return;
+  const int c = static_cast<int>(idx % p.d);
+  const int64_t r = idx / p.d;
+  const int n = static_cast<int>(r % p.n_tokens);
+  const int b = static_cast<int>(r / p.n_tokens);
+  const IoSlot* s = p.slot;
+  float v = 0.f;
+  switch (p.kind) {
+    case SGD_STEM_TIME_ADD:
+      v = reinterpret_cast<const float*>(s->state)[idx] + sinusoid_at(s->t, p.d, c);
+      break;
+    case SGD_STEM_IDENTITY:
+      v = reinterpret_cast<const float*>(s->state)[idx];
+      break;
+    case SGD_STEM_EMBED: {
+      const int id = reinterpret_cast<const int32_t*>(s->state)[r];
+      v = __bfloat162float(p.embed[static_cast<int64_t>(id) * p.d + c]);
+      break;
+    }
+    case SGD_STEM_PATCH:
+    case SGD_STEM_PATCH_TOKENS: {
+      const int np = n - p.n_prefix;
+      if (np < 0) {
+        v = (n == 0) ? sinusoid_at(s->t, p.d, c)
+                     : __bfloat162float(p.class_emb[static_cast<int64_t>(s->class_ids[b]) * p.d + c]);
+      } else {
+        const float* z = reinterpret_cast<const float*>(s->state) +
+                         (static_cast<int64_t>(b) * (p.n_tokens - p.n_prefix) + np) * p.d_in;
+        const bf16* w = p.w_stem + static_cast<int64_t>(c) * p.d_in;
+        float acc = 0.f;
+        for (int k = 0; k < p.d_in; ++k) acc = fmaf(z[k], __bfloat162float(w[k]), acc);
+        v = acc;
+      }
+      v += __bfloat162float(p.pos[static_cast<int64_t>(n) * p.d + c]);
+      break;
+    }
+    default:
+      break;
+  }
+  p.h[idx] = v;
+}
+
+// One warp per output column j; all rows (<= 16) share the weight row read.
+constexpr int kGemvMaxRows = 16;
+__global__ void __launch_bounds__(256) gemv_kernel(const GemvParams p) {
+  extern __shared__ float xs[];  // [rows][K]
+  const int xrows = p.x_sinusoid ? 1 : (p.ldx == 0 ? 1 : p.rows);
+  for (int i = threadIdx.x; i < xrows * p.K; i += blockDim.x) {
+    const int r = i / p.K, k = i % p.K;
+    float x = p.x_sinusoid ? sinusoid_at(p.slot->t, p.K, k) : p.x[static_cast<int64_t>(r) * p.ldx + k];
+    if (p.in_silu) x = silu_f(x);
+    xs[i] = x;
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int j = blockIdx.x * (blockDim.x >> 5) + warp;
+  if (j >= p.N) return;
+  float acc[kGemvMaxRows];
+#pragma unroll
+  for (int r = 0; r < kGemvMaxRows; ++r) acc[r] = 0.f;
+  const bf16* w = p.W + static_cast<int64_t>(j) * p.K;
+  for (int k = lane * 8; k < p.K; k += 256) {
+    float f[8];
+    unpack_bf16x8(*reinterpret_cast<const uint4*>(w + k), f);
+#pragma unroll
+    for (int r = 0; r < kGemvMaxRows; ++r) {
+      if (r < xrows) {
+        const float* x = xs + r * p.K + k;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[r] = fmaf(f[q], x[q], acc[r]);
+      }
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < kGemvMaxRows; ++r) {
+    if (r < xrows) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) acc[r] += __shfl_xor_sync(0xffffffffu, acc[r], o);
+    }
+  }
+  if (lane == 0) {
+    for (int r = 0; r < p.rows; ++r) {
+      float v = acc[xrows == 1 ? 0 : r];
+      if (p.add_class)
+        v += __bfloat162float(p.add_class[static_cast<int64_t>(p.slot->class_ids[r]) * p.N + j]);
+      if (p.add_vec) v += p.add_vec[j];
+      p.out[static_cast<int64_t>(r) * p.ldo + j] = v;
+    }
+  }
+}
+
+// One warp per row; W rows re-read from L1.
+__global__ void __launch_bounds__(256) head_small_kernel(const HeadParams p) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t r = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + warp;
+  const int64_t rows = static_cast<int64_t>(p.batch) * p.n_tokens;
+  if (r >= rows) return;
+  const int n = static_cast<int>(r % p.n_tokens), b = static_cast<int>(r / p.n_tokens);
+  if (n < p.n_prefix) return;
+  float* out = reinterpret_cast<float*>(p.slot->out) +
+               (static_cast<int64_t>(b) * (p.n_tokens - p.n_prefix) + (n - p.n_prefix)) *
+                   p.out_channels;
+  const bf16* x = p.x + r * p.ldx;
+  for (int j = 0; j < p.out_channels; ++j) {
+    const bf16* w = p.W + static_cast<int64_t>(j) * p.K;
+    float acc = 0.f;
+    for (int k = lane * 8; k < p.K; k += 256) {
+      float fx[8], fw[8];
+      unpack_bf16x8(*reinterpret_cast<const uint4*>(x + k), fx);
+      unpack_bf16x8(*reinterpret_cast<const uint4*>(w + k), fw);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) acc = fmaf(fx[q], fw[q], acc);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) out[j] = acc;
+  }
+}
+
+__global__ void copy_out_kernel(const IoSlot* slot, const float* h, int64_t n4) {
+  float4* o = reinterpret_cast<float4*>(slot->out);
+  const float4* s = reinterpret_cast<const float4*>(h);
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride)
+    o[i] = s[i];
+}
+
+__global__ void pack_bf16_kernel(bf16* dst, int ld_dst, int col0, const float* h, int rows, int d) {
+  const int64_t n4 = static_cast<int64_t>(rows) * d / 4;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
+    const int64_t e = i * 4;
+    const int64_t r = e / d;
+    const int c = static_cast<int>(e % d);
+    const float4 v = reinterpret_cast<const float4*>(h)[i];
+    uint2 u;
+    u.x = pack_bf16x2(v.x, v.y);
+    u.y = pack_bf16x2(v.z, v.w);
+    *reinterpret_cast<uint2*>(dst + r * ld_dst + col0 + c) = u;
+  }
+}
+
+__global__ void sampler_kernel(float* z, const float* eps, float alpha, float beta, int64_t n) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n; i += stride)
+    z[i] = alpha * z[i] - beta * eps[i];
+}
+
+int grid_for(int64_t work, int threads) {
+  const int64_t cap = static_cast<int64_t>(num_sms()) * 8;
+  int64_t g = (work + threads - 1) / threads;
+  if (g > cap) g = cap;
+  return g < 1 ? 1 : static_cast<int>(g);
+}
+
+}  // namespace
+
+cudaError_t norm_launch(const NormParams& p, cudaStream_t s) {
+  norm_kernel<<<p.rows, kNormThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t frozen_launch(const FrozenParams& p, cudaStream_t s) {
+  frozen_kernel<<<grid_for(p.n / 8, 256), 256, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t io_set_launch(IoSlot* slot, const IoSlot& v, cudaStream_t s) {
+  io_set_kernel<<<1, 1, 0, s>>>(slot, v);
+  return cudaGetLastError();
+}
+
+cudaError_t stem_launch(const StemParams& p, cudaStream_t s) {
+  const int64_t total = static_cast<int64_t>(p.batch) * p.n_tokens * p.d;
+  stem_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t gemv_launch(const GemvParams& p, cudaStream_t s) {
+  const int xrows = p.x_sinusoid ? 1 : (p.ldx == 0 ? 1 : p.rows);
+  const size_t smem = static_cast<size_t>(xrows) * p.K * sizeof(float);
+  if (p.rows > kGemvMaxRows || smem > 200 * 1024) return cudaErrorInvalidValue;
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(gemv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  gemv_kernel<<<(p.N + 7) / 8, 256, smem, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t head_small_launch(const HeadParams& p, cudaStream_t s) {
+  const int64_t rows = static_cast<int64_t>(p.batch) * p.n_tokens;
+  head_small_kernel<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t copy_out_launch(const IoSlot* slot, const float* h, int64_t n, cudaStream_t s) {
+  copy_out_kernel<<<grid_for(n / 4, 256), 256, 0, s>>>(slot, h, n / 4);
+  return cudaGetLastError();
+}
+
+cudaError_t pack_bf16_launch(bf16* dst, int ld_dst, int col0, const float* h, int rows, int d,
+                             cudaStream_t s) {
+  pack_bf16_kernel<<<grid_for(static_cast<int64_t>(rows) * d / 4, 256), 256, 0, s>>>(dst, ld_dst,
+                                                                                    col0, h, rows, d);
+  return cudaGetLastError();
+}
+
+cudaError_t sampler_launch(float* z, const float* eps, float alpha, float beta, int64_t n,
+                           cudaStream_t s) {
+  sampler_kernel<<<grid_for(n, 256), 256, 0, s>>>(z, eps, alpha, beta, n);
+  return cudaGetLastError();
+}
+
+}  // namespace sgd

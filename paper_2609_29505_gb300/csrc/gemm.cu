@@ -1,0 +1,555 @@
+// C = A B^T on the 5th-generation tensor cores (tcgen05) with fused epilogues.
+//
+// This is the projection kernel of every active residual branch (Algorithm 2: an
+// active unit computes Delta = F_l(h; c), refreshes its cache and adds Delta to the
+// residual stream).  The branch's last projection runs with the DELTA epilogue,
+// which stores the bf16 cache entry and adds Delta to the fp32 residual h in the
+// same pass over the tile.
+//
+// Design (one CTA per SM, persistent over 128 x 256 output tiles):
+//   warp 0      TMA producer: A box 128x64 and two B boxes 128x64 per stage into a
+//               4-stage ring of 48 KB stages (128-byte swizzle).
+//   warp 1      allocates 512 TMEM columns (two 128x256 fp32 accumulators) and one
+//               elected lane issues tcgen05.mma (M=128, N=256, K=16) four times per
+//               stage, committing each stage back to the producer.
+//   warps 2-5   epilogue: tcgen05.ld rows out of TMEM (warp w owns TMEM lanes
+//               32 (w % 4) ...), apply the epilogue, store to global memory.  The two
+//               accumulators let the epilogue of tile i overlap the MMAs of tile i+1.
+// Every wait is bounded (common.cuh); on expiry the CTA drains its own copies and
+// MMAs, frees TMEM and exits with the device status word set.
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace sgd {
+
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kBN = 256;        // accumulator columns per tile
+constexpr int kBK = 64;         // bf16 elements per 128-byte row
+constexpr int kStages = 4;
+constexpr int kTileA = kBM * kBK * 2;          // 16 KB
+constexpr int kTileBHalf = 128 * kBK * 2;      // 16 KB
+constexpr int kStageBytes = kTileA + 2 * kTileBHalf;  // 48 KB
+constexpr int kTmemCols = 512;
+constexpr int kThreads = 192;
+constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+
+struct TcArgs {
+  CUtensorMap tmap_a;
+  CUtensorMap tmap_b;
+  EpiParams epi;
+  int M, N, K;  // N = output columns
+  int num_m, num_n, num_k;
+  int gated;    // B second half starts at row N (= f)
+  int* status;
+};
+
+__device__ int g_status;  // device status word (bounded-wait expiry codes)
+
+// ----------------------------------------------------------------------------
+// epilogue: 8 consecutive output columns of one row
+// ----------------------------------------------------------------------------
+
+__device__ __forceinline__ void store8_bf16(void* base, int ld, int row, int col, const float* v) {
+  bf16* p = reinterpret_cast<bf16*>(base) + static_cast<int64_t>(row) * ld + col;
+  *reinterpret_cast<uint4*>(p) = pack_bf16x8(v);
+}
+
+__device__ __forceinline__ void epi_store8(const EpiParams& e, void* out, int row, int col,
+                                           float* v) {
+  switch (e.kind) {
+    case SGD_EPI_BF16:
+    case SGD_EPI_ROPE:
+    case SGD_EPI_GATED:
+      store8_bf16(out, e.ldo, row, col, v);
+      break;
+    case SGD_EPI_GELU: {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) v[i] = e.act ? gelu_erf_f(v[i]) : gelu_tanh_f(v[i]);
+      store8_bf16(out, e.ldo, row, col, v);
+      break;
+    }
+    case SGD_EPI_F32: {
+      float4* p = reinterpret_cast<float4*>(reinterpret_cast<float*>(out) +
+                                            static_cast<int64_t>(row) * e.ldo + col);
+      p[0] = make_float4(v[0], v[1], v[2], v[3]);
+      p[1] = make_float4(v[4], v[5], v[6], v[7]);
+      break;
+    }
+    case SGD_EPI_DELTA: {
+      if (e.gate) {
+        const float4* g = reinterpret_cast<const float4*>(
+            e.gate + static_cast<int64_t>(row / e.rows_per_batch) * e.ld_gate + col);
+        const float4 g0 = g[0], g1 = g[1];
+        v[0] *= g0.x; v[1] *= g0.y; v[2] *= g0.z; v[3] *= g0.w;
+        v[4] *= g1.x; v[5] *= g1.y; v[6] *= g1.z; v[7] *= g1.w;
+      }
+      float4* hp = reinterpret_cast<float4*>(e.h + static_cast<int64_t>(row) * e.ldh + col);
+      float4 h0 = hp[0], h1 = hp[1];
+      h0.x += v[0]; h0.y += v[1]; h0.z += v[2]; h0.w += v[3];
+      h1.x += v[4]; h1.y += v[5]; h1.z += v[6]; h1.w += v[7];
+      hp[0] = h0;
+      hp[1] = h1;
+      if (e.cache) store8_bf16(e.cache, e.ld_cache, row, col, v);
+      break;
+    }
+    default:
+      break;
+  }
+}
+
+__device__ __forceinline__ void u32_to_f32x16(const uint32_t* r, float* f) {
+#pragma unroll
+  for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(r[i]);
+}
+
+// Epilogue of one 128 x 256 accumulator, executed by all 128 epilogue threads; this
+// thread owns tile row `row` (TMEM lane row - m0) and reads from `tbase`.
+__device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int row, int n_blk,
+                                              uint32_t tbase) {
+  const EpiParams& e = a.epi;
+  const bool row_ok = row < a.M;
+  uint32_t r0[16], r1[16];
+  float x[16], y[16];
+  if (a.gated) {
+    const int n0 = n_blk * 128;
+    for (int c = 0; c < 128; c += 16) {
+      if (n0 + c >= a.N) break;
+      tmem_ld16(tbase + c, r0);
+      tmem_ld16(tbase + 128 + c, r1);
+      tmem_ld_wait16(r0);
+      tmem_ld_wait16(r1);
+      u32_to_f32x16(r0, x);
+      u32_to_f32x16(r1, y);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) x[i] = e.act ? x[i] * gelu_erf_f(y[i]) : silu_f(x[i]) * y[i];
+      if (row_ok) {
+        if (n0 + c < a.N) epi_store8(e, out, row, n0 + c, x);
+        if (n0 + c + 8 < a.N) epi_store8(e, out, row, n0 + c + 8, x + 8);
+      }
+    }
+    return;
+  }
+  const int n0 = n_blk * kBN;
+  if (e.kind == SGD_EPI_ROPE) {
+    const int dh = e.d_head, half = dh >> 1;
+    const int pos = row_ok ? row % e.rope_tokens : 0;
+    for (int hb = 0; hb < kBN; hb += dh) {
+      if (n0 + hb >= a.N) break;
+      const bool rot = (n0 + hb) < e.rope_cols;
+      for (int j = 0; j < half; j += 16) {
+        tmem_ld16(tbase + hb + j, r0);
+        tmem_ld16(tbase + hb + half + j, r1);
+        tmem_ld_wait16(r0);
+        tmem_ld_wait16(r1);
+        u32_to_f32x16(r0, x);
+        u32_to_f32x16(r1, y);
+        if (rot && row_ok) {
+          const float* cs = e.rope_cos + static_cast<int64_t>(pos) * half + j;
+          const float* sn = e.rope_sin + static_cast<int64_t>(pos) * half + j;
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const float c_ = cs[i], s_ = sn[i];
+            const float a1 = x[i], a2 = y[i];
+            x[i] = a1 * c_ - a2 * s_;
+            y[i] = a2 * c_ + a1 * s_;
+          }
+        }
+        if (row_ok) {
+          const int c1 = n0 + hb + j, c2 = c1 + half;
+          epi_store8(e, out, row, c1, x);
+          epi_store8(e, out, row, c1 + 8, x + 8);
+          epi_store8(e, out, row, c2, y);
+          epi_store8(e, out, row, c2 + 8, y + 8);
+        }
+      }
+    }
+    return;
+  }
+  for (int c = 0; c < kBN; c += 32) {
+    if (n0 + c >= a.N) break;
+    tmem_ld16(tbase + c, r0);
+    tmem_ld16(tbase + c + 16, r1);
+    tmem_ld_wait16(r0);
+    tmem_ld_wait16(r1);
+    u32_to_f32x16(r0, x);
+    u32_to_f32x16(r1, y);
+    if (row_ok) {
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        if (n0 + c + 8 * q < a.N) epi_store8(e, out, row, n0 + c + 8 * q, x + 8 * q);
+        if (n0 + c + 16 + 8 * q < a.N) epi_store8(e, out, row, n0 + c + 16 + 8 * q, y + 8 * q);
+      }
+    }
+  }
+}
+
+// Wait on a barrier with the whole warp: lane 0 polls, the verdict is broadcast so
+// that the warp stays converged for the .sync.aligned tcgen05 instructions.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                          int* status, int code) {
+  int ok = 0;
+  if (lane_id() == 0) ok = mbar_wait(bar, parity, abort_flag, status, code) ? 1 : 0;
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  return ok != 0;
+}
+
+// Bounded wait that ignores the abort flag (used while draining after an abort).
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (global_timer_ns() - t0 > kWaitTimeoutNs) break;
+  }
+}
+
+__global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* tiles = smem;
+  uint64_t* full = reinterpret_cast<uint64_t*>(tiles + kStages * kStageBytes);
+  uint64_t* empty = full + kStages;
+  uint64_t* tfull = empty + kStages;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tfull[i], 1);
+      mbar_init(&tempty[i], 4);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&a.tmap_a);
+    tma_prefetch_desc(&a.tmap_b);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int num_tiles = a.num_m * a.num_n;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int it = 0;
+      for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+        const int m_blk = tile % a.num_m, n_blk = tile / a.num_m;
+        const int rb0 = a.gated ? n_blk * 128 : n_blk * kBN;
+        const int rb1 = a.gated ? a.N + n_blk * 128 : rb0 + 128;
+        bool ok = true;
+        for (int kb = 0; kb < a.num_k; ++kb, ++it) {
+          const int s = it % kStages;
+          const uint32_t ph = (it / kStages) & 1;
+          if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status, 1)) {
+            ok = false;
+            break;
+          }
+          uint8_t* st = tiles + s * kStageBytes;
+          mbar_arrive_expect_tx(&full[s], kStageBytes);
+          tma_load_2d(st, &a.tmap_a, &full[s], kb * kBK, m_blk * kBM);
+          tma_load_2d(st + kTileA, &a.tmap_b, &full[s], kb * kBK, rb0);
+          tma_load_2d(st + kTileA + kTileBHalf, &a.tmap_b, &full[s], kb * kBK, rb1);
+        }
+        if (!ok) break;
+      }
+      if (*abort_flag) {
+        // wait for the loads still in flight (the latest issue of each stage)
+        for (int i = (it > kStages ? it - kStages : 0); i < it; ++i)
+          drain_wait(&full[i % kStages], (i / kStages) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = umma_idesc_bf16(kBM, kBN);
+      int it = 0, lt = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++lt) {
+        const int acc = lt & 1;
+        const uint32_t aph = (lt >> 1) & 1;
+        if (!mbar_wait(&tempty[acc], aph ^ 1u, abort_flag, a.status, 2)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * kBN;
+        for (int kb = 0; kb < a.num_k; ++kb, ++it) {
+          const int s = it % kStages;
+          const uint32_t ph = (it / kStages) & 1;
+          if (!mbar_wait(&full[s], ph, abort_flag, a.status, 3)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_addr = smem_u32(tiles + s * kStageBytes);
+          const uint32_t b_addr = a_addr + kTileA;
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k) {
+            umma_bf16(d_tmem, smem_desc_sw128(a_addr + 32 * k), smem_desc_sw128(b_addr + 32 * k),
+                      idesc, (kb | k) != 0 ? 1u : 0u);
+          }
+          umma_commit(&empty[s]);
+        }
+        if (!ok) break;
+        umma_commit(&tfull[acc]);
+      }
+      // every MMA issued by this thread has finished once `drain` completes
+      umma_commit(drain);
+      drain_wait(drain, 0);
+    }
+  } else {
+    const int q = warp & 3;
+    int lt = 0;
+    void* out = a.epi.out_slot ? *a.epi.out_slot : a.epi.out;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
+      const int m_blk = tile % a.num_m, n_blk = tile / a.num_m;
+      const int acc = lt & 1;
+      const uint32_t aph = (lt >> 1) & 1;
+      if (!warp_wait(&tfull[acc], aph, abort_flag, a.status, 4)) break;
+      tc_fence_after();
+      const int row = m_blk * kBM + q * 32 + lane;
+      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * kBN;
+      epilogue_tile(a, out, row, n_blk, tbase);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+// ----------------------------------------------------------------------------
+// SIMT reference GEMM: one output element per thread, fp32 accumulation in K order.
+// ----------------------------------------------------------------------------
+
+struct SimtArgs {
+  const bf16* A;
+  int lda;
+  const bf16* B;
+  int ldb;
+  int M, N, K;
+  EpiParams epi;
+};
+
+__device__ __forceinline__ float dot_bf16(const bf16* a, const bf16* b, int K) {
+  float acc = 0.f;
+  int k = 0;
+  for (; k + 8 <= K; k += 8) {
+    float fa[8], fb[8];
+    unpack_bf16x8(*reinterpret_cast<const uint4*>(a + k), fa);
+    unpack_bf16x8(*reinterpret_cast<const uint4*>(b + k), fb);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc = fmaf(fa[i], fb[i], acc);
+  }
+  for (; k < K; ++k) acc = fmaf(__bfloat162float(a[k]), __bfloat162float(b[k]), acc);
+  return acc;
+}
+
+__global__ void gemm_simt_kernel(const SimtArgs a) {
+  const int col = blockIdx.x * blockDim.x + threadIdx.x;
+  const int row = blockIdx.y;
+  if (col >= a.N || row >= a.M) return;
+  const EpiParams& e = a.epi;
+  void* out = e.out_slot ? *e.out_slot : e.out;
+  const bf16* arow = a.A + static_cast<int64_t>(row) * a.lda;
+  float v = dot_bf16(arow, a.B + static_cast<int64_t>(col) * a.ldb, a.K);
+  switch (e.kind) {
+    case SGD_EPI_GATED: {
+      const float u = dot_bf16(arow, a.B + static_cast<int64_t>(a.N + col) * a.ldb, a.K);
+      v = e.act ? v * gelu_erf_f(u) : silu_f(v) * u;
+      break;
+    }
+    case SGD_EPI_GELU:
+      v = e.act ? gelu_erf_f(v) : gelu_tanh_f(v);
+      break;
+    case SGD_EPI_ROPE:
+      if (col < e.rope_cols) {
+        const int half = e.d_head >> 1;
+        const int i = col % e.d_head;
+        const int pos = row % e.rope_tokens;
+        const int partner = i < half ? col + half : col - half;
+        const int fi = i < half ? i : i - half;
+        const float c_ = e.rope_cos[pos * half + fi], s_ = e.rope_sin[pos * half + fi];
+        const float p = dot_bf16(arow, a.B + static_cast<int64_t>(partner) * a.ldb, a.K);
+        v = i < half ? v * c_ - p * s_ : v * c_ + p * s_;
+      }
+      break;
+    case SGD_EPI_DELTA: {
+      if (e.gate) v *= e.gate[static_cast<int64_t>(row / e.rows_per_batch) * e.ld_gate + col];
+      float* hp = e.h + static_cast<int64_t>(row) * e.ldh + col;
+      *hp = *hp + v;
+      if (e.cache) e.cache[static_cast<int64_t>(row) * e.ld_cache + col] = __float2bfloat16_rn(v);
+      return;
+    }
+    default:
+      break;
+  }
+  if (e.kind == SGD_EPI_F32)
+    reinterpret_cast<float*>(out)[static_cast<int64_t>(row) * e.ldo + col] = v;
+  else
+    reinterpret_cast<bf16*>(out)[static_cast<int64_t>(row) * e.ldo + col] = __float2bfloat16_rn(v);
+}
+
+// ----------------------------------------------------------------------------
+// host side
+// ----------------------------------------------------------------------------
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// bf16 [rows, cols] with row stride ld elements; box = 64 columns x box_rows rows.
+bool make_tmap(CUtensorMap* m, const void* base, int rows, int cols, int ld, int box_rows) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+int num_sms() {
+  int dev = 0, n = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  return n > 0 ? n : 1;
+}
+
+int* device_status_ptr() {
+  static int* ptr[64] = {nullptr};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64) return nullptr;
+  if (!ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return nullptr;
+    ptr[dev] = static_cast<int*>(p);
+  }
+  return ptr[dev];
+}
+
+int gemm_plan(GemmPlan& p, const char** why) {
+  const EpiParams& e = p.epi;
+  const bool gated = e.kind == SGD_EPI_GATED;
+  if (!p.A || !p.B || p.M <= 0 || p.N <= 0 || p.K <= 0) {
+    *why = "gemm: null operand or empty shape";
+    return -1;
+  }
+  if ((p.K % 8) || (p.lda % 8) || (p.ldb % 8) || (p.N % 8) || !aligned16(p.A) || !aligned16(p.B)) {
+    *why = "gemm: K, lda, ldb, N must be multiples of 8 and operands 16-byte aligned";
+    return -2;
+  }
+  if (e.kind == SGD_EPI_DELTA) {
+    if (!e.h || (e.ldh % 4) || !aligned16(e.h) || (e.cache && (e.ld_cache % 8)) ||
+        (e.gate && (e.ld_gate % 4 || e.rows_per_batch <= 0))) {
+      *why = "gemm: DELTA epilogue needs an aligned residual (ldh % 4), ld_cache % 8, ld_gate % 4";
+      return -2;
+    }
+  } else if (!e.out && !e.out_slot) {
+    *why = "gemm: missing output";
+    return -1;
+  } else if (e.ldo % 8) {
+    *why = "gemm: ldo must be a multiple of 8";
+    return -2;
+  }
+  if (e.kind == SGD_EPI_ROPE &&
+      (!(e.d_head == 64 || e.d_head == 128) || !e.rope_cos || !e.rope_sin || e.rope_tokens <= 0 ||
+       (e.rope_cols % e.d_head))) {
+    *why = "gemm: RoPE epilogue needs d_head 64 or 128 and cos/sin tables";
+    return -2;
+  }
+  if (p.simt) return 0;
+  const int b_rows = gated ? 2 * p.N : p.N;
+  if (!make_tmap(&p.tmap_a, p.A, p.M, p.K, p.lda, 128) ||
+      !make_tmap(&p.tmap_b, p.B, b_rows, p.K, p.ldb, 128)) {
+    *why = "gemm: cuTensorMapEncodeTiled failed (driver entry point unavailable or bad layout)";
+    return -5;
+  }
+  const int num_m = (p.M + kBM - 1) / kBM;
+  const int num_n = gated ? (p.N + 127) / 128 : (p.N + kBN - 1) / kBN;
+  const int tiles = num_m * num_n;
+  const int sms = num_sms();
+  p.grid = tiles < sms ? tiles : sms;
+  return 0;
+}
+
+cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s) {
+  if (p.simt) {
+    SimtArgs a{p.A, p.lda, p.B, p.ldb, p.M, p.N, p.K, p.epi};
+    dim3 grid((p.N + 127) / 128, p.M);
+    gemm_simt_kernel<<<grid, 128, 0, s>>>(a);
+    return cudaGetLastError();
+  }
+  static bool attr_done[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    if (err != cudaSuccess) return err;
+    attr_done[dev] = true;
+  }
+  TcArgs a;
+  memcpy(&a.tmap_a, &p.tmap_a, sizeof(CUtensorMap));
+  memcpy(&a.tmap_b, &p.tmap_b, sizeof(CUtensorMap));
+  a.epi = p.epi;
+  a.epi.M = p.M;
+  a.epi.N = p.N;
+  a.M = p.M;
+  a.N = p.N;
+  a.K = p.K;
+  a.gated = p.epi.kind == SGD_EPI_GATED;
+  a.num_m = (p.M + kBM - 1) / kBM;
+  a.num_n = a.gated ? (p.N + 127) / 128 : (p.N + kBN - 1) / kBN;
+  a.num_k = (p.K + kBK - 1) / kBK;
+  a.status = device_status_ptr();
+  gemm_tc_kernel<<<p.grid, kThreads, kSmemBytes, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace sgd

@@ -1,0 +1,160 @@
+// Internal interface between the C ABI (api.cu) and the kernel translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "../../include/sgd.h"
+#include "../../include/sgd_kernels.h"
+
+namespace sgd {
+
+using bf16 = __nv_bfloat16;
+
+// Epilogue parameters as the kernels see them (mirror of sgd_epilogue_args plus the
+// output-pointer slot used by captured graphs and the output extent).
+struct EpiParams {
+  int kind;
+  void* out;
+  int ldo;
+  void* const* out_slot;  // device address holding the output pointer (overrides out)
+  float* h;
+  int ldh;
+  bf16* cache;
+  int ld_cache;
+  const float* gate;
+  int ld_gate;
+  int rows_per_batch;
+  int act;
+  const float* rope_cos;
+  const float* rope_sin;
+  int rope_tokens;
+  int d_head;
+  int rope_cols;
+  int M;
+  int N;  // output columns (gated: f)
+};
+
+// A planned GEMM: operands, epilogue and prebuilt TMA descriptors.
+struct GemmPlan {
+  const bf16* A = nullptr;
+  int lda = 0;
+  const bf16* B = nullptr;
+  int ldb = 0;
+  int M = 0, N = 0, K = 0;   // N = output columns
+  EpiParams epi{};
+  bool simt = false;
+  CUtensorMap tmap_a;
+  CUtensorMap tmap_b;
+  int grid = 0;
+};
+
+// Validates shapes and builds the tensor maps; returns an sgd_status.
+int gemm_plan(GemmPlan& p, const char** why);
+cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s);
+int* device_status_ptr();  // device address of the shared status word
+int num_sms();
+
+// Attention.
+struct AttnParams {
+  const bf16* q;
+  int ldq;
+  const bf16* k;
+  const bf16* v;
+  int ldkv;
+  bf16* o;
+  int ldo;
+  int batch, n_q, n_kv, n_heads, d_head;
+};
+int attn_check(const AttnParams& p, const char** why);
+cudaError_t attn_launch(const AttnParams& p, cudaStream_t s);
+
+// Norm: out = norm(h) [* (1 + scale) + shift].
+struct NormParams {
+  const float* h;
+  bf16* out;
+  int rows, d, kind;
+  const bf16* g;
+  const bf16* b;
+  const float* shift;
+  const float* scale;
+  int ld_mod, rows_per_batch;
+  float eps;
+};
+cudaError_t norm_launch(const NormParams& p, cudaStream_t s);
+
+// Frozen run: h += sum caches.
+constexpr int kMaxRun = 96;
+struct FrozenParams {
+  float* h;
+  const bf16* caches[kMaxRun];
+  int n_caches;
+  int64_t n;
+};
+cudaError_t frozen_launch(const FrozenParams& p, cudaStream_t s);
+
+// Per-step I/O slot (device memory) read by graph kernels.
+struct IoSlot {
+  const void* state;
+  void* out;
+  const int32_t* class_ids;
+  const void* ctx;
+  float t;
+  int step;
+};
+cudaError_t io_set_launch(IoSlot* slot, const IoSlot& v, cudaStream_t s);
+
+// Small always-on pieces (stem, conditioning, heads).
+struct StemParams {
+  int kind;
+  const IoSlot* slot;
+  float* h;
+  int batch, n_tokens, n_prefix, d, d_in;
+  const bf16* w_stem;
+  const bf16* pos;
+  const bf16* class_emb;
+  const bf16* embed;
+};
+cudaError_t stem_launch(const StemParams& p, cudaStream_t s);
+
+// out[r, j] = sum_k act(x[r, k]) W[j, k] (+ add[r, j]); x fp32 or computed on the fly.
+struct GemvParams {
+  float* out;
+  int ldo;
+  const float* x;      // [rows, K] fp32 (ignored when x_sinusoid)
+  int ldx;
+  int x_sinusoid;      // x = sinusoid(t, K) from the slot, one row
+  const IoSlot* slot;
+  int in_silu;         // act = silu
+  const bf16* W;       // [N, K]
+  int N, K, rows;
+  const bf16* add_class;  // optional: + class_emb[class_ids[r]] (bf16 [*, N])
+  const float* add_vec;   // optional: + add_vec[j] (broadcast over rows)
+};
+cudaError_t gemv_launch(const GemvParams& p, cudaStream_t s);
+
+// Row-wise small-N linear for heads: out[r, j] = x[r] . W[j] for j < N (N <= 64).
+struct HeadParams {
+  const bf16* x;       // [rows_total, K] bf16 (normalised states)
+  int ldx;
+  const bf16* W;       // [N, K]
+  int N, K;
+  int batch, n_tokens, n_prefix;  // rows r = b * n_tokens + n, n >= n_prefix are output
+  int out_channels;               // columns written (<= N)
+  const IoSlot* slot;             // out pointer: fp32 [batch, n_tokens - n_prefix, out_channels]
+};
+cudaError_t head_small_launch(const HeadParams& p, cudaStream_t s);
+
+// Identity head: out (from slot) = h.
+cudaError_t copy_out_launch(const IoSlot* slot, const float* h, int64_t n, cudaStream_t s);
+
+// U-ViT: dst bf16 [rows, ld_dst] columns [col0, col0 + d) = bf16(h).
+cudaError_t pack_bf16_launch(bf16* dst, int ld_dst, int col0, const float* h, int rows, int d,
+                             cudaStream_t s);
+
+cudaError_t sampler_launch(float* z, const float* eps, float alpha, float beta, int64_t n,
+                           cudaStream_t s);
+
+}  // namespace sgd

@@ -1,0 +1,78 @@
+"""The product's offline schedule (paper_2609_29505_gb300.schedule) against the oracle:
+lifetimes must agree bit for bit (integers) on every small config, budget and
+unit granularity; scores to float64 rounding."""
+import numpy as np
+import pytest
+
+from oracle import denoiser as odn
+from oracle import spectral as osp
+from paper_2609_29505_gb300 import schedule, synth
+
+SMALL = ["tiny", "dit_small", "uvit_small", "sdxl_small", "llada_small"]
+
+
+@pytest.fixture(scope="module")
+def weights():
+    return {n: synth.make_weights(synth.get_config(n), "cpu") for n in SMALL}
+
+
+@pytest.mark.parametrize("name", SMALL)
+def test_branch_scores_match_oracle(name, weights):
+    cfg = synth.get_config(name)
+    W = odn.to_numpy_weights(weights[name])
+    want = np.array(osp.branch_scores(cfg, W))
+    got = schedule.branch_scores(cfg, weights[name])
+    np.testing.assert_allclose(got, want, rtol=1e-9)
+
+
+@pytest.mark.parametrize("name", SMALL)
+@pytest.mark.parametrize("budget", [1.0, 0.5, 0.33])
+@pytest.mark.parametrize("gran", ["block", "branch"])
+def test_lifetimes_bit_exact(name, budget, gran, weights):
+    cfg = synth.get_config(name)
+    T = cfg.T
+    W = odn.to_numpy_weights(weights[name])
+    groups = synth.block_groups(cfg) if gran == "block" else synth.branch_groups(cfg)
+    want = osp.schedule(cfg, W, T, budget, groups)
+    got = schedule.build_schedule(cfg, weights[name], T, budget=budget, granularity=gran)
+    np.testing.assert_array_equal(got["lifetimes"], want["lifetimes"])
+    np.testing.assert_array_equal(got["groups"], np.asarray(groups))
+    assert got["ratio"] == pytest.approx(want["ratio"])
+    assert got["ratio"] <= budget + 1e-12
+
+
+@pytest.mark.parametrize("T", [10, 30, 50, 64, 100])
+def test_budget_rule_matches_oracle_on_random_scores(T):
+    rng = np.random.default_rng(T)
+    for G in (4, 21, 28, 32):
+        lam = osp.normalise(rng.uniform(0.02, 1.0, size=G))
+        for budget in (1.0, 0.5, 0.35, 0.33, 0.2):
+            s_min = osp.min_lifetime(T)
+            _, want, ok_w = osp.tau_for_budget(lam, T, budget, s_min)
+            _, got, ok_g = schedule.tau_for_budget(lam, T, budget, s_min)
+            assert ok_w == ok_g
+            np.testing.assert_array_equal(got, want)
+
+
+def test_fixed_tau_matches_oracle(weights):
+    cfg = synth.get_config("dit_small")
+    W = odn.to_numpy_weights(weights["dit_small"])
+    groups = synth.block_groups(cfg)
+    lam = osp.normalise(osp.unit_scores(osp.branch_scores(cfg, W), groups))
+    for tau in (0.5, 1.0, 2.0):
+        want = osp.lifetimes(lam, cfg.T, tau, osp.min_lifetime(cfg.T))
+        got = schedule.build_schedule(cfg, weights["dit_small"], cfg.T, tau=tau)
+        np.testing.assert_array_equal(got["group_lifetimes"], want)
+
+
+@pytest.mark.parametrize("ranking", ["frobenius", "spectral", "stable_rank", "frob_stable_rank",
+                                     "raw_scr", "depth", "random"])
+def test_alternative_rankings_meet_budget(ranking, weights):
+    cfg = synth.get_config("dit_small")
+    res = schedule.build_schedule(cfg, weights["dit_small"], cfg.T, budget=0.5, ranking=ranking)
+    assert res["ratio"] <= 0.5
+    assert res["lifetimes"].min() >= res["s_min"]
+    lam = res["lam"]
+    S = res["group_lifetimes"]
+    order = np.argsort(lam, kind="stable")
+    assert np.all(np.diff(S[order]) >= 0)
