@@ -1,0 +1,440 @@
+"""Benchmark: scheduled denoiser steps/s at a layer-step budget on one GB300.
+
+Default workload: the LLaDA-8B-shaped masked-diffusion transformer (32 blocks,
+d 4096, 32 heads x 128, SwiGLU 12288, RMSNorm, RoPE, 126464-token head), batch 4 x
+1024 tokens, horizon T = 64, 50% layer-step budget from the SCR/Frobenius
+schedule.  A bench "step" is one denoiser evaluation (one sgd_step: stem, every
+active unit, frozen runs, head) at trajectory position s; timed steps run whole
+trajectories from s = 1, cycling every T steps.
+
+Prints ONE JSON line (rank 0).  --impl reference times the CPU oracle instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "scheduled denoiser steps/s at 50% layer-step budget; % of BF16/HBM roofline"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=None, help="timed denoiser steps (default T)")
+    ap.add_argument("--warmup", type=int, default=None, help="untimed steps (default T)")
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--config", default="llada")
+    ap.add_argument("--budget", type=float, default=0.5)
+    ap.add_argument("--T", type=int, default=None)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sus=d["bf16_tflops_sustained"],
+                    source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms while running."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        self.lines = []
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in getattr(self, "lines", []):
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = max(mx, float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        loaded = [x for x in sm if x > 0.5 * max(sm)] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_setup(n_gpus):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(0)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+# workload
+# ---------------------------------------------------------------------------
+
+def setup_workload(args, device):
+    import torch
+    from paper_2609_29505_gb300 import schedule, synth
+    cfg = synth.get_config(args.config)
+    T = args.T or cfg.T
+    t0 = time.time()
+    weights = synth.make_weights(cfg, device)
+    inp = synth.make_inputs(cfg, device)
+    torch.cuda.synchronize()
+    t_w = time.time() - t0
+    t0 = time.time()
+    sched = schedule.build_schedule(cfg, weights, T, budget=args.budget)
+    t_s = time.time() - t0
+    return cfg, T, weights, inp, sched, dict(weights_s=round(t_w, 1), schedule_s=round(t_s, 1))
+
+
+def step_inputs(cfg, inp, T, device):
+    """Per-step device inputs for positions s = 1..T (token models: reveal schedule;
+    continuous models: the seeded initial state, held fixed)."""
+    import torch
+    from paper_2609_29505_gb300 import synth
+    if cfg.stem == "embed":
+        return [synth.token_ids_at(cfg, inp, s, T).to(device).contiguous() for s in range(1, T + 1)]
+    z = inp.z0.to(device).contiguous()
+    return [z for _ in range(T)]
+
+
+def out_buffer(cfg, device, pinned=False):
+    import torch
+    if cfg.head == "logits":
+        shape, dt = (cfg.batch, cfg.n_tokens, cfg.d_out), torch.float16
+    elif cfg.head == "identity":
+        shape, dt = (cfg.batch, cfg.n_tokens, cfg.d), torch.float32
+    else:
+        shape, dt = (cfg.batch, cfg.n_out_tokens, cfg.out_channels), torch.float32
+    if device == "cpu":
+        t = torch.empty(shape, dtype=dt)
+        return t.pin_memory() if pinned else t
+    return torch.empty(shape, dtype=dt, device=device)
+
+
+def run_native(args):
+    import torch
+    from paper_2609_29505_gb300 import binding, build
+
+    build.build()
+    rank, world, local = dist_setup(args.gpus)
+    dev = torch.device("cuda", local if world > 1 else 0)
+    peaks = load_peaks()
+    cfg, T, weights, inp, sched, setup_t = setup_workload(args, dev)
+    K = args.steps if args.steps is not None else T
+    W = args.warmup if args.warmup is not None else T
+    W = max(W, 3)
+    model = binding.Denoiser(cfg, weights)
+    t0 = time.time()
+    model.set_schedule(T, sched["lifetimes"], sched["groups"])
+    setup_t["capture_s"] = round(time.time() - t0, 2)
+    info = model.info()
+    xs = step_inputs(cfg, inp, T, dev)
+    cls = None if inp.class_ids is None else inp.class_ids.to(dev)
+    ctx = None if inp.ctx is None else inp.ctx.to(dev)
+    out = out_buffer(cfg, dev)
+    stream = torch.cuda.current_stream()
+    from paper_2609_29505_gb300.synth import timestep
+
+    def run_steps(n, start_fresh=True):
+        if start_fresh:
+            model.reset()
+        for i in range(n):
+            s = i % T + 1
+            model.step(xs[s - 1], out, timestep(cfg, s, T), s, class_ids=cls, ctx=ctx, stream=stream)
+
+    run_steps(W)
+    torch.cuda.synchronize()
+    model.check_device(stream)
+    # timed region: exactly K steps from s = 1
+    model.reset()
+    barrier(world)
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(dev.index if dev.index is not None else 0) as clk:
+        ev0.record(stream)
+        run_steps(K, start_fresh=False)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    ms = ev0.elapsed_time(ev1)
+    ms = max_over_ranks(ms, world)
+    model.check_device(stream)
+    value = K * world / (ms / 1000.0)
+
+    # per-op timing of one trajectory (same kernels, launched op by op with events)
+    recs_by_step = []
+    model.reset()
+    for s in range(1, T + 1):
+        recs_by_step.append(model.profile_step(xs[s - 1], out, timestep(cfg, s, T), s,
+                                               class_ids=cls, ctx=ctx, stream=stream))
+    launches_per_pos = [len(r) + 1 for r in recs_by_step]  # + the per-step I/O-slot kernel
+    gpu_launches = sum(launches_per_pos[i % T] for i in range(K))
+    if cfg.block == "xattn":
+        gpu_launches += cfg.n_blocks * ((K + T - 1) // T)  # context K/V at each s = 1
+    by_kernel = {}
+    tot_flops = tot_bytes = tot_ms = 0.0
+    for recs in recs_by_step:
+        for r in recs:
+            k = by_kernel.setdefault(r["kernel"], dict(ms=0.0, flops=0.0, bytes=0.0, launches=0))
+            k["ms"] += r["ms"]
+            k["flops"] += r["flops"]
+            k["bytes"] += r["bytes"]
+            k["launches"] += 1
+            tot_flops += r["flops"]
+            tot_bytes += r["bytes"]
+            tot_ms += r["ms"]
+    gemm = by_kernel.get("gemm_tc", by_kernel.get("gemm_simt"))
+    achieved = gemm["flops"] / (gemm["ms"] / 1e3) / 1e12
+    roofline = {"bound": "tensor", "kernel": "gemm_tcgen05", "achieved": round(achieved, 1),
+                "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
+                "frac": round(achieved / peaks["bf16_sus"], 4),
+                "peak_source": f"{peaks['source']} bf16 sustained", "traffic": None,
+                "launches_per_trajectory": gemm["launches"],
+                "share_of_step": round(gemm["ms"] / tot_ms, 3)}
+    fz = by_kernel.get("frozen_run")
+    # whole-step roofline: max(FLOPs / bf16 peak, bytes / HBM peak) per step vs measured
+    t_roof = max(tot_flops / (peaks["bf16_sus"] * 1e12), tot_bytes / (peaks["hbm"] * 1e9)) / T
+    step_roof = {"t_roofline_ms": round(t_roof * 1e3, 3), "t_measured_ms": round(ms / K, 3),
+                 "frac": round(t_roof * 1e3 / (ms / K), 4),
+                 "flops_per_step": tot_flops / T, "bytes_per_step": tot_bytes / T,
+                 "roofline_steps_per_s": round(1.0 / t_roof, 2)}
+    kernels = {k: {"launches": v["launches"], "ms_per_traj": round(v["ms"], 3),
+                   "share": round(v["ms"] / tot_ms, 4),
+                   "tflops": round(v["flops"] / max(v["ms"], 1e-9) / 1e9, 1),
+                   "gbs": round(v["bytes"] / max(v["ms"], 1e-9) / 1e6, 1)} for k, v in by_kernel.items()}
+    if fz:
+        kernels["frozen_run"]["frac_of_hbm"] = round(fz["bytes"] / (fz["ms"] / 1e3) / 1e9 / peaks["hbm"], 4)
+
+    # end to end through the C ABI with host buffers (pinned), copies inside the region
+    e2e = None
+    if not args.no_e2e:
+        import torch as _t
+        xs_h = [x.cpu().pin_memory() for x in xs[:T]]
+        out_h = out_buffer(cfg, "cpu", pinned=True)
+        cls_h = None if inp.class_ids is None else inp.class_ids.cpu().pin_memory()
+        ctx_h = None if inp.ctx is None else inp.ctx.cpu().pin_memory()
+        model.reset()
+        barrier(world)
+        _t.cuda.synchronize()
+        t0 = time.perf_counter()
+        for i in range(K):
+            s = i % T + 1
+            model.step_host(xs_h[s - 1], out_h, timestep(cfg, s, T), s, class_ids_host=cls_h,
+                            ctx_host=ctx_h, stream=stream)
+        _t.cuda.synchronize()
+        e2e_s = max_over_ranks(time.perf_counter() - t0, world)
+        h2d = xs_h[0].numel() * xs_h[0].element_size() + (0 if cls_h is None else cls_h.numel() * 4)
+        e2e = {"value": round(K * world / e2e_s, 3), "unit": "steps/s", "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(out_h.numel() * out_h.element_size())}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(cfg, T, weights, inp, sched, n_steps=4)
+
+    model.close()
+    res = {
+        "metric": METRIC if args.budget == 0.5 else METRIC.replace("50%", f"{args.budget:.0%}"),
+        "value": round(value, 3), "unit": "steps/s", "n_gpus": world, "steps": K, "warmup": W,
+        "ms_per_step": round(ms / K, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": workload_name(cfg, T, args.budget), "batch": cfg.batch,
+                   "seq_len": cfg.n_tokens, "T": T, "budget": args.budget,
+                   "achieved_layer_step_ratio": round(sched["ratio"], 4),
+                   "tokens_per_s": round(value * cfg.batch * cfg.n_tokens, 1),
+                   "parallelism": f"replicas{world}" if world > 1 else "single",
+                   "l2": "inputs larger than L2 (bf16 weights ~16 GB per step)",
+                   "n_patterns": info["n_patterns"], "n_graphs": info["n_graphs"],
+                   "cache_gb": round(info["cache_bytes"] / 2 ** 30, 2), "setup": setup_t},
+        "roofline": roofline, "step_roofline": step_roof, "kernels": kernels,
+        "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(gpu_launches),
+        "clocks": clk.summary(),
+    }
+    if rank == 0:
+        print(json.dumps(res), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def workload_name(cfg, T, budget):
+    names = {"llada": "LLaDA-8B-shaped", "dit": "DiT-XL/2-shaped", "uvit": "U-ViT-L-shaped",
+             "sdxl": "SDXL-transformer-shaped", "tiny": "tiny pre-norm"}
+    return (f"{names.get(cfg.name, cfg.name)} B={cfg.batch} N={cfg.n_tokens} d={cfg.d} "
+            f"L={cfg.n_blocks} T={T} budget={budget:.0%}")
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline and the reference arm)
+# ---------------------------------------------------------------------------
+
+TOKEN_SAMPLE = 128
+
+
+def oracle_sample(cfg, T, weights, inp, sched):
+    """Bounded sample of the workload for the CPU oracle: batch row 0 and, for token
+    models, its first TOKEN_SAMPLE positions (full depth, width and head).  Returns the
+    oracle model config, fp32 weights, a state function and the scale factor from
+    sample steps/s to workload steps/s."""
+    import numpy as np
+    from oracle import denoiser as odn
+    from paper_2609_29505_gb300 import synth
+    W = {k: v.detach().float().cpu().numpy() for k, v in weights.items()}
+    if cfg.stem == "embed":
+        n = min(TOKEN_SAMPLE, cfg.n_tokens)
+        ocfg = cfg.with_(batch=1, n_tokens=n)
+        state = lambda s: synth.token_ids_at(cfg, inp, s, T)[:1, :n].cpu().numpy()
+        scale = (n / cfg.n_tokens) / cfg.batch
+        desc = f"batch row 0 of {cfg.batch}, first {n} of {cfg.n_tokens} tokens, all layers"
+    else:
+        ocfg = cfg.with_(batch=1)
+        z0 = inp.z0[:1].cpu().numpy()
+        state = lambda s: z0
+        scale = 1.0 / cfg.batch
+        desc = f"batch row 0 of {cfg.batch}, all tokens and layers"
+    cls = None if inp.class_ids is None else inp.class_ids[:1].cpu().numpy()
+    ctx = None if inp.ctx is None else inp.ctx[:1].float().cpu().numpy()
+    return ocfg, W, state, scale, cls, ctx, desc
+
+
+def cpu_threads():
+    try:
+        import threadpoolctl
+        info = threadpoolctl.threadpool_info()
+        return max((i.get("num_threads", 1) for i in info), default=os.cpu_count())
+    except Exception:
+        return os.cpu_count()
+
+
+def cpu_baseline(cfg, T, weights, inp, sched, n_steps=4, oracle_ctx=None):
+    """Oracle steps/s on the host cores for a bounded sample (about 10-30 s of work)."""
+    from oracle import trajectory as otj
+    ocfg, W, state, scale, cls, ctx, desc = oracle_ctx or oracle_sample(cfg, T, weights, inp, sched)
+    S = sched["lifetimes"]
+    # trajectory positions spread evenly over the horizon
+    steps = sorted({max(1, round((i + 0.5) * T / n_steps)) for i in range(n_steps)})
+    times = otj.time_steps(ocfg, W, S, T, steps, state, cls, ctx)
+    per_step = sum(times) / len(times)
+    return {"value": round(scale / per_step, 5), "unit": "steps/s", "cores": cpu_threads(),
+            "kind": "oracle",
+            "sample": f"{desc}; steps {steps} of T={T}, mean {per_step:.2f} s/step, "
+                      f"scaled by {1 / scale:g}x to the full batch"}
+
+
+def run_reference(args):
+    """--impl reference: the CPU oracle timed on the host cores (rank 0 only)."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import torch
+    from paper_2609_29505_gb300 import synth
+    from oracle import trajectory as otj
+    cfg = synth.get_config(args.config)
+    T = args.T or cfg.T
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    cfg0, T, weights, inp, sched, _ = setup_workload(args, dev)
+    K = args.steps if args.steps is not None else T
+    W = args.warmup if args.warmup is not None else 1
+    octx = oracle_sample(cfg0, T, weights, inp, sched)
+    ocfg, Wn, state, scale, cls, ctx, desc = octx
+    del weights
+    S = sched["lifetimes"]
+    otj.time_steps(ocfg, Wn, S, T, [i % T + 1 for i in range(W)], state, cls, ctx)
+    t0 = time.perf_counter()
+    otj.time_steps(ocfg, Wn, S, T, [i % T + 1 for i in range(K)], state, cls, ctx)
+    el = time.perf_counter() - t0
+    value = scale * K / el
+    res = {"impl": "reference", "metric": METRIC if args.budget == 0.5 else
+           METRIC.replace("50%", f"{args.budget:.0%}"), "value": round(value, 5), "unit": "steps/s",
+           "n_gpus": 1, "steps": K, "warmup": W, "ms_per_step": round(1000.0 / value, 3),
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+           "data": "synthetic",
+           "config": {"workload": workload_name(cfg0, T, args.budget), "batch": cfg0.batch,
+                      "seq_len": cfg0.n_tokens, "T": T, "budget": args.budget},
+           "cpu_baseline": {"value": round(value, 5), "unit": "steps/s", "cores": cpu_threads(),
+                            "kind": "oracle", "sample": desc + f"; scaled by {1 / scale:g}x"},
+           "e2e": {"value": round(value, 5), "unit": "steps/s", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(res), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_native(args)
+
+
+if __name__ == "__main__":
+    main()

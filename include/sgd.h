@@ -20,8 +20,12 @@
  *   - Every function returns an sgd_status (0 = success, negative = error) and never
  *     aborts or throws.  On error, sgd_last_error() describes it.
  *   - A context is not thread-safe: calls on one context must be serialised.
- *   - All weights are bf16, row-major [out, in] for linear maps; activations are
- *     computed in bf16 with fp32 accumulation; the residual stream h is fp32.
+ *   - All weights are passed as bf16, row-major [out, in] for linear maps.  At
+ *     sgd_create the projection weights are converted once into library-owned fp16
+ *     copies scaled by a power of two (exact for every entry in fp16's normal range);
+ *     the tensor cores then multiply fp16 operands with fp32 accumulation (same
+ *     tcgen05 kind::f16 rate as bf16, 8x finer operand rounding).  Activations
+ *     between kernels are fp16, the residual stream h and all reductions fp32.
  */
 #ifndef SGD_H
 #define SGD_H
@@ -78,7 +82,7 @@ typedef enum {
   SGD_HEAD_LINEAR = 0,       /* norm_f then W_head; fp32 out [B, N - n_prefix, out_channels] */
   SGD_HEAD_ADALN_LINEAR = 1, /* AdaLN(final) then W_head; fp32 out, first out_channels      */
   SGD_HEAD_IDENTITY = 2,     /* out = h_L; fp32 [B, N, d]                                  */
-  SGD_HEAD_LOGITS = 3        /* RMSNorm then W_head; bf16 logits [B, N, d_out]            */
+  SGD_HEAD_LOGITS = 3        /* RMSNorm then W_head; fp16 logits [B, N, d_out]            */
 } sgd_head_kind;
 
 /* Debug flag: run every GEMM on the plain SIMT kernel instead of tcgen05. */
@@ -141,17 +145,19 @@ typedef struct {
   int n_graphs;         /* captured graphs (patterns x cache-refresh variants)   */
   int T;                /* horizon of the current schedule (0 if none)            */
   int64_t layer_steps;  /* sum over steps of active units                         */
-  size_t cache_bytes;   /* device bytes of the per-unit update caches             */
+  size_t cache_bytes;   /* device bytes of the per-unit update caches (fp16)      */
   size_t workspace_bytes;
+  size_t weight_bytes;  /* device bytes of the library's fp16 projection weights  */
 } sgd_info;
 
 typedef struct sgd_ctx sgd_ctx;
 
 /*
- * sgd_create — validate the model shape, borrow the weights, allocate caches and
- * workspaces on the current device, build TMA descriptors.
- * desc, w: host structs (copied).  Weight pointers: device, must stay valid and
- * unchanged for the context's lifetime, 16-byte aligned.
+ * sgd_create — validate the model shape, borrow the weights, make the fp16 projection
+ * copies, allocate caches and workspaces on the current device.
+ * desc, w: host structs (copied).  Weight pointers: device, 16-byte aligned; norm
+ * gains, embeddings, stem, conditioning and small-head weights are read in place and
+ * must stay valid and unchanged for the context's lifetime.
  * Errors: SGD_ERR_ARG (null/misaligned), SGD_ERR_SHAPE, SGD_ERR_OOM, SGD_ERR_CUDA.
  */
 int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out);
@@ -174,7 +180,7 @@ int sgd_set_schedule(sgd_ctx* ctx, int T, int n_units, const int32_t* lifetimes_
  * sgd_step — one denoiser evaluation at step `step` (Algorithm 2), asynchronous on
  * `stream` (a cudaStream_t).  step must be 1 (starts a trajectory) or last_step + 1.
  * state_in_dev: fp32 [B, N_in, d_in], or int32 ids [B, N] for SGD_STEM_EMBED.
- * out_dev: fp32 [B, N_out, out_channels] or bf16 logits [B, N, d_out].
+ * out_dev: fp32 [B, N_out, out_channels] or fp16 logits [B, N, d_out].
  * timestep: t_s fed to the stem / conditioning.  cond: see sgd_cond (may be NULL).
  * Errors: SGD_ERR_STATE (no schedule), SGD_ERR_CACHE_INVALID (out-of-order step),
  * SGD_ERR_ARG, SGD_ERR_CUDA.  Kernel timeouts surface through sgd_check_device.

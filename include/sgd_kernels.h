@@ -29,20 +29,22 @@ extern "C" {
 #endif
 
 /* Epilogue applied to the fp32 accumulator tile of C = A B^T. */
+/* acc = alpha * (A B^T), fp32.  fp16 outputs saturate at +-65504. */
 typedef enum {
-  SGD_EPI_BF16 = 0,   /* out bf16 [M, N] = acc                                          */
+  SGD_EPI_F16 = 0,    /* out fp16 [M, N] = acc                                          */
   SGD_EPI_F32 = 1,    /* out fp32 [M, N] = acc                                          */
-  SGD_EPI_DELTA = 2,  /* Delta = gate * acc; h fp32 [M, N] += Delta; cache bf16 = Delta   */
-  SGD_EPI_GATED = 3,  /* B has 2f rows; out bf16 [M, f] = act(acc[:, :f], acc[:, f:])   */
-  SGD_EPI_GELU = 4,   /* out bf16 [M, N] = gelu(acc)                                    */
-  SGD_EPI_ROPE = 5    /* out bf16 [M, N] = acc with rotate-half RoPE on columns < rope_cols */
+  SGD_EPI_DELTA = 2,  /* Delta = gate * acc; h fp32 [M, N] += Delta; cache fp16 = Delta   */
+  SGD_EPI_GATED = 3,  /* B has 2f rows; out fp16 [M, f] = act(acc[:, :f], acc[:, f:])   */
+  SGD_EPI_GELU = 4,   /* out fp16 [M, N] = gelu(acc)                                    */
+  SGD_EPI_ROPE = 5    /* out fp16 [M, N] = acc with rotate-half RoPE on columns < rope_cols */
 } sgd_epilogue_kind;
 
 typedef struct {
   int kind;                      /* sgd_epilogue_kind                                        */
+  float alpha;                   /* accumulator scale (0 is read as 1)                        */
   void* out; int ldo;            /* output (elements); unused by SGD_EPI_DELTA               */
   float* h; int ldh;             /* DELTA: fp32 residual updated in place                   */
-  void* cache; int ld_cache;     /* DELTA: optional bf16 copy of Delta (NULL: not stored)    */
+  void* cache; int ld_cache;     /* DELTA: optional fp16 copy of Delta (NULL: not stored)    */
   const float* gate;             /* DELTA: optional fp32 gate [B, ld_gate], row r uses sample r / rows_per_batch */
   int ld_gate, rows_per_batch;
   int act;                       /* GATED: 0 = silu(a) * b (SwiGLU), 1 = a * gelu_erf(b) (GEGLU);
@@ -53,10 +55,11 @@ typedef struct {
 } sgd_epilogue_args;
 
 /*
- * C = A B^T.  A bf16 [M, K] (row stride lda elements), B bf16 [N or 2N, K] (row
- * stride ldb).  K, lda, ldb multiples of 8; N multiple of 8; pointers 16-byte
+ * C = alpha A B^T.  A fp16 [M, K] (row stride lda elements), B fp16 [N or 2N, K]
+ * (row stride ldb).  K, lda, ldb multiples of 8; N multiple of 8; pointers 16-byte
  * aligned.  use_simt = 1 runs the plain SIMT kernel (reference / debugging), 0 the
- * tcgen05 + TMA kernel.
+ * tcgen05 + TMA kernel (M = 128, N = 256, K = 16 instructions, fp32 accumulators in
+ * TMEM).
  */
 int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
                     const sgd_epilogue_args* epi, int use_simt, void* stream);
@@ -64,7 +67,7 @@ int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N
 /*
  * O = softmax(Q K^T / sqrt(d_head)) V per (sample, head), non-causal, keys beyond n_kv
  * masked.  Row r = b * n_q + i of q / o, row b * n_kv + j of k / v; head h occupies
- * columns [h d_head, (h+1) d_head).  bf16 in and out; d_head in {64, 72, 128};
+ * columns [h d_head, (h+1) d_head).  fp16 in and out; d_head in {64, 72, 128};
  * leading dimensions in elements, multiples of 8.
  */
 int sgd_kernel_attention(const void* q, int ldq, const void* k, const void* v, int ldkv,
@@ -72,7 +75,7 @@ int sgd_kernel_attention(const void* q, int ldq, const void* k, const void* v, i
                          int d_head, void* stream);
 
 /*
- * out bf16 [rows, d] = norm(h fp32 [rows, d]); kind = sgd_norm_kind.  g, b: bf16 [d]
+ * out fp16 [rows, d] = norm(h fp32 [rows, d]); kind = sgd_norm_kind.  g, b: bf16 [d]
  * (NULL allowed for LN_PLAIN).  shift/scale: optional fp32 AdaLN modulation
  * [B, ld_mod]: out = norm(h) * (1 + scale[r / rows_per_batch]) + shift[...].
  */
@@ -81,7 +84,7 @@ int sgd_kernel_norm(const float* h, void* out, int rows, int d, int kind, const 
                     int rows_per_batch, float eps, void* stream);
 
 /*
- * h fp32 [n] += sum_{i < n_caches} caches[i] (bf16 [n]), summed in order i = 0, 1, ...
+ * h fp32 [n] += sum_{i < n_caches} caches[i] (fp16 [n]), summed in order i = 0, 1, ...
  * in fp32.  caches_host: host array of n_caches (<= 96) device pointers.  n multiple
  * of 8, pointers 16-byte aligned.
  */

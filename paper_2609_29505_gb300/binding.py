@@ -37,7 +37,7 @@ MLP = {"swiglu": 0, "gelu_tanh": 1, "gelu_erf": 2, "geglu": 3}
 HEAD = {"linear": 0, "adaln_linear": 1, "identity": 2, "logits": 3}
 FLAG_SIMT_GEMM = 1
 
-EPI_BF16, EPI_F32, EPI_DELTA, EPI_GATED, EPI_GELU, EPI_ROPE = range(6)
+EPI_F16, EPI_F32, EPI_DELTA, EPI_GATED, EPI_GELU, EPI_ROPE = range(6)
 KERNEL_NAMES = ["gemm_tc", "gemm_simt", "attention", "norm", "frozen_run", "small"]
 
 # every symbol include/*.h declares
@@ -78,7 +78,7 @@ class sgd_cond(C.Structure):
 class sgd_info(C.Structure):
     _fields_ = [("n_units", C.c_int), ("n_patterns", C.c_int), ("n_graphs", C.c_int),
                 ("T", C.c_int), ("layer_steps", C.c_int64), ("cache_bytes", C.c_size_t),
-                ("workspace_bytes", C.c_size_t)]
+                ("workspace_bytes", C.c_size_t), ("weight_bytes", C.c_size_t)]
 
 
 class sgd_op_record(C.Structure):
@@ -87,7 +87,8 @@ class sgd_op_record(C.Structure):
 
 
 class sgd_epilogue_args(C.Structure):
-    _fields_ = [("kind", C.c_int), ("out", C.c_void_p), ("ldo", C.c_int), ("h", C.c_void_p),
+    _fields_ = [("kind", C.c_int), ("alpha", C.c_float), ("out", C.c_void_p), ("ldo", C.c_int),
+                ("h", C.c_void_p),
                 ("ldh", C.c_int), ("cache", C.c_void_p), ("ld_cache", C.c_int),
                 ("gate", C.c_void_p), ("ld_gate", C.c_int), ("rows_per_batch", C.c_int),
                 ("act", C.c_int), ("rope_cos", C.c_void_p), ("rope_sin", C.c_void_p),

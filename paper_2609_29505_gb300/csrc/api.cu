@@ -102,8 +102,24 @@ void compile_patterns(int T, int n_units, const int32_t* S, std::vector<int>& pa
 
 }  // namespace
 
+// A GEMM weight as the tensor cores read it: fp16 copy of the user's bf16 matrix scaled
+// by 2^shift (exact conversion), with alpha = 2^-shift applied to the accumulator.
+struct PW {
+  const f16* w = nullptr;
+  float alpha = 1.f;
+};
+
+struct BlockPW {
+  PW qkv, o, xq, xkv, xo, w1, w2;
+};
+
 struct sgd_ctx {
   sgd_model_desc d{};
+  std::vector<BlockPW> pw;
+  std::vector<PW> pw_skip;
+  PW pw_head;
+  float* absmax = nullptr;
+  f16* ctx16 = nullptr;
   std::vector<sgd_block_weights> blk;
   std::vector<const bf16*> skip_w;
   sgd_weights w{};
@@ -111,10 +127,10 @@ struct sgd_ctx {
   int M = 0, U = 0, nbr = 0;
   // buffers
   float* h = nullptr;
-  bf16* xn = nullptr;
-  bf16* qkv = nullptr;
-  bf16* attn = nullptr;
-  bf16* act = nullptr;
+  f16* xn = nullptr;
+  f16* qkv = nullptr;
+  f16* attn = nullptr;
+  f16* act = nullptr;
   float* t_hidden = nullptr;
   float* cond_c = nullptr;
   float* mod = nullptr;
@@ -122,11 +138,11 @@ struct sgd_ctx {
   float* rope_cos = nullptr;
   float* rope_sin = nullptr;
   IoSlot* slot = nullptr;
-  std::vector<bf16*> cache;
-  std::vector<bf16*> ctxkv;
-  std::vector<bf16*> skipcat;
+  std::vector<f16*> cache;
+  std::vector<f16*> ctxkv;
+  std::vector<f16*> skipcat;
   std::vector<void*> allocs;
-  size_t cache_bytes = 0, ws_bytes = 0;
+  size_t cache_bytes = 0, ws_bytes = 0, weight_bytes = 0;
   // schedule
   int T = 0;
   std::vector<int32_t> S, groups;
@@ -171,7 +187,7 @@ struct sgd_ctx {
     return static_cast<size_t>(d.batch) * (d.n_tokens - d.n_prefix) * d.d_in * 4;
   }
   size_t out_bytes() const {
-    if (d.head == SGD_HEAD_LOGITS) return static_cast<size_t>(M) * d.d_out * 2;
+    if (d.head == SGD_HEAD_LOGITS) return static_cast<size_t>(M) * d.d_out * 2;  // fp16 logits
     if (d.head == SGD_HEAD_IDENTITY) return static_cast<size_t>(M) * d.d * 4;
     return static_cast<size_t>(d.batch) * (d.n_tokens - d.n_prefix) * d.out_channels * 4;
   }
@@ -180,17 +196,19 @@ struct sgd_ctx {
 namespace {
 
 const bf16* B16(const void* p) { return static_cast<const bf16*>(p); }
+const f16* H16(const void* p) { return static_cast<const f16*>(p); }
 
 // ---------------------------------------------------------------------------
 // op builders
 // ---------------------------------------------------------------------------
 
-int make_gemm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, const bf16* A,
-                 int lda, const bf16* B, int ldb, int M, int N, int K, const EpiParams& epi) {
+int make_gemm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, const f16* A,
+                 int lda, const PW& B, int ldb, int M, int N, int K, EpiParams epi) {
+  epi.alpha = B.alpha;
   auto plan = std::make_shared<GemmPlan>();
   plan->A = A;
   plan->lda = lda;
-  plan->B = B;
+  plan->B = B.w;
   plan->ldb = ldb;
   plan->M = M;
   plan->N = N;
@@ -220,6 +238,7 @@ int make_gemm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, cons
 EpiParams epi_base(int kind) {
   EpiParams e{};
   e.kind = kind;
+  e.alpha = 1.f;
   e.rows_per_batch = 1;
   return e;
 }
@@ -272,7 +291,7 @@ void make_gemv_op(std::vector<Op>& ops, const std::string& name, const GemvParam
   ops.push_back(std::move(op));
 }
 
-void flush_run(sgd_ctx* c, std::vector<Op>& ops, std::vector<const bf16*>& run, int first_unit) {
+void flush_run(sgd_ctx* c, std::vector<Op>& ops, std::vector<const f16*>& run, int first_unit) {
   size_t i = 0;
   while (i < run.size()) {
     FrozenParams p{};
@@ -294,11 +313,12 @@ void flush_run(sgd_ctx* c, std::vector<Op>& ops, std::vector<const bf16*>& run, 
 int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_cache, int u) {
   const sgd_model_desc& d = c->d;
   const sgd_block_weights& W = c->blk[b];
+  const BlockPW& P = c->pw[b];
   const int M = c->M, D = d.d, F = d.d_ff;
   const std::string pre = "b" + std::to_string(b) + ".";
   const bool adaln = d.block == SGD_BLOCK_ADALN;
   float* mod = adaln ? c->mod + static_cast<size_t>(b) * d.batch * 6 * D : nullptr;
-  bf16* cache = write_cache ? c->cache[u] : nullptr;
+  f16* cache = write_cache ? c->cache[u] : nullptr;
   EpiParams delta = epi_base(SGD_EPI_DELTA);
   delta.h = c->h;
   delta.ldh = D;
@@ -308,7 +328,7 @@ int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_c
   if (kind == 0) {  // self-attention
     make_norm_op(c, ops, pre + "attn.norm", d.norm, W.norm1_w, W.norm1_b, adaln ? mod : nullptr,
                  adaln ? mod + D : nullptr, 6 * D);
-    EpiParams e = epi_base(d.rope ? SGD_EPI_ROPE : SGD_EPI_BF16);
+    EpiParams e = epi_base(d.rope ? SGD_EPI_ROPE : SGD_EPI_F16);
     e.out = c->qkv;
     e.ldo = 3 * D;
     if (d.rope) {
@@ -318,7 +338,7 @@ int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_c
       e.d_head = d.d_head;
       e.rope_cols = 2 * D;
     }
-    if ((rc = make_gemm_op(c, ops, pre + "attn.qkv", c->xn, D, B16(W.w_qkv), D, M, 3 * D, D, e)))
+    if ((rc = make_gemm_op(c, ops, pre + "attn.qkv", c->xn, D, P.qkv, D, M, 3 * D, D, e)))
       return rc;
     AttnParams ap{c->qkv, 3 * D, c->qkv + D, c->qkv + 2 * D, 3 * D, c->attn, D,
                   d.batch, d.n_tokens, d.n_tokens, d.n_heads, d.d_head};
@@ -328,18 +348,18 @@ int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_c
       delta.ld_gate = 6 * D;
       delta.rows_per_batch = d.n_tokens;
     }
-    return make_gemm_op(c, ops, pre + "attn.out", c->attn, D, B16(W.w_o), D, M, D, D, delta);
+    return make_gemm_op(c, ops, pre + "attn.out", c->attn, D, P.o, D, M, D, D, delta);
   }
   if (kind == 1) {  // cross-attention
     make_norm_op(c, ops, pre + "xattn.norm", SGD_NORM_LN, W.normx_w, W.normx_b, nullptr, nullptr, 0);
-    EpiParams e = epi_base(SGD_EPI_BF16);
+    EpiParams e = epi_base(SGD_EPI_F16);
     e.out = c->qkv;
     e.ldo = D;
-    if ((rc = make_gemm_op(c, ops, pre + "xattn.q", c->xn, D, B16(W.wx_q), D, M, D, D, e))) return rc;
+    if ((rc = make_gemm_op(c, ops, pre + "xattn.q", c->xn, D, P.xq, D, M, D, D, e))) return rc;
     AttnParams ap{c->qkv, D, c->ctxkv[b], c->ctxkv[b] + D, 2 * D, c->attn, D,
                   d.batch, d.n_tokens, d.ctx_len, d.n_heads, d.d_head};
     if ((rc = make_attn_op(c, ops, pre + "xattn.sdpa", ap))) return rc;
-    return make_gemm_op(c, ops, pre + "xattn.out", c->attn, D, B16(W.wx_o), D, M, D, D, delta);
+    return make_gemm_op(c, ops, pre + "xattn.out", c->attn, D, P.xo, D, M, D, D, delta);
   }
   // MLP
   make_norm_op(c, ops, pre + "mlp.norm", d.norm, W.norm2_w, W.norm2_b, adaln ? mod + 3 * D : nullptr,
@@ -349,13 +369,13 @@ int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_c
   e.out = c->act;
   e.ldo = F;
   e.act = (d.mlp == SGD_MLP_GEGLU || d.mlp == SGD_MLP_GELU_ERF) ? 1 : 0;
-  if ((rc = make_gemm_op(c, ops, pre + "mlp.up", c->xn, D, B16(W.w_1), D, M, F, D, e))) return rc;
+  if ((rc = make_gemm_op(c, ops, pre + "mlp.up", c->xn, D, P.w1, D, M, F, D, e))) return rc;
   if (adaln) {
     delta.gate = mod + 5 * D;
     delta.ld_gate = 6 * D;
     delta.rows_per_batch = d.n_tokens;
   }
-  return make_gemm_op(c, ops, pre + "mlp.down", c->act, F, B16(W.w_2), F, M, D, F, delta);
+  return make_gemm_op(c, ops, pre + "mlp.down", c->act, F, P.w2, F, M, D, F, delta);
 }
 
 int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vector<uint8_t>& write,
@@ -378,6 +398,8 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
     p.pos = B16(c->w.pos_emb);
     p.class_emb = B16(c->w.class_emb);
     p.embed = B16(c->w.embed);
+    p.vocab = d.vocab;
+    p.n_classes = d.n_classes;
     Op op;
     op.name = "stem";
     op.kernel = SGD_KERNEL_SMALL;
@@ -410,6 +432,7 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
     g2.K = D;
     g2.rows = d.batch;
     g2.add_class = B16(c->w.class_emb);
+    g2.n_classes = d.n_classes;
     make_gemv_op(ops, "cond.t2", g2);
     for (int b = 0; b < d.n_blocks; ++b) {
       bool any = false;
@@ -429,14 +452,14 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
       make_gemv_op(ops, "b" + std::to_string(b) + ".mod", gm);
     }
   }
-  std::vector<const bf16*> run;
+  std::vector<const f16*> run;
   int run_first = 0;
   int u = 0;
   for (int b = 0; b < d.n_blocks; ++b) {
     if (d.n_skips && b > d.n_skips) {  // U-ViT deep block: h = W_skip [h; skip]
       flush_run(c, ops, run, run_first);
       const int j = b - d.n_skips - 1;
-      bf16* cat = c->skipcat[j];
+      f16* cat = c->skipcat[j];
       const float* hh = c->h;
       const int Mr = M;
       Op op;
@@ -444,13 +467,13 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
       op.kernel = SGD_KERNEL_SMALL;
       op.flops = 0;
       op.bytes = 6.0 * M * D;
-      op.run = [cat, hh, Mr, D](cudaStream_t s) { return pack_bf16_launch(cat, 2 * D, 0, hh, Mr, D, s); };
+      op.run = [cat, hh, Mr, D](cudaStream_t s) { return pack_f16_launch(cat, 2 * D, 0, hh, Mr, D, s); };
       ops.push_back(std::move(op));
       EpiParams e = epi_base(SGD_EPI_F32);
       e.out = c->h;
       e.ldo = D;
       if ((rc = make_gemm_op(c, ops, "b" + std::to_string(b) + ".skip_linear", cat, 2 * D,
-                             c->skip_w[j], 2 * D, M, D, 2 * D, e)))
+                             c->pw_skip[j], 2 * D, M, D, 2 * D, e)))
         return rc;
     }
     for (int k = 0; k < c->nbr; ++k, ++u) {
@@ -465,7 +488,7 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
     }
     if (d.n_skips && b < d.n_skips) {  // U-ViT shallow block: push the current h
       flush_run(c, ops, run, run_first);
-      bf16* cat = c->skipcat[d.n_skips - 1 - b];
+      f16* cat = c->skipcat[d.n_skips - 1 - b];
       const float* hh = c->h;
       const int Mr = M;
       Op op;
@@ -473,7 +496,7 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
       op.kernel = SGD_KERNEL_SMALL;
       op.flops = 0;
       op.bytes = 6.0 * M * D;
-      op.run = [cat, hh, Mr, D](cudaStream_t s) { return pack_bf16_launch(cat, 2 * D, D, hh, Mr, D, s); };
+      op.run = [cat, hh, Mr, D](cudaStream_t s) { return pack_f16_launch(cat, 2 * D, D, hh, Mr, D, s); };
       ops.push_back(std::move(op));
     }
   }
@@ -532,10 +555,10 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
     ops.push_back(std::move(op));
     return SGD_OK;
   }
-  EpiParams e = epi_base(d.head == SGD_HEAD_LOGITS ? SGD_EPI_BF16 : SGD_EPI_F32);
+  EpiParams e = epi_base(d.head == SGD_HEAD_LOGITS ? SGD_EPI_F16 : SGD_EPI_F32);
   e.out_slot = out_slot;
   e.ldo = d.head == SGD_HEAD_LOGITS ? d.d_out : d.out_channels;
-  return make_gemm_op(c, ops, "head.linear", c->xn, D, B16(c->w.w_head), D, M, d.d_out, D, e);
+  return make_gemm_op(c, ops, "head.linear", c->xn, D, c->pw_head, D, M, d.d_out, D, e);
 }
 
 int run_ops(const std::vector<Op>& ops, cudaStream_t s) {
@@ -640,6 +663,7 @@ int ensure_alloc(sgd_ctx* c) {
     if ((rc = c->alloc(&c->modf, d.batch * 2 * D, &c->ws_bytes))) return rc;
   }
   if (d.block == SGD_BLOCK_XATTN) {
+    if ((rc = c->alloc(&c->ctx16, static_cast<size_t>(d.batch) * d.ctx_len * d.d_ctx, &c->ws_bytes))) return rc;
     c->ctxkv.assign(d.n_blocks, nullptr);
     for (int b = 0; b < d.n_blocks; ++b)
       if ((rc = c->alloc(&c->ctxkv[b], static_cast<size_t>(d.batch) * d.ctx_len * 2 * D, &c->ws_bytes))) return rc;
@@ -667,6 +691,57 @@ int ensure_alloc(sgd_ctx* c) {
   return SGD_OK;
 }
 
+// fp16 copy of a bf16 [rows, cols] weight, scaled by the largest power of two that
+// keeps max |w| finite in fp16 (exact conversion of every entry in the normal range).
+int prep_weight(sgd_ctx* c, const void* src, int64_t n, PW& out) {
+  f16* dst = nullptr;
+  int rc = c->alloc(&dst, static_cast<size_t>(n), &c->weight_bytes);
+  if (rc) return rc;
+  CUDA_TRY(cudaMemset(c->absmax, 0, sizeof(float)));
+  CUDA_TRY(absmax_bf16_launch(B16(src), n, c->absmax, 0));
+  float m = 0.f;
+  CUDA_TRY(cudaMemcpy(&m, c->absmax, sizeof(float), cudaMemcpyDeviceToHost));
+  int shift = 0;
+  if (m > 0.f && std::isfinite(m)) {
+    shift = static_cast<int>(std::floor(std::log2(65504.0 / m)));
+    shift = std::max(-100, std::min(100, shift));
+  }
+  CUDA_TRY(convert_bf16_f16_launch(B16(src), dst, n, shift, 0));
+  out.w = dst;
+  out.alpha = std::ldexp(1.0f, -shift);
+  return SGD_OK;
+}
+
+int prep_weights(sgd_ctx* c) {
+  const sgd_model_desc& d = c->d;
+  const int64_t D = d.d, F = d.d_ff;
+  const bool gated = d.mlp == SGD_MLP_SWIGLU || d.mlp == SGD_MLP_GEGLU;
+  int rc;
+  if ((rc = c->alloc(&c->absmax, 1, &c->ws_bytes))) return rc;
+  c->pw.assign(d.n_blocks, BlockPW{});
+  for (int b = 0; b < d.n_blocks; ++b) {
+    const sgd_block_weights& W = c->blk[b];
+    BlockPW& P = c->pw[b];
+    if ((rc = prep_weight(c, W.w_qkv, 3 * D * D, P.qkv))) return rc;
+    if ((rc = prep_weight(c, W.w_o, D * D, P.o))) return rc;
+    if ((rc = prep_weight(c, W.w_1, (gated ? 2 : 1) * F * D, P.w1))) return rc;
+    if ((rc = prep_weight(c, W.w_2, D * F, P.w2))) return rc;
+    if (d.block == SGD_BLOCK_XATTN) {
+      if ((rc = prep_weight(c, W.wx_q, D * D, P.xq))) return rc;
+      if ((rc = prep_weight(c, W.wx_kv, 2 * D * d.d_ctx, P.xkv))) return rc;
+      if ((rc = prep_weight(c, W.wx_o, D * D, P.xo))) return rc;
+    }
+  }
+  c->pw_skip.assign(d.n_skips, PW{});
+  for (int j = 0; j < d.n_skips; ++j)
+    if ((rc = prep_weight(c, c->skip_w[j], D * 2 * D, c->pw_skip[j]))) return rc;
+  const bool tc_head = d.head == SGD_HEAD_LOGITS || (d.head == SGD_HEAD_LINEAR && d.d_out > 64);
+  if (tc_head && (rc = prep_weight(c, c->w.w_head, static_cast<int64_t>(d.d_out) * D, c->pw_head)))
+    return rc;
+  CUDA_TRY(cudaDeviceSynchronize());
+  return SGD_OK;
+}
+
 void drop_graphs(sgd_ctx* c) {
   for (auto e : c->execs) cudaGraphExecDestroy(e);
   for (auto g : c->graphs) cudaGraphDestroy(g);
@@ -681,11 +756,11 @@ int ctx_kv_ops(sgd_ctx* c, const void* ctx_dev, std::vector<Op>& ops) {
   const sgd_model_desc& d = c->d;
   ops.clear();
   for (int b = 0; b < d.n_blocks; ++b) {
-    EpiParams e = epi_base(SGD_EPI_BF16);
+    EpiParams e = epi_base(SGD_EPI_F16);
     e.out = c->ctxkv[b];
     e.ldo = 2 * d.d;
-    int rc = make_gemm_op(c, ops, "b" + std::to_string(b) + ".xattn.ctx_kv", B16(ctx_dev), d.d_ctx,
-                          B16(c->blk[b].wx_kv), d.d_ctx, d.batch * d.ctx_len, 2 * d.d, d.d_ctx, e);
+    int rc = make_gemm_op(c, ops, "b" + std::to_string(b) + ".xattn.ctx_kv", c->ctx16, d.d_ctx,
+                          c->pw[b].xkv, d.d_ctx, d.batch * d.ctx_len, 2 * d.d, d.d_ctx, e);
     if (rc) return rc;
   }
   return SGD_OK;
@@ -720,6 +795,8 @@ int prepare_step(sgd_ctx* c, const void* in, void* out, float t, const sgd_cond*
   v.step = step;
   CUDA_TRY(io_set_launch(c->slot, v, s));
   if (step == 1 && c->d.block == SGD_BLOCK_XATTN) {
+    const int64_t n = static_cast<int64_t>(c->d.batch) * c->d.ctx_len * c->d.d_ctx;
+    CUDA_TRY(convert_bf16_f16_launch(B16(cond->ctx), c->ctx16, n, 0, s));
     std::vector<Op> ops;
     int rc = ctx_kv_ops(c, cond->ctx, ops);
     if (rc) return rc;
@@ -758,7 +835,7 @@ int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out) 
   c->M = desc->batch * desc->n_tokens;
   c->nbr = desc->block == SGD_BLOCK_XATTN ? 3 : 2;
   c->U = desc->n_blocks * c->nbr;
-  if ((rc = ensure_alloc(c))) {
+  if ((rc = ensure_alloc(c)) || (rc = prep_weights(c))) {
     delete c;
     return rc;
   }
@@ -945,6 +1022,7 @@ int sgd_get_info(const sgd_ctx* c, sgd_info* info) {
   info->layer_steps = ls;
   info->cache_bytes = c->cache_bytes;
   info->workspace_bytes = c->ws_bytes;
+  info->weight_bytes = c->weight_bytes;
   return SGD_OK;
 }
 
@@ -979,9 +1057,9 @@ int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N
   if (!ea) return fail(SGD_ERR_ARG, "null epilogue");
   if (ea->kind < 0 || ea->kind > SGD_EPI_ROPE) return fail(SGD_ERR_ARG, "bad epilogue kind");
   GemmPlan p;
-  p.A = B16(A);
+  p.A = H16(A);
   p.lda = lda;
-  p.B = B16(B);
+  p.B = H16(B);
   p.ldb = ldb;
   p.M = M;
   p.N = N;
@@ -990,11 +1068,12 @@ int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N
   EpiParams& e = p.epi;
   e = EpiParams{};
   e.kind = ea->kind;
+  e.alpha = ea->alpha != 0.f ? ea->alpha : 1.f;
   e.out = ea->out;
   e.ldo = ea->ldo;
   e.h = ea->h;
   e.ldh = ea->ldh;
-  e.cache = static_cast<bf16*>(ea->cache);
+  e.cache = static_cast<f16*>(ea->cache);
   e.ld_cache = ea->ld_cache;
   e.gate = ea->gate;
   e.ld_gate = ea->ld_gate;
@@ -1016,7 +1095,7 @@ int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N
 
 int sgd_kernel_attention(const void* q, int ldq, const void* k, const void* v, int ldkv, void* o,
                          int ldo, int batch, int n_q, int n_kv, int n_heads, int d_head, void* stream) {
-  AttnParams p{B16(q), ldq, B16(k), B16(v), ldkv, static_cast<bf16*>(o), ldo,
+  AttnParams p{H16(q), ldq, H16(k), H16(v), ldkv, static_cast<f16*>(o), ldo,
                batch, n_q, n_kv, n_heads, d_head};
   const char* why = "";
   const int rc = attn_check(p, &why);
@@ -1032,7 +1111,7 @@ int sgd_kernel_norm(const float* h, void* out, int rows, int d, int kind, const 
     return fail(SGD_ERR_ARG, "norm: bad arguments (d must be a multiple of 4, <= 4096)");
   if ((shift == nullptr) != (scale == nullptr) || (shift && rows_per_batch < 1))
     return fail(SGD_ERR_ARG, "norm: shift and scale go together, rows_per_batch >= 1");
-  NormParams p{h, static_cast<bf16*>(out), rows, d, kind, B16(g), B16(b), shift, scale, ld_mod,
+  NormParams p{h, static_cast<f16*>(out), rows, d, kind, B16(g), B16(b), shift, scale, ld_mod,
                rows_per_batch > 0 ? rows_per_batch : 1, eps};
   CUDA_TRY(norm_launch(p, static_cast<cudaStream_t>(stream)));
   return SGD_OK;
@@ -1047,7 +1126,7 @@ int sgd_kernel_frozen_run(float* h, const void* const* caches, int n_caches, int
   p.n_caches = n_caches;
   for (int i = 0; i < n_caches; ++i) {
     if (!caches[i] || !al16(caches[i])) return fail(SGD_ERR_ARG, "frozen_run: null or misaligned cache");
-    p.caches[i] = B16(caches[i]);
+    p.caches[i] = H16(caches[i]);
   }
   CUDA_TRY(frozen_launch(p, static_cast<cudaStream_t>(stream)));
   return SGD_OK;

@@ -5,8 +5,9 @@
 //
 // One CTA = 64 query rows of one (sample, head), 4 warps x 16 rows.  K/V tiles of
 // 64 keys stream through a double-buffered cp.async ring; S = Q K^T and O += P V run
-// on mma.sync m16n8k16 (bf16 in, fp32 accumulate) with an online softmax in
-// registers (exp2 with the scale folded in).  Keys beyond n_kv are masked and their
+// on mma.sync m16n8k16 (fp16 in, fp32 accumulate) with an online softmax in
+// registers (exp2 with the scale folded in).  Q, K, V, P and O are fp16 (m16n8k16
+// f16 x f16 -> f32).  Keys beyond n_kv are masked and their
 // shared-memory rows zero-filled; head dims 72 are padded to 80 in shared memory.
 #include "common.cuh"
 #include "kernels.h"
@@ -42,9 +43,9 @@ __device__ __forceinline__ void ldmatrix_x4_trans(uint32_t* r, const void* p) {
                : "r"(smem_u32(p)));
 }
 
-__device__ __forceinline__ void mma_bf16_16816(float* c, const uint32_t* a, const uint32_t* b) {
+__device__ __forceinline__ void mma_f16_16816(float* c, const uint32_t* a, const uint32_t* b) {
   asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
       "{%8, %9}, {%0, %1, %2, %3};"
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
@@ -57,30 +58,30 @@ __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnParams p) {
   constexpr int kChunks = DH / 8;          // 16-byte chunks of real data per row
   constexpr int kPadChunks = DP / 8;
   extern __shared__ __align__(16) uint8_t smem_raw[];
-  bf16* sQ = reinterpret_cast<bf16*>(smem_raw);
-  bf16* sK = sQ + kBQ * kPitch;            // [2][kBKV][kPitch]
-  bf16* sV = sK + 2 * kBKV * kPitch;       // [2][kBKV][kPitch]
+  f16* sQ = reinterpret_cast<f16*>(smem_raw);
+  f16* sK = sQ + kBQ * kPitch;            // [2][kBKV][kPitch]
+  f16* sV = sK + 2 * kBKV * kPitch;       // [2][kBKV][kPitch]
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
   const int q0 = blockIdx.x * kBQ;
   const int bh = blockIdx.y;
   const int b = bh / p.n_heads, h = bh % p.n_heads;
-  const bf16* qbase = p.q + (static_cast<int64_t>(b) * p.n_q) * p.ldq + h * DH;
-  const bf16* kbase = p.k + (static_cast<int64_t>(b) * p.n_kv) * p.ldkv + h * DH;
-  const bf16* vbase = p.v + (static_cast<int64_t>(b) * p.n_kv) * p.ldkv + h * DH;
+  const f16* qbase = p.q + (static_cast<int64_t>(b) * p.n_q) * p.ldq + h * DH;
+  const f16* kbase = p.k + (static_cast<int64_t>(b) * p.n_kv) * p.ldkv + h * DH;
+  const f16* vbase = p.v + (static_cast<int64_t>(b) * p.n_kv) * p.ldkv + h * DH;
 
   // Q tile
   for (int i = tid; i < kBQ * kPadChunks; i += kWarps * 32) {
     const int r = i / kPadChunks, c = i % kPadChunks;
     const bool ok = (q0 + r) < p.n_q && c < kChunks;
-    const bf16* src = ok ? qbase + static_cast<int64_t>(q0 + r) * p.ldq + c * 8 : p.q;
+    const f16* src = ok ? qbase + static_cast<int64_t>(q0 + r) * p.ldq + c * 8 : p.q;
     cp_async16(sQ + r * kPitch + c * 8, src, ok);
   }
   auto load_kv = [&](int tile, int buf) {
     const int k0 = tile * kBKV;
-    bf16* dk = sK + buf * kBKV * kPitch;
-    bf16* dv = sV + buf * kBKV * kPitch;
+    f16* dk = sK + buf * kBKV * kPitch;
+    f16* dv = sV + buf * kBKV * kPitch;
     for (int i = tid; i < kBKV * kPadChunks; i += kWarps * 32) {
       const int r = i / kPadChunks, c = i % kPadChunks;
       const bool ok = (k0 + r) < p.n_kv && c < kChunks;
@@ -121,8 +122,8 @@ __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnParams p) {
         ldmatrix_x4(qf[ks], sQ + r * kPitch + c);
       }
     }
-    const bf16* tk = sK + buf * kBKV * kPitch;
-    const bf16* tv = sV + buf * kBKV * kPitch;
+    const f16* tk = sK + buf * kBKV * kPitch;
+    const f16* tv = sV + buf * kBKV * kPitch;
     // S = Q K^T : 16 x 64 per warp
     float s[8][4];
 #pragma unroll
@@ -135,8 +136,8 @@ __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnParams p) {
         const int r = np * 16 + (lane & 7) + ((lane >> 4) << 3);
         const int c = ks * 16 + ((lane >> 3) & 1) * 8;
         ldmatrix_x4(kb, tk + r * kPitch + c);
-        mma_bf16_16816(s[2 * np], qf[ks], kb);
-        mma_bf16_16816(s[2 * np + 1], qf[ks], kb + 2);
+        mma_f16_16816(s[2 * np], qf[ks], kb);
+        mma_f16_16816(s[2 * np + 1], qf[ks], kb + 2);
       }
     }
     // mask keys beyond n_kv
@@ -179,8 +180,8 @@ __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnParams p) {
       rs[0] += p0 + p1;
       rs[1] += p2 + p3;
       const int kk = nt >> 1, hi = nt & 1;
-      pf[kk][hi * 2 + 0] = pack_bf16x2(p0, p1);
-      pf[kk][hi * 2 + 1] = pack_bf16x2(p2, p3);
+      pf[kk][hi * 2 + 0] = pack_f16x2(p0, p1);
+      pf[kk][hi * 2 + 1] = pack_f16x2(p2, p3);
     }
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
@@ -204,8 +205,8 @@ __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnParams p) {
         const int r = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
         const int c = np * 16 + (lane >> 4) * 8;
         ldmatrix_x4_trans(vb, tv + r * kPitch + c);
-        mma_bf16_16816(o[2 * np], a, vb);
-        mma_bf16_16816(o[2 * np + 1], a, vb + 2);
+        mma_f16_16816(o[2 * np], a, vb);
+        mma_f16_16816(o[2 * np + 1], a, vb + 2);
       }
     }
     __syncthreads();
@@ -213,17 +214,17 @@ __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnParams p) {
   // normalise and store
   const float inv0 = 1.f / l_r[0], inv1 = 1.f / l_r[1];
   const int row0 = q0 + warp * 16 + g, row1 = row0 + 8;
-  bf16* ob = p.o + (static_cast<int64_t>(b) * p.n_q) * p.ldo + h * DH;
+  f16* ob = p.o + (static_cast<int64_t>(b) * p.n_q) * p.ldo + h * DH;
 #pragma unroll
   for (int nt = 0; nt < NO; ++nt) {
     const int c = nt * 8 + 2 * t4;
     if (c < DH) {
       if (row0 < p.n_q)
         *reinterpret_cast<uint32_t*>(ob + static_cast<int64_t>(row0) * p.ldo + c) =
-            pack_bf16x2(o[nt][0] * inv0, o[nt][1] * inv0);
+            pack_f16x2(o[nt][0] * inv0, o[nt][1] * inv0);
       if (row1 < p.n_q)
         *reinterpret_cast<uint32_t*>(ob + static_cast<int64_t>(row1) * p.ldo + c) =
-            pack_bf16x2(o[nt][2] * inv1, o[nt][3] * inv1);
+            pack_f16x2(o[nt][2] * inv1, o[nt][3] * inv1);
     }
   }
 }

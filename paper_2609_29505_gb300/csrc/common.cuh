@@ -7,11 +7,13 @@
 
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <stdint.h>
 
 namespace sgd {
 
 using bf16 = __nv_bfloat16;
+using f16 = __half;
 
 constexpr uint64_t kWaitTimeoutNs = 2000000000ull;  // 2 s: far above any legitimate wait
 
@@ -40,6 +42,34 @@ __device__ __forceinline__ uint4 pack_bf16x8(const float* f) {
   u.y = pack_bf16x2(f[2], f[3]);
   u.z = pack_bf16x2(f[4], f[5]);
   u.w = pack_bf16x2(f[6], f[7]);
+  return u;
+}
+
+// fp16 operands: values are clamped to the finite fp16 range before rounding so that
+// an out-of-range activation saturates instead of turning into inf / NaN downstream.
+__device__ __forceinline__ float sat_f16(float x) { return fminf(fmaxf(x, -65504.f), 65504.f); }
+
+__device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
+  __half2 v = __floats2half2_rn(sat_f16(lo), sat_f16(hi));
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ void unpack_f16x8(const uint4& u, float* f) {
+  const __half2* p = reinterpret_cast<const __half2*>(&u);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    float2 t = __half22float2(p[i]);
+    f[2 * i] = t.x;
+    f[2 * i + 1] = t.y;
+  }
+}
+
+__device__ __forceinline__ uint4 pack_f16x8(const float* f) {
+  uint4 u;
+  u.x = pack_f16x2(f[0], f[1]);
+  u.y = pack_f16x2(f[2], f[3]);
+  u.z = pack_f16x2(f[4], f[5]);
+  u.w = pack_f16x2(f[6], f[7]);
   return u;
 }
 
@@ -175,8 +205,8 @@ __device__ __forceinline__ void tc_fence_after() {
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-// D[tmem] (+)= A[smem] * B[smem]^T, bf16 x bf16 -> fp32, shape from idesc.
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+// D[tmem] (+)= A[smem] * B[smem]^T, f16 x f16 -> fp32, shape from idesc.
+__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
                                           uint32_t idesc, uint32_t accumulate) {
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
@@ -231,12 +261,12 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
   return d;
 }
 
-// Instruction descriptor of tcgen05.mma kind::f16: fp32 accumulator, bf16 A and B,
-// both K-major, M x N.
-__host__ __device__ constexpr uint32_t umma_idesc_bf16(int M, int N) {
+// Instruction descriptor of tcgen05.mma kind::f16: fp32 accumulator, fp16 A and B
+// (format code 0 in both fields; A and B always share one type), both K-major, M x N.
+__host__ __device__ constexpr uint32_t umma_idesc_f16(int M, int N) {
   return (1u << 4)                                   // D format: f32
-         | (1u << 7)                                 // A format: bf16
-         | (1u << 10)                                // B format: bf16
+         | (0u << 7)                                 // A format: f16
+         | (0u << 10)                                // B format: f16
          | (static_cast<uint32_t>(N >> 3) << 17)     // N / 8
          | (static_cast<uint32_t>(M >> 4) << 24);    // M / 16
 }

@@ -1,10 +1,10 @@
 // Bandwidth-bound kernels of the scheduled step:
 //   frozen_run   — Algorithm 2, frozen branch: h_{l,s} = h_{l-1,s} + Delta_{l, r_l(s)}
 //                  for a run of consecutive frozen units in one read-modify-write of h
-//                  (16-byte vectors: 8 fp32 of h, 8 bf16 of each cached update).
+//                  (16-byte vectors: 8 fp32 of h, 8 fp16 of each cached update).
 //   norm         — pre-norm of an active branch (RMSNorm / LayerNorm / AdaLN modulate),
-//                  fp32 residual in, bf16 GEMM operand out.
-//   stem, gemv, head_small, copy_out, pack_bf16 — the always-on parts around the
+//                  fp32 residual in, fp16 GEMM operand out.
+//   stem, gemv, head_small, copy_out, pack_f16 — the always-on parts around the
 //                  scheduled units (input stage, conditioning, output head, U-ViT skip
 //                  operands), Sec. 4.2: conditioning and skip features stay current.
 #include <cmath>
@@ -80,7 +80,7 @@ __global__ void __launch_bounds__(kNormThreads) norm_kernel(const NormParams p) 
   }
   const float* sh = p.shift ? p.shift + static_cast<int64_t>(row / p.rows_per_batch) * p.ld_mod : nullptr;
   const float* sc = p.scale ? p.scale + static_cast<int64_t>(row / p.rows_per_batch) * p.ld_mod : nullptr;
-  bf16* orow = p.out + static_cast<int64_t>(row) * p.d;
+  f16* orow = p.out + static_cast<int64_t>(row) * p.d;
 #pragma unroll
   for (int j = 0; j < kNormMaxVec; ++j) {
     const int i = threadIdx.x + j * kNormThreads;
@@ -104,8 +104,8 @@ __global__ void __launch_bounds__(kNormThreads) norm_kernel(const NormParams p) 
         for (int k = 0; k < 4; ++k) y[k] = y[k] * (1.f + sc[4 * i + k]) + sh[4 * i + k];
       }
       uint2 u;
-      u.x = pack_bf16x2(y[0], y[1]);
-      u.y = pack_bf16x2(y[2], y[3]);
+      u.x = pack_f16x2(y[0], y[1]);
+      u.y = pack_f16x2(y[2], y[3]);
       *reinterpret_cast<uint2*>(orow + 4 * i) = u;
     }
   }
@@ -121,7 +121,7 @@ __global__ void __launch_bounds__(256) frozen_kernel(const __grid_constant__ Fro
     for (int c = 0; c < p.n_caches; ++c) {
       const uint4 u = __ldcs(reinterpret_cast<const uint4*>(p.caches[c]) + i);
       float f[8];
-      unpack_bf16x8(u, f);
+      unpack_f16x8(u, f);
 #pragma unroll
       for (int k = 0; k < 8; ++k) acc[k] += f[k];
     }
@@ -159,7 +159,7 @@ __global__ void stem_kernel(const StemParams p) {
       v = reinterpret_cast<const float*>(s->state)[idx];
       break;
     case SGD_STEM_EMBED: {
-      const int id = reinterpret_cast<const int32_t*>(s->state)[r];
+      const int id = min(max(reinterpret_cast<const int32_t*>(s->state)[r], 0), p.vocab - 1);
       v = __bfloat162float(p.embed[static_cast<int64_t>(id) * p.d + c]);
       break;
     }
@@ -167,8 +167,9 @@ __global__ void stem_kernel(const StemParams p) {
     case SGD_STEM_PATCH_TOKENS: {
       const int np = n - p.n_prefix;
       if (np < 0) {
+        const int cls = min(max(s->class_ids[b], 0), p.n_classes - 1);
         v = (n == 0) ? sinusoid_at(s->t, p.d, c)
-                     : __bfloat162float(p.class_emb[static_cast<int64_t>(s->class_ids[b]) * p.d + c]);
+                     : __bfloat162float(p.class_emb[static_cast<int64_t>(cls) * p.d + c]);
       } else {
         const float* z = reinterpret_cast<const float*>(s->state) +
                          (static_cast<int64_t>(b) * (p.n_tokens - p.n_prefix) + np) * p.d_in;
@@ -227,8 +228,10 @@ __global__ void __launch_bounds__(256) gemv_kernel(const GemvParams p) {
   if (lane == 0) {
     for (int r = 0; r < p.rows; ++r) {
       float v = acc[xrows == 1 ? 0 : r];
-      if (p.add_class)
-        v += __bfloat162float(p.add_class[static_cast<int64_t>(p.slot->class_ids[r]) * p.N + j]);
+      if (p.add_class) {
+        const int cls = min(max(p.slot->class_ids[r], 0), p.n_classes - 1);
+        v += __bfloat162float(p.add_class[static_cast<int64_t>(cls) * p.N + j]);
+      }
       if (p.add_vec) v += p.add_vec[j];
       p.out[static_cast<int64_t>(r) * p.ldo + j] = v;
     }
@@ -246,13 +249,13 @@ __global__ void __launch_bounds__(256) head_small_kernel(const HeadParams p) {
   float* out = reinterpret_cast<float*>(p.slot->out) +
                (static_cast<int64_t>(b) * (p.n_tokens - p.n_prefix) + (n - p.n_prefix)) *
                    p.out_channels;
-  const bf16* x = p.x + r * p.ldx;
+  const f16* x = p.x + r * p.ldx;
   for (int j = 0; j < p.out_channels; ++j) {
     const bf16* w = p.W + static_cast<int64_t>(j) * p.K;
     float acc = 0.f;
     for (int k = lane * 8; k < p.K; k += 256) {
       float fx[8], fw[8];
-      unpack_bf16x8(*reinterpret_cast<const uint4*>(x + k), fx);
+      unpack_f16x8(*reinterpret_cast<const uint4*>(x + k), fx);
       unpack_bf16x8(*reinterpret_cast<const uint4*>(w + k), fw);
 #pragma unroll
       for (int q = 0; q < 8; ++q) acc = fmaf(fx[q], fw[q], acc);
@@ -271,7 +274,7 @@ __global__ void copy_out_kernel(const IoSlot* slot, const float* h, int64_t n4) 
     o[i] = s[i];
 }
 
-__global__ void pack_bf16_kernel(bf16* dst, int ld_dst, int col0, const float* h, int rows, int d) {
+__global__ void pack_f16_kernel(f16* dst, int ld_dst, int col0, const float* h, int rows, int d) {
   const int64_t n4 = static_cast<int64_t>(rows) * d / 4;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
@@ -280,10 +283,36 @@ __global__ void pack_bf16_kernel(bf16* dst, int ld_dst, int col0, const float* h
     const int c = static_cast<int>(e % d);
     const float4 v = reinterpret_cast<const float4*>(h)[i];
     uint2 u;
-    u.x = pack_bf16x2(v.x, v.y);
-    u.y = pack_bf16x2(v.z, v.w);
+    u.x = pack_f16x2(v.x, v.y);
+    u.y = pack_f16x2(v.z, v.w);
     *reinterpret_cast<uint2*>(dst + r * ld_dst + col0 + c) = u;
   }
+}
+
+// max |w| over a bf16 tensor: per-block maxima combined with an integer atomicMax on
+// the float bit pattern (valid for non-negative floats); *out must start at 0.
+__global__ void absmax_bf16_kernel(const bf16* w, int64_t n, float* out) {
+  __shared__ float red[8];
+  float m = 0.f;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n; i += stride)
+    m = fmaxf(m, fabsf(__bfloat162float(w[i])));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = m;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int i = 1; i < (blockDim.x >> 5); ++i) m = fmaxf(m, red[i]);
+    atomicMax(reinterpret_cast<int*>(out), __float_as_int(m));
+  }
+}
+
+// dst = fp16(w * 2^shift): exact for every bf16 value whose scaled magnitude lies in
+// the normal fp16 range (bf16 keeps 8 significant bits, fp16 11).
+__global__ void convert_bf16_f16_kernel(const bf16* w, f16* dst, int64_t n, float scale) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n; i += stride)
+    dst[i] = __float2half_rn(sat_f16(__bfloat162float(w[i]) * scale));
 }
 
 __global__ void sampler_kernel(float* z, const float* eps, float alpha, float beta, int64_t n) {
@@ -346,10 +375,20 @@ cudaError_t copy_out_launch(const IoSlot* slot, const float* h, int64_t n, cudaS
   return cudaGetLastError();
 }
 
-cudaError_t pack_bf16_launch(bf16* dst, int ld_dst, int col0, const float* h, int rows, int d,
-                             cudaStream_t s) {
-  pack_bf16_kernel<<<grid_for(static_cast<int64_t>(rows) * d / 4, 256), 256, 0, s>>>(dst, ld_dst,
-                                                                                    col0, h, rows, d);
+cudaError_t pack_f16_launch(f16* dst, int ld_dst, int col0, const float* h, int rows, int d,
+                            cudaStream_t s) {
+  pack_f16_kernel<<<grid_for(static_cast<int64_t>(rows) * d / 4, 256), 256, 0, s>>>(dst, ld_dst,
+                                                                                  col0, h, rows, d);
+  return cudaGetLastError();
+}
+
+cudaError_t absmax_bf16_launch(const bf16* w, int64_t n, float* out, cudaStream_t s) {
+  absmax_bf16_kernel<<<grid_for(n, 256), 256, 0, s>>>(w, n, out);
+  return cudaGetLastError();
+}
+
+cudaError_t convert_bf16_f16_launch(const bf16* w, f16* dst, int64_t n, int shift, cudaStream_t s) {
+  convert_bf16_f16_kernel<<<grid_for(n, 256), 256, 0, s>>>(w, dst, n, ldexpf(1.0f, shift));
   return cudaGetLastError();
 }
 

@@ -3,8 +3,9 @@
 // This is the projection kernel of every active residual branch (Algorithm 2: an
 // active unit computes Delta = F_l(h; c), refreshes its cache and adds Delta to the
 // residual stream).  The branch's last projection runs with the DELTA epilogue,
-// which stores the bf16 cache entry and adds Delta to the fp32 residual h in the
-// same pass over the tile.
+// which stores the fp16 cache entry and adds Delta to the fp32 residual h in the
+// same pass over the tile.  Operands are fp16 (weights converted exactly from bf16
+// with a power-of-two scale, undone by `alpha`), accumulation is fp32 in TMEM.
 //
 // Design (one CTA per SM, persistent over 128 x 256 output tiles):
 //   warp 0      TMA producer: A box 128x64 and two B boxes 128x64 per stage into a
@@ -30,7 +31,7 @@ namespace {
 
 constexpr int kBM = 128;
 constexpr int kBN = 256;        // accumulator columns per tile
-constexpr int kBK = 64;         // bf16 elements per 128-byte row
+constexpr int kBK = 64;         // fp16 elements per 128-byte row
 constexpr int kStages = 4;
 constexpr int kTileA = kBM * kBK * 2;          // 16 KB
 constexpr int kTileBHalf = 128 * kBK * 2;      // 16 KB
@@ -55,23 +56,23 @@ __device__ int g_status;  // device status word (bounded-wait expiry codes)
 // epilogue: 8 consecutive output columns of one row
 // ----------------------------------------------------------------------------
 
-__device__ __forceinline__ void store8_bf16(void* base, int ld, int row, int col, const float* v) {
-  bf16* p = reinterpret_cast<bf16*>(base) + static_cast<int64_t>(row) * ld + col;
-  *reinterpret_cast<uint4*>(p) = pack_bf16x8(v);
+__device__ __forceinline__ void store8_f16(void* base, int ld, int row, int col, const float* v) {
+  f16* p = reinterpret_cast<f16*>(base) + static_cast<int64_t>(row) * ld + col;
+  *reinterpret_cast<uint4*>(p) = pack_f16x8(v);
 }
 
 __device__ __forceinline__ void epi_store8(const EpiParams& e, void* out, int row, int col,
                                            float* v) {
   switch (e.kind) {
-    case SGD_EPI_BF16:
+    case SGD_EPI_F16:
     case SGD_EPI_ROPE:
     case SGD_EPI_GATED:
-      store8_bf16(out, e.ldo, row, col, v);
+      store8_f16(out, e.ldo, row, col, v);
       break;
     case SGD_EPI_GELU: {
 #pragma unroll
       for (int i = 0; i < 8; ++i) v[i] = e.act ? gelu_erf_f(v[i]) : gelu_tanh_f(v[i]);
-      store8_bf16(out, e.ldo, row, col, v);
+      store8_f16(out, e.ldo, row, col, v);
       break;
     }
     case SGD_EPI_F32: {
@@ -95,7 +96,7 @@ __device__ __forceinline__ void epi_store8(const EpiParams& e, void* out, int ro
       h1.x += v[4]; h1.y += v[5]; h1.z += v[6]; h1.w += v[7];
       hp[0] = h0;
       hp[1] = h1;
-      if (e.cache) store8_bf16(e.cache, e.ld_cache, row, col, v);
+      if (e.cache) store8_f16(e.cache, e.ld_cache, row, col, v);
       break;
     }
     default:
@@ -103,9 +104,9 @@ __device__ __forceinline__ void epi_store8(const EpiParams& e, void* out, int ro
   }
 }
 
-__device__ __forceinline__ void u32_to_f32x16(const uint32_t* r, float* f) {
+__device__ __forceinline__ void u32_to_f32x16(const uint32_t* r, float* f, float alpha) {
 #pragma unroll
-  for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(r[i]);
+  for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(r[i]) * alpha;
 }
 
 // Epilogue of one 128 x 256 accumulator, executed by all 128 epilogue threads; this
@@ -124,8 +125,8 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
       tmem_ld16(tbase + 128 + c, r1);
       tmem_ld_wait16(r0);
       tmem_ld_wait16(r1);
-      u32_to_f32x16(r0, x);
-      u32_to_f32x16(r1, y);
+      u32_to_f32x16(r0, x, e.alpha);
+      u32_to_f32x16(r1, y, e.alpha);
 #pragma unroll
       for (int i = 0; i < 16; ++i) x[i] = e.act ? x[i] * gelu_erf_f(y[i]) : silu_f(x[i]) * y[i];
       if (row_ok) {
@@ -147,8 +148,8 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
         tmem_ld16(tbase + hb + half + j, r1);
         tmem_ld_wait16(r0);
         tmem_ld_wait16(r1);
-        u32_to_f32x16(r0, x);
-        u32_to_f32x16(r1, y);
+        u32_to_f32x16(r0, x, e.alpha);
+        u32_to_f32x16(r1, y, e.alpha);
         if (rot && row_ok) {
           const float* cs = e.rope_cos + static_cast<int64_t>(pos) * half + j;
           const float* sn = e.rope_sin + static_cast<int64_t>(pos) * half + j;
@@ -177,8 +178,8 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
     tmem_ld16(tbase + c + 16, r1);
     tmem_ld_wait16(r0);
     tmem_ld_wait16(r1);
-    u32_to_f32x16(r0, x);
-    u32_to_f32x16(r1, y);
+    u32_to_f32x16(r0, x, e.alpha);
+    u32_to_f32x16(r1, y, e.alpha);
     if (row_ok) {
 #pragma unroll
       for (int q = 0; q < 2; ++q) {
@@ -279,7 +280,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      const uint32_t idesc = umma_idesc_bf16(kBM, kBN);
+      const uint32_t idesc = umma_idesc_f16(kBM, kBN);
       int it = 0, lt = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++lt) {
@@ -300,7 +301,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
           const uint32_t b_addr = a_addr + kTileA;
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k) {
-            umma_bf16(d_tmem, smem_desc_sw128(a_addr + 32 * k), smem_desc_sw128(b_addr + 32 * k),
+            umma_f16(d_tmem, smem_desc_sw128(a_addr + 32 * k), smem_desc_sw128(b_addr + 32 * k),
                       idesc, (kb | k) != 0 ? 1u : 0u);
           }
           umma_commit(&empty[s]);
@@ -345,25 +346,25 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
 // ----------------------------------------------------------------------------
 
 struct SimtArgs {
-  const bf16* A;
+  const f16* A;
   int lda;
-  const bf16* B;
+  const f16* B;
   int ldb;
   int M, N, K;
   EpiParams epi;
 };
 
-__device__ __forceinline__ float dot_bf16(const bf16* a, const bf16* b, int K) {
+__device__ __forceinline__ float dot_f16(const f16* a, const f16* b, int K) {
   float acc = 0.f;
   int k = 0;
   for (; k + 8 <= K; k += 8) {
     float fa[8], fb[8];
-    unpack_bf16x8(*reinterpret_cast<const uint4*>(a + k), fa);
-    unpack_bf16x8(*reinterpret_cast<const uint4*>(b + k), fb);
+    unpack_f16x8(*reinterpret_cast<const uint4*>(a + k), fa);
+    unpack_f16x8(*reinterpret_cast<const uint4*>(b + k), fb);
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc = fmaf(fa[i], fb[i], acc);
   }
-  for (; k < K; ++k) acc = fmaf(__bfloat162float(a[k]), __bfloat162float(b[k]), acc);
+  for (; k < K; ++k) acc = fmaf(__half2float(a[k]), __half2float(b[k]), acc);
   return acc;
 }
 
@@ -373,11 +374,11 @@ __global__ void gemm_simt_kernel(const SimtArgs a) {
   if (col >= a.N || row >= a.M) return;
   const EpiParams& e = a.epi;
   void* out = e.out_slot ? *e.out_slot : e.out;
-  const bf16* arow = a.A + static_cast<int64_t>(row) * a.lda;
-  float v = dot_bf16(arow, a.B + static_cast<int64_t>(col) * a.ldb, a.K);
+  const f16* arow = a.A + static_cast<int64_t>(row) * a.lda;
+  float v = dot_f16(arow, a.B + static_cast<int64_t>(col) * a.ldb, a.K) * e.alpha;
   switch (e.kind) {
     case SGD_EPI_GATED: {
-      const float u = dot_bf16(arow, a.B + static_cast<int64_t>(a.N + col) * a.ldb, a.K);
+      const float u = dot_f16(arow, a.B + static_cast<int64_t>(a.N + col) * a.ldb, a.K) * e.alpha;
       v = e.act ? v * gelu_erf_f(u) : silu_f(v) * u;
       break;
     }
@@ -392,7 +393,7 @@ __global__ void gemm_simt_kernel(const SimtArgs a) {
         const int partner = i < half ? col + half : col - half;
         const int fi = i < half ? i : i - half;
         const float c_ = e.rope_cos[pos * half + fi], s_ = e.rope_sin[pos * half + fi];
-        const float p = dot_bf16(arow, a.B + static_cast<int64_t>(partner) * a.ldb, a.K);
+        const float p = dot_f16(arow, a.B + static_cast<int64_t>(partner) * a.ldb, a.K) * e.alpha;
         v = i < half ? v * c_ - p * s_ : v * c_ + p * s_;
       }
       break;
@@ -400,7 +401,7 @@ __global__ void gemm_simt_kernel(const SimtArgs a) {
       if (e.gate) v *= e.gate[static_cast<int64_t>(row / e.rows_per_batch) * e.ld_gate + col];
       float* hp = e.h + static_cast<int64_t>(row) * e.ldh + col;
       *hp = *hp + v;
-      if (e.cache) e.cache[static_cast<int64_t>(row) * e.ld_cache + col] = __float2bfloat16_rn(v);
+      if (e.cache) e.cache[static_cast<int64_t>(row) * e.ld_cache + col] = __float2half_rn(sat_f16(v));
       return;
     }
     default:
@@ -409,7 +410,7 @@ __global__ void gemm_simt_kernel(const SimtArgs a) {
   if (e.kind == SGD_EPI_F32)
     reinterpret_cast<float*>(out)[static_cast<int64_t>(row) * e.ldo + col] = v;
   else
-    reinterpret_cast<bf16*>(out)[static_cast<int64_t>(row) * e.ldo + col] = __float2bfloat16_rn(v);
+    reinterpret_cast<f16*>(out)[static_cast<int64_t>(row) * e.ldo + col] = __float2half_rn(sat_f16(v));
 }
 
 // ----------------------------------------------------------------------------
@@ -435,7 +436,7 @@ EncodeTiledFn get_encode_fn() {
   return fn;
 }
 
-// bf16 [rows, cols] with row stride ld elements; box = 64 columns x box_rows rows.
+// fp16 [rows, cols] with row stride ld elements; box = 64 columns x box_rows rows.
 bool make_tmap(CUtensorMap* m, const void* base, int rows, int cols, int ld, int box_rows) {
   EncodeTiledFn fn = get_encode_fn();
   if (!fn) return false;
@@ -443,7 +444,7 @@ bool make_tmap(CUtensorMap* m, const void* base, int rows, int cols, int ld, int
   cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
   cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), static_cast<cuuint32_t>(box_rows)};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides,
                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;

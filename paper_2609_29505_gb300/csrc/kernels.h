@@ -4,6 +4,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <stdint.h>
 
 #include "../../include/sgd.h"
@@ -12,17 +13,19 @@
 namespace sgd {
 
 using bf16 = __nv_bfloat16;
+using f16 = __half;
 
 // Epilogue parameters as the kernels see them (mirror of sgd_epilogue_args plus the
 // output-pointer slot used by captured graphs and the output extent).
 struct EpiParams {
   int kind;
+  float alpha;            // accumulator scale (undoes the power-of-two weight scale)
   void* out;
   int ldo;
   void* const* out_slot;  // device address holding the output pointer (overrides out)
   float* h;
   int ldh;
-  bf16* cache;
+  f16* cache;
   int ld_cache;
   const float* gate;
   int ld_gate;
@@ -39,9 +42,9 @@ struct EpiParams {
 
 // A planned GEMM: operands, epilogue and prebuilt TMA descriptors.
 struct GemmPlan {
-  const bf16* A = nullptr;
+  const f16* A = nullptr;
   int lda = 0;
-  const bf16* B = nullptr;
+  const f16* B = nullptr;
   int ldb = 0;
   int M = 0, N = 0, K = 0;   // N = output columns
   EpiParams epi{};
@@ -59,12 +62,12 @@ int num_sms();
 
 // Attention.
 struct AttnParams {
-  const bf16* q;
+  const f16* q;
   int ldq;
-  const bf16* k;
-  const bf16* v;
+  const f16* k;
+  const f16* v;
   int ldkv;
-  bf16* o;
+  f16* o;
   int ldo;
   int batch, n_q, n_kv, n_heads, d_head;
 };
@@ -74,7 +77,7 @@ cudaError_t attn_launch(const AttnParams& p, cudaStream_t s);
 // Norm: out = norm(h) [* (1 + scale) + shift].
 struct NormParams {
   const float* h;
-  bf16* out;
+  f16* out;
   int rows, d, kind;
   const bf16* g;
   const bf16* b;
@@ -89,7 +92,7 @@ cudaError_t norm_launch(const NormParams& p, cudaStream_t s);
 constexpr int kMaxRun = 96;
 struct FrozenParams {
   float* h;
-  const bf16* caches[kMaxRun];
+  const f16* caches[kMaxRun];
   int n_caches;
   int64_t n;
 };
@@ -116,6 +119,7 @@ struct StemParams {
   const bf16* pos;
   const bf16* class_emb;
   const bf16* embed;
+  int vocab, n_classes;  // ids are clamped into [0, vocab) / [0, n_classes)
 };
 cudaError_t stem_launch(const StemParams& p, cudaStream_t s);
 
@@ -130,14 +134,15 @@ struct GemvParams {
   int in_silu;         // act = silu
   const bf16* W;       // [N, K]
   int N, K, rows;
-  const bf16* add_class;  // optional: + class_emb[class_ids[r]] (bf16 [*, N])
+  const bf16* add_class;  // optional: + class_emb[class_ids[r]] (bf16 [n_classes, N])
+  int n_classes;          // class ids are clamped into [0, n_classes)
   const float* add_vec;   // optional: + add_vec[j] (broadcast over rows)
 };
 cudaError_t gemv_launch(const GemvParams& p, cudaStream_t s);
 
 // Row-wise small-N linear for heads: out[r, j] = x[r] . W[j] for j < N (N <= 64).
 struct HeadParams {
-  const bf16* x;       // [rows_total, K] bf16 (normalised states)
+  const f16* x;        // [rows_total, K] fp16 (normalised states)
   int ldx;
   const bf16* W;       // [N, K]
   int N, K;
@@ -150,9 +155,14 @@ cudaError_t head_small_launch(const HeadParams& p, cudaStream_t s);
 // Identity head: out (from slot) = h.
 cudaError_t copy_out_launch(const IoSlot* slot, const float* h, int64_t n, cudaStream_t s);
 
-// U-ViT: dst bf16 [rows, ld_dst] columns [col0, col0 + d) = bf16(h).
-cudaError_t pack_bf16_launch(bf16* dst, int ld_dst, int col0, const float* h, int rows, int d,
-                             cudaStream_t s);
+// U-ViT: dst fp16 [rows, ld_dst] columns [col0, col0 + d) = fp16(h).
+cudaError_t pack_f16_launch(f16* dst, int ld_dst, int col0, const float* h, int rows, int d,
+                            cudaStream_t s);
+
+// Weight preparation: max |w| of a bf16 tensor (into *out, device) and the exact
+// conversion dst = fp16(w * 2^shift); also plain bf16 -> fp16 conversion (shift 0).
+cudaError_t absmax_bf16_launch(const bf16* w, int64_t n, float* out, cudaStream_t s);
+cudaError_t convert_bf16_f16_launch(const bf16* w, f16* dst, int64_t n, int shift, cudaStream_t s);
 
 cudaError_t sampler_launch(float* z, const float* eps, float alpha, float beta, int64_t n,
                            cudaStream_t s);

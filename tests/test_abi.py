@@ -112,7 +112,7 @@ def test_null_context_calls_fail_cleanly(lib):
 def test_kernel_entry_points_validate_on_host(lib):
     epi = binding.sgd_epilogue_args(kind=99)
     assert lib.sgd_kernel_gemm(None, 8, None, 8, 8, 8, 8, C.byref(epi), 0, None) == binding.SGD_ERR_ARG
-    epi = binding.sgd_epilogue_args(kind=binding.EPI_BF16, out=64, ldo=8)
+    epi = binding.sgd_epilogue_args(kind=binding.EPI_F16, out=64, ldo=8)
     # K not a multiple of 8
     assert lib.sgd_kernel_gemm(64, 12, 64, 12, 8, 8, 12, C.byref(epi), 0, None) == binding.SGD_ERR_SHAPE
     assert lib.sgd_kernel_attention(64, 8, 64, 64, 8, 64, 8, 1, 4, 4, 1, 96, None) == binding.SGD_ERR_SHAPE

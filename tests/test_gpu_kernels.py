@@ -1,0 +1,225 @@
+"""Kernel-level parity on the GPU: every hot-path kernel of libsgd, called through
+the C ABI (include/sgd_kernels.h), against the CPU oracle's definition of the same
+operation, on seeded inputs with ragged tails (M, N, K, keys not tile multiples).
+
+Operands and stored activations are fp16 (fp32 accumulation).  Tolerances: an
+fp16 output may differ from the fp32 oracle by the rounding of the result
+(relative 2^-11) plus fp32 accumulation-order noise; fp32 outputs (the residual
+update) by accumulation order only."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import denoiser as odn
+
+pytestmark = pytest.mark.gpu
+
+F16_REL = 2.0 ** -11
+
+
+@pytest.fixture(scope="module")
+def B():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    from paper_2609_29505_gb300 import binding, build
+    build.build()
+    binding.lib()
+    return binding
+
+
+def _rand(rng, shape, scale=1.0, dtype=torch.float16):
+    return torch.from_numpy((rng.standard_normal(shape) * scale).astype(np.float32)).to(dtype)
+
+
+def _f(t):
+    return t.float().cpu().numpy()
+
+
+def _check_f16(got, want, extra_abs=0.0):
+    got = _f(got)
+    scale = float(np.sqrt(np.mean(want.astype(np.float64) ** 2))) + 1e-30
+    bound = F16_REL * np.abs(want) + 2e-5 * scale + extra_abs
+    bad = np.abs(got - want) > bound
+    assert not bad.any(), (f"{bad.sum()} of {bad.size} outside fp16 rounding; max err "
+                           f"{np.max(np.abs(got - want)):.3e}, rms(want) {scale:.3e}")
+
+
+GEMM_SHAPES = [(64, 256, 256), (300, 520, 688), (129, 264, 72), (1000, 1376, 512), (4128, 1024, 2048)]
+
+
+@pytest.mark.parametrize("simt", [0, 1], ids=["tcgen05", "simt"])
+@pytest.mark.parametrize("M,N,K", GEMM_SHAPES)
+def test_gemm_bf16(B, M, N, K, simt):
+    rng = np.random.default_rng(M + N + K)
+    A = _rand(rng, (M, K)).cuda()
+    W = _rand(rng, (N, K), 1 / math.sqrt(K)).cuda()
+    out = torch.empty(M, N, dtype=torch.float16, device="cuda")
+    epi = B.sgd_epilogue_args(kind=B.EPI_F16, out=out.data_ptr(), ldo=N)
+    B.sgd_kernel_gemm(A, W, M, N, K, epi, use_simt=simt)
+    torch.cuda.synchronize()
+    assert B.sgd_kernel_status() == 0
+    _check_f16(out, odn.linear(_f(A), _f(W)))
+
+
+@pytest.mark.parametrize("simt", [0, 1], ids=["tcgen05", "simt"])
+@pytest.mark.parametrize("gated", [False, True])
+def test_gemm_delta_residual_and_cache(B, simt, gated):
+    rng = np.random.default_rng(5)
+    M, N, K, rpb = 520, 264, 688, 130
+    A = _rand(rng, (M, K)).cuda()
+    W = _rand(rng, (N, K), 1 / math.sqrt(K)).cuda()
+    h0 = torch.from_numpy(rng.standard_normal((M, N)).astype(np.float32)).cuda()
+    h = h0.clone()
+    cache = torch.zeros(M, N, dtype=torch.float16, device="cuda")
+    gate = torch.from_numpy(rng.standard_normal((M // rpb, N)).astype(np.float32)).cuda()
+    epi = B.sgd_epilogue_args(kind=B.EPI_DELTA, h=h.data_ptr(), ldh=N, cache=cache.data_ptr(),
+                              ld_cache=N, gate=gate.data_ptr() if gated else None, ld_gate=N,
+                              rows_per_batch=rpb)
+    B.sgd_kernel_gemm(A, W, M, N, K, epi, use_simt=simt)
+    torch.cuda.synchronize()
+    delta = odn.linear(_f(A), _f(W))
+    if gated:
+        delta = delta * np.repeat(gate.cpu().numpy(), rpb, axis=0)
+    want_h = h0.cpu().numpy() + delta
+    np.testing.assert_allclose(h.cpu().numpy(), want_h, rtol=2e-5, atol=2e-5)
+    _check_f16(cache, delta)
+
+
+@pytest.mark.parametrize("simt", [0, 1], ids=["tcgen05", "simt"])
+@pytest.mark.parametrize("act", [0, 1])
+def test_gemm_gated_activation(B, simt, act):
+    rng = np.random.default_rng(6)
+    M, f, K = 300, 688, 256
+    A = _rand(rng, (M, K)).cuda()
+    W = _rand(rng, (2 * f, K), 1 / math.sqrt(K)).cuda()
+    out = torch.empty(M, f, dtype=torch.float16, device="cuda")
+    epi = B.sgd_epilogue_args(kind=B.EPI_GATED, out=out.data_ptr(), ldo=f, act=act)
+    B.sgd_kernel_gemm(A, W, M, f, K, epi, use_simt=simt)
+    torch.cuda.synchronize()
+    u = odn.linear(_f(A), _f(W))
+    want = odn.silu(u[:, :f]) * u[:, f:] if act == 0 else u[:, :f] * odn.gelu_erf(u[:, f:])
+    _check_f16(out, want, extra_abs=1e-4 * float(np.abs(want).max()))
+
+
+@pytest.mark.parametrize("simt", [0, 1], ids=["tcgen05", "simt"])
+@pytest.mark.parametrize("act", [0, 1])
+def test_gemm_gelu(B, simt, act):
+    rng = np.random.default_rng(7)
+    M, N, K = 200, 1152, 288
+    A = _rand(rng, (M, K)).cuda()
+    W = _rand(rng, (N, K), 1 / math.sqrt(K)).cuda()
+    out = torch.empty(M, N, dtype=torch.float16, device="cuda")
+    epi = B.sgd_epilogue_args(kind=B.EPI_GELU, out=out.data_ptr(), ldo=N, act=act)
+    B.sgd_kernel_gemm(A, W, M, N, K, epi, use_simt=simt)
+    torch.cuda.synchronize()
+    u = odn.linear(_f(A), _f(W))
+    want = odn.gelu_erf(u) if act else odn.gelu_tanh(u)
+    _check_f16(out, want, extra_abs=1e-4 * float(np.abs(want).max()))
+
+
+@pytest.mark.parametrize("simt", [0, 1], ids=["tcgen05", "simt"])
+@pytest.mark.parametrize("dh", [64, 128])
+def test_gemm_rope_epilogue(B, simt, dh):
+    rng = np.random.default_rng(8)
+    H, n_tok, bsz = 4, 96, 3
+    d = H * dh
+    M, N, K = bsz * n_tok, 3 * d, d
+    A = _rand(rng, (M, K)).cuda()
+    W = _rand(rng, (N, K), 1 / math.sqrt(K)).cuda()
+    half = dh // 2
+    pos = np.arange(n_tok, dtype=np.float64)[:, None]
+    freq = 10000.0 ** (-np.arange(half) * 2.0 / dh)
+    cos = torch.from_numpy(np.cos(pos * freq).astype(np.float32)).cuda()
+    sin = torch.from_numpy(np.sin(pos * freq).astype(np.float32)).cuda()
+    out = torch.empty(M, N, dtype=torch.float16, device="cuda")
+    epi = B.sgd_epilogue_args(kind=B.EPI_ROPE, out=out.data_ptr(), ldo=N, rope_cos=cos.data_ptr(),
+                              rope_sin=sin.data_ptr(), rope_tokens=n_tok, d_head=dh, rope_cols=2 * d)
+    B.sgd_kernel_gemm(A, W, M, N, K, epi, use_simt=simt)
+    torch.cuda.synchronize()
+    qkv = odn.linear(_f(A), _f(W)).reshape(bsz, n_tok, 3, H, dh)
+    want = qkv.copy()
+    for j in range(2):  # q and k rotate, v does not
+        x = qkv[:, :, j].transpose(0, 2, 1, 3)  # [b, H, n, dh]
+        want[:, :, j] = odn.rope(x, np.arange(n_tok), 10000.0).transpose(0, 2, 1, 3)
+    _check_f16(out, want.reshape(M, N), extra_abs=1e-4)
+
+
+@pytest.mark.parametrize("dh,H,nq,nkv,bsz", [(64, 4, 64, 64, 1), (72, 3, 136, 136, 2),
+                                              (128, 2, 192, 192, 2), (64, 5, 200, 77, 2),
+                                              (64, 4, 258, 258, 2), (128, 2, 33, 5, 3)])
+def test_attention(B, dh, H, nq, nkv, bsz):
+    rng = np.random.default_rng(dh + nq + nkv)
+    d = H * dh
+    q = _rand(rng, (bsz * nq, d), 1.5).cuda()
+    k = _rand(rng, (bsz * nkv, d), 1.5).cuda()
+    v = _rand(rng, (bsz * nkv, d)).cuda()
+    o = torch.empty(bsz * nq, d, dtype=torch.float16, device="cuda")
+    B.sgd_kernel_attention(q, d, k, v, d, o, d, bsz, nq, nkv, H, dh)
+    torch.cuda.synchronize()
+    want = odn.attention(_f(q).reshape(bsz, nq, d), _f(k).reshape(bsz, nkv, d),
+                         _f(v).reshape(bsz, nkv, d), H).reshape(bsz * nq, d)
+    got = _f(o)
+    # P is rounded to bf16 before P V: relative error of a few bf16 ulps on O
+    err = np.linalg.norm(got - want) / np.linalg.norm(want)
+    assert err < 6e-3, err
+    assert np.max(np.abs(got - want)) < 0.03 * float(np.abs(want).max())
+
+
+@pytest.mark.parametrize("kind,d", [(0, 256), (0, 4096), (1, 1280), (2, 1152), (1, 1024)])
+def test_norm(B, kind, d):
+    rng = np.random.default_rng(kind * 10000 + d)
+    rows, rpb = 260, 130
+    h = torch.from_numpy((rng.standard_normal((rows, d)) * 3 + 0.5).astype(np.float32)).cuda()
+    g = _rand(rng, (d,), 0.1).float().add(1.0).to(torch.bfloat16).cuda() if kind != 2 else None
+    b = _rand(rng, (d,), 0.1, torch.bfloat16).cuda() if kind == 1 else None
+    out = torch.empty(rows, d, dtype=torch.float16, device="cuda")
+    shift = scale = None
+    if kind == 2:
+        mod = torch.from_numpy(rng.standard_normal((rows // rpb, 2 * d)).astype(np.float32) * 0.3).cuda()
+        shift, scale = mod[:, :d], mod[:, d:]
+        B.sgd_kernel_norm(h, out, rows, d, kind, shift=mod, scale=mod[:, d:], ld_mod=2 * d,
+                          rows_per_batch=rpb, eps=1e-6)
+    else:
+        B.sgd_kernel_norm(h, out, rows, d, kind, g=g, b=b, eps=1e-6)
+    torch.cuda.synchronize()
+    hn = h.cpu().numpy()
+    if kind == 0:
+        want = odn.rms_norm(hn, _f(g), 1e-6)
+    elif kind == 1:
+        want = odn.layer_norm(hn, _f(g), _f(b), 1e-6)
+    else:
+        x = odn.layer_norm(hn, None, None, 1e-6).reshape(rows // rpb, rpb, d)
+        want = odn.modulate(x, shift.cpu().numpy(), scale.cpu().numpy()).reshape(rows, d)
+    _check_f16(out, want, extra_abs=1e-5)
+
+
+@pytest.mark.parametrize("n_caches", [1, 3, 17])
+def test_frozen_run_sums_in_unit_order(B, n_caches):
+    rng = np.random.default_rng(n_caches)
+    n = 4128 * 64
+    h0 = rng.standard_normal(n).astype(np.float32)
+    caches = [_rand(rng, (n,)).cuda() for _ in range(n_caches)]
+    h = torch.from_numpy(h0).cuda()
+    B.sgd_kernel_frozen_run(h, caches)
+    torch.cuda.synchronize()
+    want = h0.copy()
+    for c in caches:  # Algorithm 2: each frozen unit adds its cached Delta in graph order
+        want = (want + _f(c)).astype(np.float32)
+    np.testing.assert_array_equal(h.cpu().numpy(), want)
+
+
+def test_gemm_large_sampled_rows_tcgen05(B):
+    """LLaDA-sized projection (M = N = K = 4096) on tcgen05; 96 sampled rows checked."""
+    rng = np.random.default_rng(9)
+    M = N = K = 4096
+    A = torch.randn(M, K, generator=torch.Generator().manual_seed(1)).to(torch.float16).cuda()
+    W = (torch.randn(N, K, generator=torch.Generator().manual_seed(2)) / 64).to(torch.float16).cuda()
+    out = torch.empty(M, N, dtype=torch.float16, device="cuda")
+    epi = B.sgd_epilogue_args(kind=B.EPI_F16, out=out.data_ptr(), ldo=N)
+    B.sgd_kernel_gemm(A, W, M, N, K, epi)
+    torch.cuda.synchronize()
+    rows = np.sort(rng.choice(M, 96, replace=False))
+    want = odn.linear(_f(A[rows]), _f(W))
+    _check_f16(out[rows], want)

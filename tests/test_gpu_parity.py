@@ -1,0 +1,200 @@
+"""End-to-end parity of the scheduled denoiser step on the GPU (through the C ABI)
+against the CPU oracle, for every architecture family at reduced size and for
+three layer-step budgets.
+
+* active sets: bit-exact against the oracle's A_s = {u : s <= S_u};
+* per step (teacher forced: the GPU evaluates the oracle's state z_s, its caches
+  are its own): relative L2 of eps_s <= 5e-3;
+* closed loop (the GPU integrates its own states with the library's sampler
+  update): relative L2 of the final state and of the last eps <= 1e-2.
+"""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import denoiser as odn
+from oracle import spectral as osp
+from oracle import trajectory as otj
+from paper_2609_29505_gb300 import schedule, synth
+
+pytestmark = pytest.mark.gpu
+
+# SGD_TEST_SIMT=1 runs every GEMM of the model on the SIMT reference kernel (debugging aid)
+FLAGS = 1 if os.environ.get("SGD_TEST_SIMT") == "1" else 0
+STEP_TOL = 5e-3
+FINAL_TOL = 1e-2
+SMALL = ["tiny", "dit_small", "uvit_small", "sdxl_small", "llada_small"]
+
+
+@pytest.fixture(scope="module")
+def B():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    from paper_2609_29505_gb300 import binding, build
+    build.build()
+    binding.lib()
+    return binding
+
+
+def rel(a, b):
+    a = np.asarray(a, np.float64)
+    b = np.asarray(b, np.float64)
+    return float(np.linalg.norm(a - b) / np.linalg.norm(b))
+
+
+class Case:
+    def __init__(self, name, budget, flags=0):
+        self.cfg = cfg = synth.get_config(name)
+        self.T = cfg.T
+        self.w_cpu = synth.make_weights(cfg, "cpu")
+        self.inp = synth.make_inputs(cfg, "cpu")
+        self.W = odn.to_numpy_weights(self.w_cpu)
+        self.sched = schedule.build_schedule(cfg, self.w_cpu, self.T, budget=budget)
+        self.w_dev = {k: v.cuda() for k, v in self.w_cpu.items()}
+        self.cls = None if self.inp.class_ids is None else self.inp.class_ids.cuda()
+        self.ctx = None if self.inp.ctx is None else self.inp.ctx.cuda()
+        self.flags = flags
+
+    def ids_at(self, s):
+        return synth.token_ids_at(self.cfg, self.inp, s, self.T)
+
+    def oracle(self):
+        cfg = self.cfg
+        return otj.run(cfg, self.W, self.sched["lifetimes"], self.T,
+                       z0=None if self.inp.z0 is None else self.inp.z0.numpy(),
+                       class_ids=None if self.inp.class_ids is None else self.inp.class_ids.numpy(),
+                       ctx=None if self.inp.ctx is None else self.inp.ctx.float().numpy(),
+                       ids_at=(lambda s: self.ids_at(s).numpy()) if cfg.stem == "embed" else None)
+
+    def model(self, B):
+        m = B.Denoiser(self.cfg, self.w_dev, flags=self.flags)
+        m.set_schedule(self.T, self.sched["lifetimes"], self.sched["groups"])
+        return m
+
+    def out_buffer(self):
+        cfg = self.cfg
+        if cfg.head == "logits":
+            return torch.empty(cfg.batch, cfg.n_tokens, cfg.d_out, dtype=torch.float16, device="cuda")
+        if cfg.head == "identity":
+            return torch.empty(cfg.batch, cfg.n_tokens, cfg.d, device="cuda")
+        return torch.empty(cfg.batch, cfg.n_out_tokens, cfg.out_channels, device="cuda")
+
+
+_cases = {}
+
+
+def case(name, budget):
+    key = (name, budget)
+    if key not in _cases:
+        c = Case(name, budget, FLAGS)
+        c.ref = c.oracle()
+        _cases[key] = c
+    return _cases[key]
+
+
+@pytest.mark.parametrize("budget", [1.0, 0.5, 0.33])
+@pytest.mark.parametrize("name", SMALL)
+def test_active_sets_and_teacher_forced_steps(B, name, budget):
+    c = case(name, budget)
+    m = c.model(B)
+    want_masks = osp.active_sets(c.sched["lifetimes"], c.T)
+    out = c.out_buffer()
+    errs = []
+    for s in range(1, c.T + 1):
+        np.testing.assert_array_equal(m.active_mask(s), want_masks[s - 1])
+        x = c.ids_at(s).cuda() if c.cfg.stem == "embed" else torch.from_numpy(c.ref["states"][s - 1]).cuda()
+        m.step(x, out, otj.timestep(c.T, s), s, class_ids=c.cls, ctx=c.ctx)
+        errs.append(rel(out.float().cpu().numpy(), c.ref["outputs"][s - 1]))
+    m.check_device()
+    info = m.info()
+    m.close()
+    assert info["layer_steps"] == int(np.sum(c.sched["lifetimes"]))
+    assert max(errs) <= STEP_TOL, f"per-step rel L2 {['%.2e' % e for e in errs]}"
+
+
+@pytest.mark.parametrize("budget", [1.0, 0.5])
+@pytest.mark.parametrize("name", ["tiny", "dit_small", "uvit_small", "sdxl_small"])
+def test_closed_loop_final_state(B, name, budget):
+    c = case(name, budget)
+    m = c.model(B)
+    out = c.out_buffer()
+    z = c.inp.z0.clone().cuda()
+    for s in range(1, c.T + 1):
+        m.step(z, out, otj.timestep(c.T, s), s, class_ids=c.cls, ctx=c.ctx)
+        B.sgd_sampler_update(z, out, 1.0, 1.0 / c.T)
+    torch.cuda.synchronize()
+    m.close()
+    assert rel(z.cpu().numpy(), c.ref["states"][-1]) <= FINAL_TOL
+    assert rel(out.cpu().numpy(), c.ref["outputs"][-1]) <= FINAL_TOL
+
+
+def test_graph_replay_equals_profiled_eager_launches(B):
+    c = case("dit_small", 0.5)
+    outs = []
+    for mode in ("graph", "profile"):
+        m = c.model(B)
+        out = c.out_buffer()
+        z = torch.from_numpy(c.ref["states"][0]).cuda()
+        res = []
+        for s in range(1, c.T + 1):
+            if mode == "graph":
+                m.step(z, out, otj.timestep(c.T, s), s, class_ids=c.cls)
+            else:
+                recs = m.profile_step(z, out, otj.timestep(c.T, s), s, class_ids=c.cls)
+                assert recs and all(r["ms"] >= 0 for r in recs)
+            res.append(out.cpu().clone())
+        m.close()
+        outs.append(res)
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
+
+
+def test_host_buffer_step_equals_device_step(B):
+    c = case("uvit_small", 0.5)
+    m = c.model(B)
+    out_d = c.out_buffer()
+    out_h = torch.empty(out_d.shape, dtype=out_d.dtype).pin_memory()
+    cls_h = c.inp.class_ids.clone().pin_memory()
+    for s in range(1, 4):
+        z = torch.from_numpy(c.ref["states"][s - 1])
+        m.step(z.cuda(), out_d, otj.timestep(c.T, s), s, class_ids=c.cls)
+        torch.cuda.synchronize()
+        a = out_d.cpu()
+    m.reset()
+    for s in range(1, 4):
+        z = torch.from_numpy(c.ref["states"][s - 1]).pin_memory()
+        m.step_host(z, out_h, otj.timestep(c.T, s), s, class_ids_host=cls_h)
+    assert torch.equal(out_h, a)
+    m.close()
+
+
+def test_step_order_and_state_errors(B):
+    c = case("tiny", 0.5)
+    m = B.Denoiser(c.cfg, c.w_dev)
+    out = c.out_buffer()
+    z = c.inp.z0.clone().cuda()
+    with pytest.raises(B.SgdError) as e:
+        m.step(z, out, 1.0, 1)
+    assert e.value.code == B.SGD_ERR_STATE
+    m.set_schedule(c.T, c.sched["lifetimes"], c.sched["groups"])
+    with pytest.raises(B.SgdError) as e:
+        m.step(z, out, 1.0, 2)
+    assert e.value.code == B.SGD_ERR_CACHE_INVALID
+    m.step(z, out, 1.0, 1)
+    with pytest.raises(B.SgdError) as e:
+        m.step(z, out, 1.0, 3)
+    assert e.value.code == B.SGD_ERR_CACHE_INVALID
+    m.step(z, out, 1.0, 2)
+    m.reset()
+    with pytest.raises(B.SgdError) as e:
+        m.step(z, out, 1.0, 3)
+    assert e.value.code == B.SGD_ERR_CACHE_INVALID
+    bad = np.array(c.sched["lifetimes"]).copy()
+    bad[0] = bad[1] + 1 if bad[1] < c.T else bad[1] - 1
+    with pytest.raises(B.SgdError) as e:
+        m.set_schedule(c.T, bad, c.sched["groups"])
+    assert e.value.code == B.SGD_ERR_SCHEDULE
+    m.check_device()
+    m.close()
