@@ -1,0 +1,129 @@
+"""Single-kernel cases of libsgd at the LLaDA-8B-shaped sizes, timed with CUDA events.
+
+Each case launches one hot-path kernel through the C ABI (include/sgd_kernels.h)
+with the same launch configuration sgd_step uses, on inputs larger than L2, and
+prints one JSON line: average launch time and achieved TFLOP/s or GB/s.  It is the
+command that the committed ncu summaries under profiles/ were captured from.
+
+    python -m paper_2609_29505_gb300.kernel_bench gemm --M 4096 --N 12288 --K 4096 --epi rope
+    python -m paper_2609_29505_gb300.kernel_bench attention --batch 4 --heads 32 --tokens 1024 --dh 128
+    python -m paper_2609_29505_gb300.kernel_bench frozen --rows 4096 --d 4096 --caches 8
+    python -m paper_2609_29505_gb300.kernel_bench norm --rows 4096 --d 4096
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+
+import torch
+
+from . import binding, build
+
+EPI = {"f16": binding.EPI_F16, "f32": binding.EPI_F32, "delta": binding.EPI_DELTA,
+       "gated": binding.EPI_GATED, "gelu": binding.EPI_GELU, "rope": binding.EPI_ROPE}
+
+
+def _time(fn, iters, warmup):
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(iters):
+        fn()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / iters
+
+
+def case_gemm(a):
+    g = torch.Generator(device="cuda").manual_seed(0)
+    M, N, K = a.M, a.N, a.K
+    rows_b = 2 * N if a.epi == "gated" else N
+    A = torch.randn(M, K, device="cuda", generator=g).half()
+    B = (torch.randn(rows_b, K, device="cuda", generator=g) / math.sqrt(K)).half()
+    epi = binding.sgd_epilogue_args(kind=EPI[a.epi], alpha=1.0)
+    keep = []
+    if a.epi == "delta":
+        h = torch.zeros(M, N, device="cuda")
+        cache = torch.empty(M, N, device="cuda", dtype=torch.float16)
+        epi.h, epi.ldh = h.data_ptr(), N
+        if a.store_cache:
+            epi.cache, epi.ld_cache = cache.data_ptr(), N
+        keep += [h, cache]
+    else:
+        out = torch.empty(M, N, device="cuda", dtype=torch.float32 if a.epi == "f32" else torch.float16)
+        epi.out, epi.ldo = out.data_ptr(), N
+        keep.append(out)
+    if a.epi == "rope":
+        half = 64
+        cos = torch.ones(a.tokens, half, device="cuda")
+        sin = torch.zeros(a.tokens, half, device="cuda")
+        epi.rope_cos, epi.rope_sin, epi.rope_tokens = cos.data_ptr(), sin.data_ptr(), a.tokens
+        epi.d_head, epi.rope_cols = 128, 2 * N // 3
+        keep += [cos, sin]
+    epi.act = 0
+    ms = _time(lambda: binding.sgd_kernel_gemm(A, B, M, N, K, epi, use_simt=a.simt), a.iters, a.warmup)
+    flops = 2.0 * M * rows_b * K
+    return dict(case="gemm", M=M, N=N, K=K, epi=a.epi, ms=ms, tflops=flops / ms / 1e9)
+
+
+def case_attention(a):
+    B, H, N, dh = a.batch, a.heads, a.tokens, a.dh
+    d = H * dh
+    qkv = torch.randn(B * N, 3 * d, device="cuda").half()
+    o = torch.empty(B * N, d, device="cuda", dtype=torch.float16)
+    q, k, v = qkv[:, :d], qkv[:, d:2 * d], qkv[:, 2 * d:]
+    ms = _time(lambda: binding.sgd_kernel_attention(q, 3 * d, k, v, 3 * d, o, d, B, N, N, H, dh),
+               a.iters, a.warmup)
+    flops = 4.0 * B * H * N * N * dh
+    return dict(case="attention", batch=B, heads=H, tokens=N, dh=dh, ms=ms, tflops=flops / ms / 1e9)
+
+
+def case_frozen(a):
+    n = a.rows * a.d
+    h = torch.zeros(n, device="cuda")
+    caches = [torch.randn(n, device="cuda").half() for _ in range(a.caches)]
+    ms = _time(lambda: binding.sgd_kernel_frozen_run(h, caches), a.iters, a.warmup)
+    bytes_ = n * (8.0 + 2.0 * a.caches)
+    return dict(case="frozen_run", n=n, caches=a.caches, ms=ms, gbs=bytes_ / ms / 1e6)
+
+
+def case_norm(a):
+    h = torch.randn(a.rows, a.d, device="cuda")
+    out = torch.empty(a.rows, a.d, device="cuda", dtype=torch.float16)
+    g = torch.ones(a.d, device="cuda", dtype=torch.bfloat16)
+    ms = _time(lambda: binding.sgd_kernel_norm(h, out, a.rows, a.d, 0, g=g), a.iters, a.warmup)
+    return dict(case="norm", rows=a.rows, d=a.d, ms=ms, gbs=6.0 * a.rows * a.d / ms / 1e6)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("case", choices=["gemm", "attention", "frozen", "norm"])
+    ap.add_argument("--M", type=int, default=4096)
+    ap.add_argument("--N", type=int, default=12288)
+    ap.add_argument("--K", type=int, default=4096)
+    ap.add_argument("--epi", default="f16", choices=list(EPI))
+    ap.add_argument("--store-cache", action="store_true")
+    ap.add_argument("--simt", type=int, default=0)
+    ap.add_argument("--tokens", type=int, default=1024)
+    ap.add_argument("--batch", type=int, default=4)
+    ap.add_argument("--heads", type=int, default=32)
+    ap.add_argument("--dh", type=int, default=128)
+    ap.add_argument("--rows", type=int, default=4096)
+    ap.add_argument("--d", type=int, default=4096)
+    ap.add_argument("--caches", type=int, default=8)
+    ap.add_argument("--iters", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    a = ap.parse_args()
+    build.build()
+    binding.lib()
+    res = {"gemm": case_gemm, "attention": case_attention, "frozen": case_frozen,
+           "norm": case_norm}[a.case](a)
+    res["status"] = binding.sgd_kernel_status()
+    print(json.dumps(res))
+
+
+if __name__ == "__main__":
+    main()
