@@ -38,6 +38,8 @@ def parse():
     ap.add_argument("--T", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--ablation", action="store_true",
+                    help="also time the execution modes of Table tab:kernel (adds key 'ablation')")
     return ap.parse_args()
 
 
@@ -299,6 +301,10 @@ def run_native(args):
         e2e = {"value": round(K * world / e2e_s, 3), "unit": "steps/s", "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(out_h.numel() * out_h.element_size())}
 
+    ablation = None
+    if args.ablation:
+        ablation = run_ablation(binding, model, cfg, T, weights, sched, xs, out, cls, ctx, stream)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(cfg, T, weights, inp, sched, n_steps=8)
@@ -321,6 +327,7 @@ def run_native(args):
                    "cache_gb": round(info["cache_bytes"] / 2 ** 30, 2), "setup": setup_t},
         "roofline": roofline, "step_roofline": step_roof, "kernels": kernels,
         "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(gpu_launches),
+        "ablation": ablation,
         "clocks": clk.summary(),
     }
     if rank == 0:
@@ -328,6 +335,42 @@ def run_native(args):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def run_ablation(binding, model, cfg, T, weights, sched, xs, out, cls, ctx, stream):
+    """Execution modes of Table tab:kernel on this workload: eager full inference (100%
+    schedule, one launch per op), host-side skipping (budget schedule, eager), padded
+    static graphs (every frozen branch still evaluated) and jagged graphs.  One whole
+    trajectory each, CUDA events on the stream."""
+    import torch
+    from paper_2609_29505_gb300.synth import timestep
+    full = [T] * cfg.n_units
+    rows = []
+    modes = [("eager_full", full, binding.EXEC_EAGER),
+             ("host_skipping", sched["lifetimes"], binding.EXEC_EAGER),
+             ("padded_graph", sched["lifetimes"], binding.EXEC_PADDED_GRAPH),
+             ("jagged_graph", sched["lifetimes"], binding.EXEC_JAGGED_GRAPH)]
+    for name, S, mode in modes:
+        model.set_schedule(T, S, sched["groups"])
+        model.set_exec_mode(mode)
+        for rep in range(2):  # first pass warms the mode up
+            model.reset()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for s in range(1, T + 1):
+                model.step(xs[s - 1], out, timestep(cfg, s, T), s, class_ids=cls, ctx=ctx, stream=stream)
+            e1.record(stream)
+            torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        executed = cfg.n_blocks * T if mode == binding.EXEC_PADDED_GRAPH else int(sum(S)) // len(cfg.branches)
+        rows.append({"mode": name, "trajectory_ms": round(ms, 2), "layer_steps_executed": executed})
+    model.set_exec_mode(binding.EXEC_JAGGED_GRAPH)
+    model.set_schedule(T, sched["lifetimes"], sched["groups"])
+    base = rows[0]["trajectory_ms"]
+    for r in rows:
+        r["speedup_vs_eager_full"] = round(base / r["trajectory_ms"], 3)
+    return rows
 
 
 def workload_name(cfg, T, budget):

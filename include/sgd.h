@@ -33,6 +33,14 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#ifndef SGD_API
+#if defined(__GNUC__)
+#define SGD_API __attribute__((visibility("default")))
+#else
+#define SGD_API
+#endif
+#endif
+
 #ifdef __cplusplus
 extern "C" {
 #endif
@@ -87,6 +95,8 @@ typedef enum {
 
 /* Debug flag: run every GEMM on the plain SIMT kernel instead of tcgen05. */
 #define SGD_FLAG_SIMT_GEMM 1
+/* Run every attention on the mma.sync kernel instead of tcgen05 (d_head 64 / 128). */
+#define SGD_FLAG_MMA_SYNC_ATTENTION 2
 
 typedef struct {
   int stem, block, norm, mlp, head;   /* enums above                                   */
@@ -160,7 +170,7 @@ typedef struct sgd_ctx sgd_ctx;
  * must stay valid and unchanged for the context's lifetime.
  * Errors: SGD_ERR_ARG (null/misaligned), SGD_ERR_SHAPE, SGD_ERR_OOM, SGD_ERR_CUDA.
  */
-int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out);
+SGD_API int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out);
 
 /*
  * sgd_set_schedule — install per-unit lifetimes (Sec. 4.1, Eq. schedule) with their
@@ -173,7 +183,7 @@ int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out);
  * Units are the residual branches in graph order: per block attn[, xattn], mlp.
  * Errors: SGD_ERR_SCHEDULE (bad lifetime, split group, n_units mismatch), SGD_ERR_CUDA.
  */
-int sgd_set_schedule(sgd_ctx* ctx, int T, int n_units, const int32_t* lifetimes_host,
+SGD_API int sgd_set_schedule(sgd_ctx* ctx, int T, int n_units, const int32_t* lifetimes_host,
                      const int32_t* group_of_unit_host);
 
 /*
@@ -185,7 +195,7 @@ int sgd_set_schedule(sgd_ctx* ctx, int T, int n_units, const int32_t* lifetimes_
  * Errors: SGD_ERR_STATE (no schedule), SGD_ERR_CACHE_INVALID (out-of-order step),
  * SGD_ERR_ARG, SGD_ERR_CUDA.  Kernel timeouts surface through sgd_check_device.
  */
-int sgd_step(sgd_ctx* ctx, const void* state_in_dev, void* out_dev, float timestep,
+SGD_API int sgd_step(sgd_ctx* ctx, const void* state_in_dev, void* out_dev, float timestep,
              const sgd_cond* cond, int step, void* stream);
 
 /*
@@ -194,27 +204,42 @@ int sgd_step(sgd_ctx* ctx, const void* state_in_dev, void* out_dev, float timest
  * on `stream`; returns after the output has arrived in out_host.  Pinned host
  * buffers give asynchronous copies.
  */
-int sgd_step_host(sgd_ctx* ctx, const void* state_in_host, void* out_host, float timestep,
+SGD_API int sgd_step_host(sgd_ctx* ctx, const void* state_in_host, void* out_host, float timestep,
                   const int32_t* class_ids_host, const void* ctx_host, int step, void* stream);
 
 /* sgd_get_active_mask — mask_host[u] = 1 iff unit u is evaluated at `step` (1..T). */
-int sgd_get_active_mask(const sgd_ctx* ctx, int step, uint8_t* mask_host, int n_units);
+SGD_API int sgd_get_active_mask(const sgd_ctx* ctx, int step, uint8_t* mask_host, int n_units);
 
 /* sgd_get_info — sizes and schedule statistics. */
-int sgd_get_info(const sgd_ctx* ctx, sgd_info* info);
+SGD_API int sgd_get_info(const sgd_ctx* ctx, sgd_info* info);
+
+/*
+ * Execution modes (the execution ablation of Table tab:kernel):
+ *   SGD_EXEC_JAGGED_GRAPH  default: one captured graph per active pattern, frozen units
+ *                          launch no branch work (Sec. 4.2).
+ *   SGD_EXEC_EAGER         the same per-step op list launched op by op from the host
+ *                          (host-side skipping of frozen units, no graphs); with a 100%
+ *                          schedule it is eager full inference.
+ *   SGD_EXEC_PADDED_GRAPH  one graph per pattern that still evaluates every frozen
+ *                          branch and discards its update (into a scratch residual),
+ *                          then adds the cached update: all layer-steps executed.
+ * All modes give bit-identical outputs.  Changing the mode resets the trajectory.
+ */
+enum { SGD_EXEC_JAGGED_GRAPH = 0, SGD_EXEC_EAGER = 1, SGD_EXEC_PADDED_GRAPH = 2 };
+SGD_API int sgd_set_exec_mode(sgd_ctx* ctx, int mode);
 
 /* sgd_reset — start a new trajectory: the next step must be 1 (caches invalidated). */
-int sgd_reset(sgd_ctx* ctx);
+SGD_API int sgd_reset(sgd_ctx* ctx);
 
 /* sgd_check_device — synchronise `stream` and report a device-side status word set by
  * a kernel whose bounded wait expired (SGD_ERR_DEVICE_TIMEOUT); clears it. */
-int sgd_check_device(sgd_ctx* ctx, void* stream);
+SGD_API int sgd_check_device(sgd_ctx* ctx, void* stream);
 
 /* sgd_destroy — free everything the context owns (graphs, caches, workspaces). */
-void sgd_destroy(sgd_ctx* ctx);
+SGD_API void sgd_destroy(sgd_ctx* ctx);
 
 /* sgd_last_error — message of the last failing call on this thread ("" if none). */
-const char* sgd_last_error(void);
+SGD_API const char* sgd_last_error(void);
 
 /*
  * sgd_compile_schedule — host-only schedule compiler (no device needed): validates
@@ -224,7 +249,7 @@ const char* sgd_last_error(void);
  * therefore store their update at s), and *n_patterns.  Arrays are [T]; any of them
  * may be NULL.
  */
-int sgd_compile_schedule(int T, int n_units, const int32_t* lifetimes_host,
+SGD_API int sgd_compile_schedule(int T, int n_units, const int32_t* lifetimes_host,
                          const int32_t* group_of_unit_host, int32_t* pattern_of_step_host,
                          int32_t* writes_at_step_host, int32_t* n_patterns);
 
@@ -247,7 +272,7 @@ enum {
  * with a CUDA event pair around every op on `stream`; synchronises and fills up to
  * max_records entries.  Same ordering rules as sgd_step.
  */
-int sgd_step_profile(sgd_ctx* ctx, const void* state_in_dev, void* out_dev, float timestep,
+SGD_API int sgd_step_profile(sgd_ctx* ctx, const void* state_in_dev, void* out_dev, float timestep,
                      const sgd_cond* cond, int step, void* stream, sgd_op_record* records_host,
                      int max_records, int* n_records);
 
@@ -255,7 +280,7 @@ int sgd_step_profile(sgd_ctx* ctx, const void* state_in_dev, void* out_dev, floa
  * sgd_sampler_update — z <- alpha z - beta eps, elementwise on n fp32 values (the
  * deterministic update of Sec. 3.1), asynchronous on `stream`.
  */
-int sgd_sampler_update(float* z_dev, const float* eps_dev, float alpha, float beta, int64_t n,
+SGD_API int sgd_sampler_update(float* z_dev, const float* eps_dev, float alpha, float beta, int64_t n,
                        void* stream);
 
 #ifdef __cplusplus

@@ -24,6 +24,14 @@
 
 #include <stdint.h>
 
+#ifndef SGD_API
+#if defined(__GNUC__)
+#define SGD_API __attribute__((visibility("default")))
+#else
+#define SGD_API
+#endif
+#endif
+
 #ifdef __cplusplus
 extern "C" {
 #endif
@@ -61,25 +69,27 @@ typedef struct {
  * tcgen05 + TMA kernel (M = 128, N = 256, K = 16 instructions, fp32 accumulators in
  * TMEM).
  */
-int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
+SGD_API int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
                     const sgd_epilogue_args* epi, int use_simt, void* stream);
 
 /*
  * O = softmax(Q K^T / sqrt(d_head)) V per (sample, head), non-causal, keys beyond n_kv
  * masked.  Row r = b * n_q + i of q / o, row b * n_kv + j of k / v; head h occupies
  * columns [h d_head, (h+1) d_head).  fp16 in and out; d_head in {64, 72, 128};
- * leading dimensions in elements, multiples of 8.
+ * leading dimensions in elements, multiples of 8.  impl = 0: the tcgen05 kernel for
+ * d_head 64 / 128 (S and O in TMEM), the mma.sync kernel for 72; impl = 1: the
+ * mma.sync kernel for every d_head.
  */
-int sgd_kernel_attention(const void* q, int ldq, const void* k, const void* v, int ldkv,
+SGD_API int sgd_kernel_attention(const void* q, int ldq, const void* k, const void* v, int ldkv,
                          void* o, int ldo, int batch, int n_q, int n_kv, int n_heads,
-                         int d_head, void* stream);
+                         int d_head, int impl, void* stream);
 
 /*
  * out fp16 [rows, d] = norm(h fp32 [rows, d]); kind = sgd_norm_kind.  g, b: bf16 [d]
  * (NULL allowed for LN_PLAIN).  shift/scale: optional fp32 AdaLN modulation
  * [B, ld_mod]: out = norm(h) * (1 + scale[r / rows_per_batch]) + shift[...].
  */
-int sgd_kernel_norm(const float* h, void* out, int rows, int d, int kind, const void* g,
+SGD_API int sgd_kernel_norm(const float* h, void* out, int rows, int d, int kind, const void* g,
                     const void* b, const float* shift, const float* scale, int ld_mod,
                     int rows_per_batch, float eps, void* stream);
 
@@ -88,11 +98,11 @@ int sgd_kernel_norm(const float* h, void* out, int rows, int d, int kind, const 
  * in fp32.  caches_host: host array of n_caches (<= 96) device pointers.  n multiple
  * of 8, pointers 16-byte aligned.
  */
-int sgd_kernel_frozen_run(float* h, const void* const* caches_host, int n_caches, int64_t n,
+SGD_API int sgd_kernel_frozen_run(float* h, const void* const* caches_host, int n_caches, int64_t n,
                           void* stream);
 
 /* Device status word shared by all kernels (bounded-wait expiry); returns and clears it. */
-int sgd_kernel_status(int* status_host);
+SGD_API int sgd_kernel_status(int* status_host);
 
 #ifdef __cplusplus
 }

@@ -36,6 +36,7 @@ NORM = {"rms": 0, "ln": 1, "ln_plain": 2}
 MLP = {"swiglu": 0, "gelu_tanh": 1, "gelu_erf": 2, "geglu": 3}
 HEAD = {"linear": 0, "adaln_linear": 1, "identity": 2, "logits": 3}
 FLAG_SIMT_GEMM = 1
+FLAG_MMA_SYNC_ATTENTION = 2
 
 EPI_F16, EPI_F32, EPI_DELTA, EPI_GATED, EPI_GELU, EPI_ROPE = range(6)
 KERNEL_NAMES = ["gemm_tc", "gemm_simt", "attention", "norm", "frozen_run", "small"]
@@ -46,7 +47,9 @@ EXPORTED = [
     "sgd_get_info", "sgd_reset", "sgd_check_device", "sgd_destroy", "sgd_last_error",
     "sgd_compile_schedule", "sgd_step_profile", "sgd_sampler_update", "sgd_kernel_gemm",
     "sgd_kernel_attention", "sgd_kernel_norm", "sgd_kernel_frozen_run", "sgd_kernel_status",
+    "sgd_set_exec_mode",
 ]
+EXEC_JAGGED_GRAPH, EXEC_EAGER, EXEC_PADDED_GRAPH = 0, 1, 2
 
 
 class sgd_model_desc(C.Structure):
@@ -122,10 +125,11 @@ def lib() -> C.CDLL:
                                      C.POINTER(sgd_op_record), i, C.POINTER(C.c_int)]),
             "sgd_sampler_update": (i, [vp, vp, f, f, i64, vp]),
             "sgd_kernel_gemm": (i, [vp, i, vp, i, i, i, i, C.POINTER(sgd_epilogue_args), i, vp]),
-            "sgd_kernel_attention": (i, [vp, i, vp, vp, i, vp, i, i, i, i, i, i, vp]),
+            "sgd_kernel_attention": (i, [vp, i, vp, vp, i, vp, i, i, i, i, i, i, i, vp]),
             "sgd_kernel_norm": (i, [vp, vp, i, i, i, vp, vp, vp, vp, i, i, f, vp]),
             "sgd_kernel_frozen_run": (i, [vp, C.POINTER(vp), i, i64, vp]),
             "sgd_kernel_status": (i, [C.POINTER(C.c_int)]),
+            "sgd_set_exec_mode": (i, [vp, i]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -183,10 +187,10 @@ def sgd_kernel_gemm(A, B, M, N, K, epi: sgd_epilogue_args, use_simt=False, lda=N
 
 
 def sgd_kernel_attention(q, ldq, k, v, ldkv, o, ldo, batch, n_q, n_kv, n_heads, d_head,
-                         stream=None):
+                         impl=0, stream=None):
     return check(lib().sgd_kernel_attention(_ptr(q), ldq, _ptr(k), _ptr(v), ldkv, _ptr(o), ldo,
-                                            batch, n_q, n_kv, n_heads, d_head, _stream(stream)),
-                 "sgd_kernel_attention")
+                                            batch, n_q, n_kv, n_heads, d_head, impl,
+                                            _stream(stream)), "sgd_kernel_attention")
 
 
 def sgd_kernel_norm(h, out, rows, d, kind, g=None, b=None, shift=None, scale=None, ld_mod=0,
@@ -308,6 +312,9 @@ class Denoiser:
 
     def reset(self):
         check(lib().sgd_reset(self.handle), "sgd_reset")
+
+    def set_exec_mode(self, mode: int):
+        check(lib().sgd_set_exec_mode(self.handle, mode), "sgd_set_exec_mode")
 
     def check_device(self, stream=None):
         return check(lib().sgd_check_device(self.handle, _stream(stream)), "sgd_check_device")

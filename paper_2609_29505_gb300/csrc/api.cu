@@ -125,6 +125,9 @@ struct sgd_ctx {
   sgd_weights w{};
   int device = 0;
   int M = 0, U = 0, nbr = 0;
+  int attn_impl = 0;  // 1: mma.sync attention everywhere (SGD_FLAG_MMA_SYNC_ATTENTION)
+  int exec_mode = SGD_EXEC_JAGGED_GRAPH;
+  float* h_pad = nullptr;  // padded mode: residual that discarded branch updates land in
   // buffers
   float* h = nullptr;
   f16* xn = nullptr;
@@ -269,14 +272,16 @@ void make_norm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, int
 
 int make_attn_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, const AttnParams& p) {
   const char* why = "";
-  if (attn_check(p, &why) != 0) return fail(SGD_ERR_SHAPE, name + ": " + why);
+  auto plan = std::make_shared<AttnPlan>();
+  plan->p = p;
+  if (attn_plan(*plan, &why) != 0) return fail(SGD_ERR_SHAPE, name + ": " + why);
   Op op;
   op.name = name;
   op.kernel = SGD_KERNEL_ATTENTION;
   const double dm = static_cast<double>(p.n_heads) * p.d_head;
   op.flops = 4.0 * p.batch * p.n_heads * static_cast<double>(p.n_q) * p.n_kv * p.d_head;
   op.bytes = 2.0 * p.batch * (2.0 * p.n_q * dm + 2.0 * p.n_kv * dm);
-  op.run = [p](cudaStream_t s) { return attn_launch(p, s); };
+  op.run = [plan](cudaStream_t s) { return attn_launch(*plan, s); };
   ops.push_back(std::move(op));
   return SGD_OK;
 }
@@ -310,7 +315,8 @@ void flush_run(sgd_ctx* c, std::vector<Op>& ops, std::vector<const f16*>& run, i
   run.clear();
 }
 
-int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_cache, int u) {
+int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_cache, int u,
+                 bool discard = false) {
   const sgd_model_desc& d = c->d;
   const sgd_block_weights& W = c->blk[b];
   const BlockPW& P = c->pw[b];
@@ -320,9 +326,9 @@ int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_c
   float* mod = adaln ? c->mod + static_cast<size_t>(b) * d.batch * 6 * D : nullptr;
   f16* cache = write_cache ? c->cache[u] : nullptr;
   EpiParams delta = epi_base(SGD_EPI_DELTA);
-  delta.h = c->h;
+  delta.h = discard ? c->h_pad : c->h;
   delta.ldh = D;
-  delta.cache = cache;
+  delta.cache = discard ? nullptr : cache;
   delta.ld_cache = D;
   int rc;
   if (kind == 0) {  // self-attention
@@ -341,7 +347,7 @@ int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_c
     if ((rc = make_gemm_op(c, ops, pre + "attn.qkv", c->xn, D, P.qkv, D, M, 3 * D, D, e)))
       return rc;
     AttnParams ap{c->qkv, 3 * D, c->qkv + D, c->qkv + 2 * D, 3 * D, c->attn, D,
-                  d.batch, d.n_tokens, d.n_tokens, d.n_heads, d.d_head};
+                  d.batch, d.n_tokens, d.n_tokens, d.n_heads, d.d_head, c->attn_impl};
     if ((rc = make_attn_op(c, ops, pre + "attn.sdpa", ap))) return rc;
     if (adaln) {
       delta.gate = mod + 2 * D;
@@ -357,7 +363,7 @@ int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_c
     e.ldo = D;
     if ((rc = make_gemm_op(c, ops, pre + "xattn.q", c->xn, D, P.xq, D, M, D, D, e))) return rc;
     AttnParams ap{c->qkv, D, c->ctxkv[b], c->ctxkv[b] + D, 2 * D, c->attn, D,
-                  d.batch, d.n_tokens, d.ctx_len, d.n_heads, d.d_head};
+                  d.batch, d.n_tokens, d.ctx_len, d.n_heads, d.d_head, c->attn_impl};
     if ((rc = make_attn_op(c, ops, pre + "xattn.sdpa", ap))) return rc;
     return make_gemm_op(c, ops, pre + "xattn.out", c->attn, D, P.xo, D, M, D, D, delta);
   }
@@ -482,6 +488,11 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
         flush_run(c, ops, run, run_first);
         if ((rc = build_branch(c, ops, b, kind, write[u] != 0, u))) return rc;
       } else {
+        if (c->exec_mode == SGD_EXEC_PADDED_GRAPH) {
+          // padded execution: the frozen branch is evaluated anyway and its update discarded
+          flush_run(c, ops, run, run_first);
+          if ((rc = build_branch(c, ops, b, kind, false, u, true))) return rc;
+        }
         if (run.empty()) run_first = u;
         run.push_back(c->cache[u]);
       }
@@ -833,6 +844,7 @@ int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out) 
     return fail(SGD_ERR_CUDA, "no CUDA device");
   }
   c->M = desc->batch * desc->n_tokens;
+  c->attn_impl = (desc->flags & SGD_FLAG_MMA_SYNC_ATTENTION) ? 1 : 0;
   c->nbr = desc->block == SGD_BLOCK_XATTN ? 3 : 2;
   c->U = desc->n_blocks * c->nbr;
   if ((rc = ensure_alloc(c)) || (rc = prep_weights(c))) {
@@ -863,21 +875,10 @@ int sgd_compile_schedule(int T, int n_units, const int32_t* lifetimes, const int
   return SGD_OK;
 }
 
-int sgd_set_schedule(sgd_ctx* c, int T, int n_units, const int32_t* lifetimes, const int32_t* groups) {
-  if (!c) return fail(SGD_ERR_ARG, "null context");
-  int rc = validate_schedule(T, n_units, lifetimes, groups, c->U);
-  if (rc) return rc;
-  CUDA_TRY(cudaSetDevice(c->device));
+static int build_graphs(sgd_ctx* c) {
+  const int T = c->T;
+  int rc;
   drop_graphs(c);
-  c->T = T;
-  c->S.assign(lifetimes, lifetimes + n_units);
-  c->groups.assign(groups, groups + n_units);
-  compile_patterns(T, n_units, lifetimes, c->pattern_of_step, c->writes, c->patterns);
-  // caches only for units that are ever frozen
-  for (int u = 0; u < c->U; ++u)
-    if (c->S[u] < T && !c->cache[u]) {
-      if ((rc = c->alloc(&c->cache[u], static_cast<size_t>(c->M) * c->d.d, &c->cache_bytes))) return rc;
-    }
   // graph variants: (pattern, cache-store set); the store set is non-empty only at steps
   // s = S_u < T, so each such step gets its own variant.
   std::map<std::pair<int, int>, int> key_to_graph;
@@ -918,7 +919,44 @@ int sgd_set_schedule(sgd_ctx* c, int T, int n_units, const int32_t* lifetimes, c
   }
   c->last_step = 0;
   c->scheduled = true;
+  return SGD_OK;
+}
+
+int sgd_set_schedule(sgd_ctx* c, int T, int n_units, const int32_t* lifetimes, const int32_t* groups) {
+  if (!c) return fail(SGD_ERR_ARG, "null context");
+  int rc = validate_schedule(T, n_units, lifetimes, groups, c->U);
+  if (rc) return rc;
+  CUDA_TRY(cudaSetDevice(c->device));
+  drop_graphs(c);
+  c->T = T;
+  c->S.assign(lifetimes, lifetimes + n_units);
+  c->groups.assign(groups, groups + n_units);
+  compile_patterns(T, n_units, lifetimes, c->pattern_of_step, c->writes, c->patterns);
+  // caches only for units that are ever frozen
+  for (int u = 0; u < c->U; ++u)
+    if (c->S[u] < T && !c->cache[u]) {
+      if ((rc = c->alloc(&c->cache[u], static_cast<size_t>(c->M) * c->d.d, &c->cache_bytes))) return rc;
+    }
+  if ((rc = build_graphs(c))) return rc;
   g_err.clear();
+  return SGD_OK;
+}
+
+int sgd_set_exec_mode(sgd_ctx* c, int mode) {
+  if (!c) return fail(SGD_ERR_ARG, "null context");
+  if (mode < SGD_EXEC_JAGGED_GRAPH || mode > SGD_EXEC_PADDED_GRAPH)
+    return fail(SGD_ERR_ARG, "unknown execution mode");
+  int rc;
+  if (mode == SGD_EXEC_PADDED_GRAPH && !c->h_pad &&
+      (rc = c->alloc(&c->h_pad, static_cast<size_t>(c->M) * c->d.d, &c->ws_bytes)))
+    return rc;
+  const bool rebuild = (mode == SGD_EXEC_PADDED_GRAPH) != (c->exec_mode == SGD_EXEC_PADDED_GRAPH);
+  c->exec_mode = mode;
+  if (rebuild && c->scheduled) {
+    CUDA_TRY(cudaSetDevice(c->device));
+    if ((rc = build_graphs(c))) return rc;
+  }
+  c->last_step = 0;
   return SGD_OK;
 }
 
@@ -928,7 +966,11 @@ int sgd_step(sgd_ctx* c, const void* in, void* out, float t, const sgd_cond* con
   if (rc) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if ((rc = prepare_step(c, in, out, t, cond, step, s))) return rc;
-  CUDA_TRY(cudaGraphLaunch(c->execs[c->graph_of_step[step]], s));
+  if (c->exec_mode == SGD_EXEC_EAGER) {
+    if ((rc = run_ops(c->programs[c->graph_of_step[step]], s))) return rc;  // one launch per op
+  } else {
+    CUDA_TRY(cudaGraphLaunch(c->execs[c->graph_of_step[step]], s));
+  }
   c->last_step = step == c->T ? 0 : step;
   return SGD_OK;
 }
@@ -1094,13 +1136,16 @@ int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N
 }
 
 int sgd_kernel_attention(const void* q, int ldq, const void* k, const void* v, int ldkv, void* o,
-                         int ldo, int batch, int n_q, int n_kv, int n_heads, int d_head, void* stream) {
-  AttnParams p{H16(q), ldq, H16(k), H16(v), ldkv, static_cast<f16*>(o), ldo,
-               batch, n_q, n_kv, n_heads, d_head};
+                         int ldo, int batch, int n_q, int n_kv, int n_heads, int d_head, int impl,
+                         void* stream) {
+  if (impl < 0 || impl > 1) return fail(SGD_ERR_ARG, "attention: impl must be 0 or 1");
+  AttnPlan plan;
+  plan.p = AttnParams{H16(q), ldq, H16(k), H16(v), ldkv, static_cast<f16*>(o), ldo,
+                      batch, n_q, n_kv, n_heads, d_head, impl};
   const char* why = "";
-  const int rc = attn_check(p, &why);
-  if (rc) return fail(rc == -1 ? SGD_ERR_ARG : SGD_ERR_SHAPE, why);
-  CUDA_TRY(attn_launch(p, static_cast<cudaStream_t>(stream)));
+  const int rc = attn_plan(plan, &why);
+  if (rc) return fail(rc == -1 ? SGD_ERR_ARG : (rc == -5 ? SGD_ERR_CUDA : SGD_ERR_SHAPE), why);
+  CUDA_TRY(attn_launch(plan, static_cast<cudaStream_t>(stream)));
   return SGD_OK;
 }
 

@@ -3,12 +3,25 @@
 // Used inside every active self-attention and cross-attention branch (Algorithm 2:
 // an active unit evaluates F_l(h_{l-1,s}; c_s)); frozen units never launch it.
 //
-// One CTA = 64 query rows of one (sample, head), 4 warps x 16 rows.  K/V tiles of
+// Two kernels:
+//   attn_tc_kernel (d_h 64, 128): tcgen05.  One CTA = 128 queries of one (sample, head),
+//     keys in tiles of 128.  Warp 0 loads Q once and K/V tiles through a 2-stage TMA ring;
+//     warp 1 issues S = Q K^T into one of two TMEM S buffers and O += P V into a TMEM O
+//     accumulator (V read as an MN-major operand straight from its row-major tile);
+//     warps 2-5 (one query row per thread) read S from TMEM, run the online softmax in
+//     fp32 and write P (fp16) into a 128-byte-swizzled shared tile for the next MMA.  O
+//     is rescaled only when a row maximum grows by more than 2^8 (P <= 256 otherwise),
+//     which keeps the result exact while avoiding most TMEM round trips.
+//   attn_kernel (any of 64, 72, 128): mma.sync, described below; used for d_h = 72.
+//
+// mma.sync kernel: one CTA = 64 query rows of one (sample, head), 4 warps x 16 rows.  K/V tiles of
 // 64 keys stream through a double-buffered cp.async ring; S = Q K^T and O += P V run
 // on mma.sync m16n8k16 (fp16 in, fp32 accumulate) with an online softmax in
 // registers (exp2 with the scale folded in).  Q, K, V, P and O are fp16 (m16n8k16
 // f16 x f16 -> f32).  Keys beyond n_kv are masked and their
 // shared-memory rows zero-filled; head dims 72 are padded to 80 in shared memory.
+#include <cstring>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -229,6 +242,292 @@ __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnParams p) {
   }
 }
 
+// ----------------------------------------------------------------------------
+// tcgen05 flash attention
+// ----------------------------------------------------------------------------
+
+constexpr int kTcThreads = 192;
+constexpr int kTcBQ = 128;
+constexpr int kTcBK = 128;
+constexpr int kAtom = 128 * 64 * 2;  // 128 rows x 64 fp16: one 128-byte-swizzle column block
+constexpr float kRescaleLog2 = 8.f;  // rescale O only when the row max grows by > 2^8
+
+struct AttnTcArgs {
+  CUtensorMap tmap_q;
+  CUtensorMap tmap_k;
+  CUtensorMap tmap_v;
+  f16* o;
+  int ldo;
+  int n_q, n_kv, n_heads;
+  float scale_log2;
+  int* status;
+};
+
+template <int DH>
+struct TcLayout {
+  static constexpr int kAtoms = DH / 64;
+  static constexpr int kQ = 0;
+  static constexpr int kKV = kAtoms * kAtom;           // stage s: K atoms, then V atoms
+  static constexpr int kStage = 2 * kAtoms * kAtom;
+  static constexpr int kP = kKV + 2 * kStage;          // two P buffers of 128 keys
+  static constexpr int kPBuf = 2 * kAtom;
+  static constexpr int kBar = kP + 2 * kPBuf;
+  static constexpr int kBytes = kBar + 256 + 1024;
+  static constexpr uint32_t kTmemS = 0;                // S buffers at columns 0, 128
+  static constexpr uint32_t kTmemO = 256;              // O at columns 256 .. 256 + DH
+};
+
+__device__ __forceinline__ bool warp_wait_bar(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                              int* status, int code) {
+  int ok = 0;
+  if (lane_id() == 0) ok = mbar_wait(bar, parity, abort_flag, status, code) ? 1 : 0;
+  return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
+__device__ __forceinline__ void drain_bar(uint64_t* bar, uint32_t parity) {
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (global_timer_ns() - t0 > kWaitTimeoutNs) break;
+  }
+}
+
+template <int DH>
+__global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const __grid_constant__ AttnTcArgs a) {
+  using L = TcLayout<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L::kBar);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;
+  uint64_t* kv_empty = bars + 3;
+  uint64_t* s_full = bars + 5;
+  uint64_t* s_free = bars + 7;
+  uint64_t* p_full = bars + 9;
+  uint64_t* o_done = bars + 11;
+  uint64_t* drain = bars + 13;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 14);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qt = blockIdx.x, bh = blockIdx.y;
+  const int b = bh / a.n_heads, h = bh % a.n_heads;
+  const int nt = (a.n_kv + kTcBK - 1) / kTcBK;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&kv_full[i], 1);
+      mbar_init(&kv_empty[i], 1);
+      mbar_init(&s_full[i], 1);
+      mbar_init(&s_free[i], 4);
+      mbar_init(&p_full[i], 4);
+      mbar_init(&o_done[i], 1);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&a.tmap_q);
+    tma_prefetch_desc(&a.tmap_k);
+    tma_prefetch_desc(&a.tmap_v);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      mbar_arrive_expect_tx(q_full, L::kAtoms * kAtom);
+      for (int at = 0; at < L::kAtoms; ++at)
+        tma_load_2d(sm + L::kQ + at * kAtom, &a.tmap_q, q_full, h * DH + at * 64,
+                    b * a.n_q + qt * kTcBQ);
+      int j = 0;
+      for (; j < nt; ++j) {
+        const int s = j & 1;
+        if (!mbar_wait(&kv_empty[s], ((j >> 1) & 1) ^ 1u, abort_flag, a.status, 11)) break;
+        uint8_t* st = sm + L::kKV + s * L::kStage;
+        mbar_arrive_expect_tx(&kv_full[s], 2 * L::kAtoms * kAtom);
+        const int row = b * a.n_kv + j * kTcBK;
+        for (int at = 0; at < L::kAtoms; ++at) {
+          tma_load_2d(st + at * kAtom, &a.tmap_k, &kv_full[s], h * DH + at * 64, row);
+          tma_load_2d(st + (L::kAtoms + at) * kAtom, &a.tmap_v, &kv_full[s], h * DH + at * 64, row);
+        }
+      }
+      if (*abort_flag) {
+        drain_bar(q_full, 0);
+        for (int i = (j > 2 ? j - 2 : 0); i < j; ++i) drain_bar(&kv_full[i & 1], (i >> 1) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc_qk = umma_idesc_f16(kTcBQ, kTcBK);
+      const uint32_t idesc_pv = umma_idesc_f16_bmn(kTcBQ, DH);
+      bool ok = mbar_wait(q_full, 0, abort_flag, a.status, 12);
+      auto issue_qk = [&](int j) -> bool {
+        const int s = j & 1;
+        const uint32_t ph = (j >> 1) & 1;
+        if (!mbar_wait(&kv_full[s], ph, abort_flag, a.status, 13)) return false;
+        if (!mbar_wait(&s_free[s], ph ^ 1u, abort_flag, a.status, 14)) return false;
+        tc_fence_after();
+        const uint32_t qa = smem_u32(sm + L::kQ);
+        const uint32_t ka = smem_u32(sm + L::kKV + s * L::kStage);
+#pragma unroll
+        for (int ks = 0; ks < DH / 16; ++ks) {
+          const uint32_t off = (ks >> 2) * kAtom + (ks & 3) * 32;
+          umma_f16(tmem + L::kTmemS + s * kTcBK, smem_desc_sw128(qa + off), smem_desc_sw128(ka + off),
+                   idesc_qk, ks > 0 ? 1u : 0u);
+        }
+        umma_commit(&s_full[s]);
+        return true;
+      };
+      if (ok) ok = issue_qk(0);
+      for (int j = 0; j < nt && ok; ++j) {
+        if (j + 1 < nt && !(ok = issue_qk(j + 1))) break;
+        const int s = j & 1;
+        if (!(ok = mbar_wait(&p_full[s], (j >> 1) & 1, abort_flag, a.status, 15))) break;
+        tc_fence_after();
+        const uint32_t pa = smem_u32(sm + L::kP + s * L::kPBuf);
+        const uint32_t va = smem_u32(sm + L::kKV + s * L::kStage + L::kAtoms * kAtom);
+#pragma unroll
+        for (int ks = 0; ks < kTcBK / 16; ++ks) {
+          const uint64_t ad = smem_desc_sw128(pa + (ks >> 2) * kAtom + (ks & 3) * 32);
+          const uint64_t bd = smem_desc_sw128_mn(va + ks * 2048, kAtom, 1024);
+          umma_f16(tmem + L::kTmemO, ad, bd, idesc_pv, (j > 0 || ks > 0) ? 1u : 0u);
+        }
+        umma_commit(&kv_empty[s]);
+        umma_commit(&o_done[s]);
+      }
+      umma_commit(drain);
+      drain_bar(drain, 0);
+    }
+  } else {
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    const uint32_t lane_base = static_cast<uint32_t>(q * 32) << 16;
+    float m2 = -INFINITY, l = 0.f;
+    bool ok = true;
+    uint32_t r[kTcBK];
+    for (int j = 0; j < nt; ++j) {
+      const int s = j & 1;
+      if (!(ok = warp_wait_bar(&s_full[s], (j >> 1) & 1, abort_flag, a.status, 16))) break;
+      tc_fence_after();
+#pragma unroll
+      for (int c = 0; c < kTcBK / 16; ++c) tmem_ld16(tmem + lane_base + L::kTmemS + s * kTcBK + 16 * c, r + 16 * c);
+#pragma unroll
+      for (int c = 0; c < kTcBK / 16; ++c) tmem_ld_wait16(r + 16 * c);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[s]);
+      const int kb = j * kTcBK;
+      float mt = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < kTcBK; ++c) {
+        const float v = (kb + c < a.n_kv) ? __uint_as_float(r[c]) * a.scale_log2 : -INFINITY;
+        r[c] = __float_as_uint(v);
+        mt = fmaxf(mt, v);
+      }
+      if (j == 0) {
+        m2 = mt;
+      } else if (mt > m2 + kRescaleLog2) {
+        // O must hold PV_{j-1} complete before it is rescaled
+        if (!(ok = warp_wait_bar(&o_done[(j - 1) & 1], ((j - 1) >> 1) & 1, abort_flag, a.status, 17))) break;
+        tc_fence_after();
+        const float corr = exp2f(m2 - mt);
+        uint32_t o16[16];
+#pragma unroll
+        for (int c = 0; c < DH / 16; ++c) {
+          tmem_ld16(tmem + lane_base + L::kTmemO + 16 * c, o16);
+          tmem_ld_wait16(o16);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) o16[i] = __float_as_uint(__uint_as_float(o16[i]) * corr);
+          tmem_st16(tmem + lane_base + L::kTmemO + 16 * c, o16);
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        l *= corr;
+        m2 = mt;
+      }
+      // P buffer s was last read by PV_{j-2}
+      if (j >= 2 && !(ok = warp_wait_bar(&o_done[s], ((j - 2) >> 1) & 1, abort_flag, a.status, 18))) break;
+      uint8_t* pbuf = sm + L::kP + s * L::kPBuf;
+#pragma unroll
+      for (int cc = 0; cc < kTcBK / 8; ++cc) {
+        float p8[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          p8[i] = exp2f(__uint_as_float(r[cc * 8 + i]) - m2);
+          l += p8[i];
+        }
+        uint8_t* dst = pbuf + (cc >> 3) * kAtom + row * 128 + ((((cc & 7) ^ (row & 7))) << 4);
+        *reinterpret_cast<uint4*>(dst) = pack_f16x8(p8);
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[s]);
+    }
+    if (ok && warp_wait_bar(&o_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, abort_flag, a.status, 19)) {
+      tc_fence_after();
+      const float inv = 1.f / l;
+      const int qrow = qt * kTcBQ + row;
+      f16* orow = a.o + (static_cast<int64_t>(b) * a.n_q + qrow) * a.ldo + h * DH;
+      uint32_t o16[16];
+#pragma unroll
+      for (int c = 0; c < DH / 16; ++c) {
+        tmem_ld16(tmem + lane_base + L::kTmemO + 16 * c, o16);
+        tmem_ld_wait16(o16);
+        float f[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(o16[i]) * inv;
+        if (qrow < a.n_q) {
+          reinterpret_cast<uint4*>(orow + 16 * c)[0] = pack_f16x8(f);
+          reinterpret_cast<uint4*>(orow + 16 * c)[1] = pack_f16x8(f + 8);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+template <int DH>
+cudaError_t launch_tc(const AttnPlan& plan, cudaStream_t s) {
+  using L = TcLayout<DH>;
+  static bool done[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !done[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         L::kBytes);
+    if (e != cudaSuccess) return e;
+    done[dev] = true;
+  }
+  const AttnParams& p = plan.p;
+  AttnTcArgs a;
+  memcpy(&a.tmap_q, &plan.tmap_q, sizeof(CUtensorMap));
+  memcpy(&a.tmap_k, &plan.tmap_kv, sizeof(CUtensorMap));
+  memcpy(&a.tmap_v, &plan.tmap_v, sizeof(CUtensorMap));
+  a.o = p.o;
+  a.ldo = p.ldo;
+  a.n_q = p.n_q;
+  a.n_kv = p.n_kv;
+  a.n_heads = p.n_heads;
+  a.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(DH));
+  a.status = device_status_ptr();
+  dim3 grid((p.n_q + kTcBQ - 1) / kTcBQ, p.batch * p.n_heads);
+  attn_tc_kernel<DH><<<grid, kTcThreads, L::kBytes, s>>>(a);
+  return cudaGetLastError();
+}
+
 template <int DH, int DP>
 cudaError_t launch_dh(const AttnParams& p, cudaStream_t s) {
   constexpr int kPitch = DP + 8;
@@ -272,7 +571,25 @@ int attn_check(const AttnParams& p, const char** why) {
   return 0;
 }
 
-cudaError_t attn_launch(const AttnParams& p, cudaStream_t s) {
+int attn_plan(AttnPlan& plan, const char** why) {
+  const AttnParams& p = plan.p;
+  int rc = attn_check(p, why);
+  if (rc) return rc;
+  plan.tc = p.impl == 0 && (p.d_head == 64 || p.d_head == 128);
+  if (!plan.tc) return 0;
+  const int cols = p.n_heads * p.d_head;
+  if (!make_tmap_f16(&plan.tmap_q, p.q, p.batch * p.n_q, cols, p.ldq, kTcBQ) ||
+      !make_tmap_f16(&plan.tmap_kv, p.k, p.batch * p.n_kv, cols, p.ldkv, kTcBK) ||
+      !make_tmap_f16(&plan.tmap_v, p.v, p.batch * p.n_kv, cols, p.ldkv, kTcBK)) {
+    *why = "attention: cuTensorMapEncodeTiled failed";
+    return -5;
+  }
+  return 0;
+}
+
+cudaError_t attn_launch(const AttnPlan& plan, cudaStream_t s) {
+  const AttnParams& p = plan.p;
+  if (plan.tc) return p.d_head == 64 ? launch_tc<64>(plan, s) : launch_tc<128>(plan, s);
   switch (p.d_head) {
     case 64: return launch_dh<64, 64>(p, s);
     case 72: return launch_dh<72, 80>(p, s);

@@ -246,6 +246,26 @@ __device__ __forceinline__ void tmem_ld_wait16(uint32_t* r) {
                : "memory");
 }
 
+// Store 16 consecutive columns of this thread's TMEM lane (32 lanes x 32 bits).
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_wait() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// Make this thread's generic-proxy shared-memory writes visible to the async proxy
+// (tensor-core operand reads) before signalling the MMA issuer.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // Shared-memory matrix descriptor for a K-major operand tile written by TMA with
 // 128-byte swizzling: rows of 128 B, 8-row groups 1024 B apart (stride byte offset),
 // descriptor version 1, layout SWIZZLE_128B.  The leading byte offset is not used by
@@ -261,6 +281,19 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
   return d;
 }
 
+// Shared-memory descriptor for an MN-major operand (the N index contiguous) stored as
+// 128-byte swizzle atoms of 8 K-rows x 64 fp16: `lbo` = bytes between atoms along N,
+// `sbo` = bytes between 8-row groups along K.
+__device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(2) << 61;
+  return d;
+}
+
 // Instruction descriptor of tcgen05.mma kind::f16: fp32 accumulator, fp16 A and B
 // (format code 0 in both fields; A and B always share one type), both K-major, M x N.
 __host__ __device__ constexpr uint32_t umma_idesc_f16(int M, int N) {
@@ -269,6 +302,11 @@ __host__ __device__ constexpr uint32_t umma_idesc_f16(int M, int N) {
          | (0u << 10)                                // B format: f16
          | (static_cast<uint32_t>(N >> 3) << 17)     // N / 8
          | (static_cast<uint32_t>(M >> 4) << 24);    // M / 16
+}
+
+// Same with B MN-major (transpose-B bit 16): B stored with its N index contiguous.
+__host__ __device__ constexpr uint32_t umma_idesc_f16_bmn(int M, int N) {
+  return umma_idesc_f16(M, N) | (1u << 16);
 }
 
 }  // namespace sgd

@@ -436,8 +436,11 @@ EncodeTiledFn get_encode_fn() {
   return fn;
 }
 
-// fp16 [rows, cols] with row stride ld elements; box = 64 columns x box_rows rows.
-bool make_tmap(CUtensorMap* m, const void* base, int rows, int cols, int ld, int box_rows) {
+}  // namespace
+
+// fp16 [rows, cols] with row stride ld elements; box = 64 columns x box_rows rows,
+// 128-byte swizzle, out-of-range elements read as zero.
+bool make_tmap_f16(CUtensorMap* m, const void* base, int rows, int cols, int ld, int box_rows) {
   EncodeTiledFn fn = get_encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
@@ -450,8 +453,8 @@ bool make_tmap(CUtensorMap* m, const void* base, int rows, int cols, int ld, int
   return r == CUDA_SUCCESS;
 }
 
+namespace {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
-
 }  // namespace
 
 int num_sms() {
@@ -506,8 +509,8 @@ int gemm_plan(GemmPlan& p, const char** why) {
   }
   if (p.simt) return 0;
   const int b_rows = gated ? 2 * p.N : p.N;
-  if (!make_tmap(&p.tmap_a, p.A, p.M, p.K, p.lda, 128) ||
-      !make_tmap(&p.tmap_b, p.B, b_rows, p.K, p.ldb, 128)) {
+  if (!make_tmap_f16(&p.tmap_a, p.A, p.M, p.K, p.lda, 128) ||
+      !make_tmap_f16(&p.tmap_b, p.B, b_rows, p.K, p.ldb, 128)) {
     *why = "gemm: cuTensorMapEncodeTiled failed (driver entry point unavailable or bad layout)";
     return -5;
   }

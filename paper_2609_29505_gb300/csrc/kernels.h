@@ -59,6 +59,9 @@ int gemm_plan(GemmPlan& p, const char** why);
 cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s);
 int* device_status_ptr();  // device address of the shared status word
 int num_sms();
+// 2-D fp16 tensor map: [rows, cols] with row stride ld elements, box 64 x box_rows,
+// 128-byte swizzle (defined in gemm.cu).
+bool make_tmap_f16(CUtensorMap* m, const void* base, int rows, int cols, int ld, int box_rows);
 
 // Attention.
 struct AttnParams {
@@ -70,9 +73,19 @@ struct AttnParams {
   f16* o;
   int ldo;
   int batch, n_q, n_kv, n_heads, d_head;
+  int impl;  // 0: tcgen05 where d_head is 64 or 128, else mma.sync; 1: mma.sync
+};
+// A planned attention launch: parameters plus TMA descriptors for the tcgen05 kernel.
+struct AttnPlan {
+  AttnParams p{};
+  bool tc = false;
+  CUtensorMap tmap_q;
+  CUtensorMap tmap_kv;
+  CUtensorMap tmap_v;
 };
 int attn_check(const AttnParams& p, const char** why);
-cudaError_t attn_launch(const AttnParams& p, cudaStream_t s);
+int attn_plan(AttnPlan& plan, const char** why);
+cudaError_t attn_launch(const AttnPlan& plan, cudaStream_t s);
 
 // Norm: out = norm(h) [* (1 + scale) + shift].
 struct NormParams {

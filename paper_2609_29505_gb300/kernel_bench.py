@@ -75,10 +75,11 @@ def case_attention(a):
     qkv = torch.randn(B * N, 3 * d, device="cuda").half()
     o = torch.empty(B * N, d, device="cuda", dtype=torch.float16)
     q, k, v = qkv[:, :d], qkv[:, d:2 * d], qkv[:, 2 * d:]
-    ms = _time(lambda: binding.sgd_kernel_attention(q, 3 * d, k, v, 3 * d, o, d, B, N, N, H, dh),
-               a.iters, a.warmup)
+    ms = _time(lambda: binding.sgd_kernel_attention(q, 3 * d, k, v, 3 * d, o, d, B, N, N, H, dh,
+                                                    impl=a.impl), a.iters, a.warmup)
     flops = 4.0 * B * H * N * N * dh
-    return dict(case="attention", batch=B, heads=H, tokens=N, dh=dh, ms=ms, tflops=flops / ms / 1e9)
+    return dict(case="attention", impl=["tcgen05", "mma_sync"][a.impl], batch=B, heads=H,
+                tokens=N, dh=dh, ms=ms, tflops=flops / ms / 1e9)
 
 
 def case_frozen(a):
@@ -111,6 +112,7 @@ def main():
     ap.add_argument("--batch", type=int, default=4)
     ap.add_argument("--heads", type=int, default=32)
     ap.add_argument("--dh", type=int, default=128)
+    ap.add_argument("--impl", type=int, default=0, help="attention: 0 tcgen05, 1 mma.sync")
     ap.add_argument("--rows", type=int, default=4096)
     ap.add_argument("--d", type=int, default=4096)
     ap.add_argument("--caches", type=int, default=8)

@@ -115,7 +115,8 @@ def test_kernel_entry_points_validate_on_host(lib):
     epi = binding.sgd_epilogue_args(kind=binding.EPI_F16, out=64, ldo=8)
     # K not a multiple of 8
     assert lib.sgd_kernel_gemm(64, 12, 64, 12, 8, 8, 12, C.byref(epi), 0, None) == binding.SGD_ERR_SHAPE
-    assert lib.sgd_kernel_attention(64, 8, 64, 64, 8, 64, 8, 1, 4, 4, 1, 96, None) == binding.SGD_ERR_SHAPE
+    assert lib.sgd_kernel_attention(64, 8, 64, 64, 8, 64, 8, 1, 4, 4, 1, 96, 0, None) == binding.SGD_ERR_SHAPE
+    assert lib.sgd_kernel_attention(64, 8, 64, 64, 8, 64, 8, 1, 4, 4, 1, 64, 7, None) == binding.SGD_ERR_ARG
     assert lib.sgd_kernel_norm(None, None, 1, 8, 0, None, None, None, None, 0, 1, 1e-6, None) == binding.SGD_ERR_ARG
     arr = (C.c_void_p * 1)(None)
     assert lib.sgd_kernel_frozen_run(None, arr, 1, 8, None) == binding.SGD_ERR_ARG

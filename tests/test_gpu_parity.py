@@ -198,3 +198,40 @@ def test_step_order_and_state_errors(B):
     assert e.value.code == B.SGD_ERR_SCHEDULE
     m.check_device()
     m.close()
+
+
+@pytest.mark.parametrize("name", ["llada_small", "uvit_small", "sdxl_small"])
+def test_execution_modes_are_bit_identical(B, name):
+    """Jagged graphs, eager op-by-op launches (host skipping) and padded graphs (frozen
+    branches evaluated and discarded) give the same outputs bit for bit."""
+    c = case(name, 0.5)
+    results = {}
+    for mode in (B.EXEC_JAGGED_GRAPH, B.EXEC_EAGER, B.EXEC_PADDED_GRAPH):
+        m = c.model(B)
+        m.set_exec_mode(mode)
+        out = c.out_buffer()
+        res = []
+        for s in range(1, c.T + 1):
+            x = c.ids_at(s).cuda() if c.cfg.stem == "embed" else torch.from_numpy(c.ref["states"][s - 1]).cuda()
+            m.step(x, out, otj.timestep(c.T, s), s, class_ids=c.cls, ctx=c.ctx)
+            res.append(out.cpu().clone())
+        m.check_device()
+        m.close()
+        results[mode] = res
+    for mode in (B.EXEC_EAGER, B.EXEC_PADDED_GRAPH):
+        for a, b in zip(results[B.EXEC_JAGGED_GRAPH], results[mode]):
+            assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("name", ["llada_small", "sdxl_small"])
+def test_mma_sync_attention_path_within_parity(B, name):
+    """The same model with every attention on the mma.sync kernel stays within parity."""
+    c = case(name, 0.5)
+    m = B.Denoiser(c.cfg, c.w_dev, flags=B.FLAG_MMA_SYNC_ATTENTION)
+    m.set_schedule(c.T, c.sched["lifetimes"], c.sched["groups"])
+    out = c.out_buffer()
+    for s in range(1, c.T + 1):
+        x = c.ids_at(s).cuda() if c.cfg.stem == "embed" else torch.from_numpy(c.ref["states"][s - 1]).cuda()
+        m.step(x, out, otj.timestep(c.T, s), s, class_ids=c.cls, ctx=c.ctx)
+        assert rel(out.float().cpu().numpy(), c.ref["outputs"][s - 1]) <= STEP_TOL
+    m.close()
