@@ -97,6 +97,8 @@ typedef enum {
 #define SGD_FLAG_SIMT_GEMM 1
 /* Run every attention on the mma.sync kernel instead of tcgen05 (d_head 64 / 128). */
 #define SGD_FLAG_MMA_SYNC_ATTENTION 2
+/* Run the tcgen05 GEMMs as 2-CTA clusters that multicast the shared B tile. */
+#define SGD_FLAG_GEMM_CLUSTER2 4
 
 typedef struct {
   int stem, block, norm, mlp, head;   /* enums above                                   */

@@ -67,7 +67,8 @@ typedef struct {
  * (row stride ldb).  K, lda, ldb multiples of 8; N multiple of 8; pointers 16-byte
  * aligned.  use_simt = 1 runs the plain SIMT kernel (reference / debugging), 0 the
  * tcgen05 + TMA kernel (M = 128, N = 256, K = 16 instructions, fp32 accumulators in
- * TMEM).
+ * TMEM), 2 the same kernel as 2-CTA clusters in which vertically adjacent tiles share
+ * one multicast load of their B tile.
  */
 SGD_API int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
                     const sgd_epilogue_args* epi, int use_simt, void* stream);

@@ -218,6 +218,7 @@ int make_gemm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, cons
   plan->K = K;
   plan->epi = epi;
   plan->simt = (c->d.flags & SGD_FLAG_SIMT_GEMM) != 0;
+  plan->cluster = (c->d.flags & SGD_FLAG_GEMM_CLUSTER2) ? 2 : 1;
   const char* why = "";
   if (gemm_plan(*plan, &why) != 0) return fail(SGD_ERR_SHAPE, std::string(name) + ": " + why);
   const bool gated = epi.kind == SGD_EPI_GATED;
@@ -1106,7 +1107,9 @@ int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N
   p.M = M;
   p.N = N;
   p.K = K;
-  p.simt = use_simt != 0;
+  if (use_simt < 0 || use_simt > 2) return fail(SGD_ERR_ARG, "gemm: use_simt must be 0, 1 or 2");
+  p.simt = use_simt == 1;
+  p.cluster = use_simt == 2 ? 2 : 1;
   EpiParams& e = p.epi;
   e = EpiParams{};
   e.kind = ea->kind;

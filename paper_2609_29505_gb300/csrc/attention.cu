@@ -424,20 +424,38 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const __grid_con
       __syncwarp();
       if (lane == 0) mbar_arrive(&s_free[s]);
       const int kb = j * kTcBK;
-      float mt = -INFINITY;
+      // scores in log2 units; 8 independent max chains (one softmax warp per SM
+      // sub-partition: the reductions are latency-, not throughput-bound)
+      float mx[8];
 #pragma unroll
-      for (int c = 0; c < kTcBK; ++c) {
-        const float v = (kb + c < a.n_kv) ? __uint_as_float(r[c]) * a.scale_log2 : -INFINITY;
-        r[c] = __float_as_uint(v);
-        mt = fmaxf(mt, v);
+      for (int i = 0; i < 8; ++i) mx[i] = -INFINITY;
+      if (kb + kTcBK <= a.n_kv) {
+#pragma unroll
+        for (int c = 0; c < kTcBK; ++c) {
+          const float v = __uint_as_float(r[c]) * a.scale_log2;
+          r[c] = __float_as_uint(v);
+          mx[c & 7] = fmaxf(mx[c & 7], v);
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < kTcBK; ++c) {
+          const float v = (kb + c < a.n_kv) ? __uint_as_float(r[c]) * a.scale_log2 : -INFINITY;
+          r[c] = __float_as_uint(v);
+          mx[c & 7] = fmaxf(mx[c & 7], v);
+        }
       }
+      const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
       if (j == 0) {
         m2 = mt;
-      } else if (mt > m2 + kRescaleLog2) {
-        // O must hold PV_{j-1} complete before it is rescaled
+      } else if (__any_sync(0xffffffffu, mt > m2 + kRescaleLog2)) {
+        // Warp-uniform branch (the TMEM loads and stores below are .sync.aligned): every
+        // lane moves its reference to max(m2, mt), which keeps O / l exact.  O must hold
+        // PV_{j-1} complete before it is rescaled.
         if (!(ok = warp_wait_bar(&o_done[(j - 1) & 1], ((j - 1) >> 1) & 1, abort_flag, a.status, 17))) break;
         tc_fence_after();
-        const float corr = exp2f(m2 - mt);
+        const float mnew = fmaxf(m2, mt);
+        const float corr = exp2f(m2 - mnew);
         uint32_t o16[16];
 #pragma unroll
         for (int c = 0; c < DH / 16; ++c) {
@@ -450,22 +468,26 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const __grid_con
         tmem_st_wait();
         tc_fence_before();
         l *= corr;
-        m2 = mt;
+        m2 = mnew;
       }
       // P buffer s was last read by PV_{j-2}
       if (j >= 2 && !(ok = warp_wait_bar(&o_done[s], ((j - 2) >> 1) & 1, abort_flag, a.status, 18))) break;
       uint8_t* pbuf = sm + L::kP + s * L::kPBuf;
+      float ls[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ls[i] = 0.f;
 #pragma unroll
       for (int cc = 0; cc < kTcBK / 8; ++cc) {
         float p8[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
           p8[i] = exp2f(__uint_as_float(r[cc * 8 + i]) - m2);
-          l += p8[i];
+          ls[i] += p8[i];
         }
         uint8_t* dst = pbuf + (cc >> 3) * kAtom + row * 128 + ((((cc & 7) ^ (row & 7))) << 4);
         *reinterpret_cast<uint4*>(dst) = pack_f16x8(p8);
       }
+      l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(&p_full[s]);

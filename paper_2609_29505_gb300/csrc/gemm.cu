@@ -208,6 +208,11 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
   }
 }
 
+// CLUSTER = 2: the two CTAs of a cluster compute vertically adjacent 128-row tiles of
+// the same 256 output columns; each loads its own A box and one of the two B halves,
+// multicast into both CTAs, so every B byte is read from L2 once per pair.  Each CTA's
+// MMA commits the release of a stage to both CTAs (empty barriers count 2 arrivals).
+template <int CLUSTER>
 __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -224,10 +229,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
+  const uint32_t crank = CLUSTER > 1 ? cluster_ctarank() : 0;
+  const uint16_t cmask = static_cast<uint16_t>((1u << CLUSTER) - 1u);
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], CLUSTER);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull[i], 1);
@@ -246,14 +253,18 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if (CLUSTER > 1) cluster_sync();  // the peer's barriers exist before any multicast lands
   const uint32_t tmem_base = *tmem_slot;
-  const int num_tiles = a.num_m * a.num_n;
+  // work units: CLUSTER vertically adjacent tiles that share their B columns
+  const int num_mu = (a.num_m + CLUSTER - 1) / CLUSTER;
+  const int num_tiles = num_mu * a.num_n;
+  const int unit0 = blockIdx.x / CLUSTER, unit_step = gridDim.x / CLUSTER;
 
   if (warp == 0) {
     if (lane == 0) {
       int it = 0;
-      for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
-        const int m_blk = tile % a.num_m, n_blk = tile / a.num_m;
+      for (int tile = unit0; tile < num_tiles; tile += unit_step) {
+        const int m_blk = (tile % num_mu) * CLUSTER + crank, n_blk = tile / num_mu;
         const int rb0 = a.gated ? n_blk * 128 : n_blk * kBN;
         const int rb1 = a.gated ? a.N + n_blk * 128 : rb0 + 128;
         bool ok = true;
@@ -267,8 +278,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
           uint8_t* st = tiles + s * kStageBytes;
           mbar_arrive_expect_tx(&full[s], kStageBytes);
           tma_load_2d(st, &a.tmap_a, &full[s], kb * kBK, m_blk * kBM);
-          tma_load_2d(st + kTileA, &a.tmap_b, &full[s], kb * kBK, rb0);
-          tma_load_2d(st + kTileA + kTileBHalf, &a.tmap_b, &full[s], kb * kBK, rb1);
+          if (CLUSTER == 1) {
+            tma_load_2d(st + kTileA, &a.tmap_b, &full[s], kb * kBK, rb0);
+            tma_load_2d(st + kTileA + kTileBHalf, &a.tmap_b, &full[s], kb * kBK, rb1);
+          } else {
+            tma_load_2d_mc(st + kTileA + crank * kTileBHalf, &a.tmap_b, &full[s], kb * kBK,
+                           crank ? rb1 : rb0, cmask);
+          }
         }
         if (!ok) break;
       }
@@ -283,7 +299,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       const uint32_t idesc = umma_idesc_f16(kBM, kBN);
       int it = 0, lt = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++lt) {
+      for (int tile = unit0; tile < num_tiles && ok; tile += unit_step, ++lt) {
         const int acc = lt & 1;
         const uint32_t aph = (lt >> 1) & 1;
         if (!mbar_wait(&tempty[acc], aph ^ 1u, abort_flag, a.status, 2)) break;
@@ -304,7 +320,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             umma_f16(d_tmem, smem_desc_sw128(a_addr + 32 * k), smem_desc_sw128(b_addr + 32 * k),
                       idesc, (kb | k) != 0 ? 1u : 0u);
           }
-          umma_commit(&empty[s]);
+          if (CLUSTER == 1)
+            umma_commit(&empty[s]);
+          else
+            umma_commit_mc(&empty[s], cmask);
         }
         if (!ok) break;
         umma_commit(&tfull[acc]);
@@ -317,8 +336,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     const int q = warp & 3;
     int lt = 0;
     void* out = a.epi.out_slot ? *a.epi.out_slot : a.epi.out;
-    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
-      const int m_blk = tile % a.num_m, n_blk = tile / a.num_m;
+    for (int tile = unit0; tile < num_tiles; tile += unit_step, ++lt) {
+      const int m_blk = (tile % num_mu) * CLUSTER + crank, n_blk = tile / num_mu;
       const int acc = lt & 1;
       const uint32_t aph = (lt >> 1) & 1;
       if (!warp_wait(&tfull[acc], aph, abort_flag, a.status, 4)) break;
@@ -334,6 +353,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
 
   tc_fence_before();
   __syncthreads();
+  // no CTA leaves while its peer may still arrive on its barriers or write its tiles
+  if (CLUSTER > 1) cluster_sync();
   tc_fence_after();
   if (warp == 1) {
     __syncwarp();
@@ -477,6 +498,37 @@ int* device_status_ptr() {
   return ptr[dev];
 }
 
+// Clusters of two that can be resident at once (pairs must share a GPC), cached per device.
+int max_active_pairs() {
+  static int cached[64] = {0};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64) return 0;
+  if (!cached[dev]) {
+    if (cudaFuncSetAttribute(gemm_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kSmemBytes) != cudaSuccess)
+      return 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<2>, &cfg) != cudaSuccess || n < 1) {
+      cudaGetLastError();
+      n = -1;
+    }
+    cached[dev] = n;
+  }
+  return cached[dev] > 0 ? cached[dev] : 0;
+}
+
 int gemm_plan(GemmPlan& p, const char** why) {
   const EpiParams& e = p.epi;
   const bool gated = e.kind == SGD_EPI_GATED;
@@ -516,9 +568,19 @@ int gemm_plan(GemmPlan& p, const char** why) {
   }
   const int num_m = (p.M + kBM - 1) / kBM;
   const int num_n = gated ? (p.N + 127) / 128 : (p.N + kBN - 1) / kBN;
-  const int tiles = num_m * num_n;
   const int sms = num_sms();
-  p.grid = tiles < sms ? tiles : sms;
+  if (p.cluster != 1 && p.cluster != 2) p.cluster = 1;
+  if (p.cluster == 2 && num_m < 2) p.cluster = 1;  // nothing to share
+  int max_units = sms;
+  if (p.cluster == 2) {
+    max_units = max_active_pairs();
+    if (max_units < 1) {
+      p.cluster = 1;
+      max_units = sms;
+    }
+  }
+  const int units = ((num_m + p.cluster - 1) / p.cluster) * num_n;
+  p.grid = (units < max_units ? units : max_units) * p.cluster;
   return 0;
 }
 
@@ -533,8 +595,11 @@ cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s) {
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel,
+    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<1>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    if (err == cudaSuccess)
+      err = cudaFuncSetAttribute(gemm_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kSmemBytes);
     if (err != cudaSuccess) return err;
     attr_done[dev] = true;
   }
@@ -552,7 +617,22 @@ cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s) {
   a.num_n = a.gated ? (p.N + 127) / 128 : (p.N + kBN - 1) / kBN;
   a.num_k = (p.K + kBK - 1) / kBK;
   a.status = device_status_ptr();
-  gemm_tc_kernel<<<p.grid, kThreads, kSmemBytes, s>>>(a);
+  if (p.cluster == 2) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(p.grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<2>, a);
+  }
+  gemm_tc_kernel<1><<<p.grid, kThreads, kSmemBytes, s>>>(a);
   return cudaGetLastError();
 }
 

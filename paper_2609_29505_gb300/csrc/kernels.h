@@ -49,6 +49,7 @@ struct GemmPlan {
   int M = 0, N = 0, K = 0;   // N = output columns
   EpiParams epi{};
   bool simt = false;
+  int cluster = 1;           // 2: pairs of CTAs share (multicast) the B tile
   CUtensorMap tmap_a;
   CUtensorMap tmap_b;
   int grid = 0;
