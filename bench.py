@@ -38,6 +38,8 @@ def parse():
     ap.add_argument("--T", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="also time one trajectory at 100/50/33%% budgets (adds key 'budget_sweep')")
     ap.add_argument("--ablation", action="store_true",
                     help="also time the execution modes of Table tab:kernel (adds key 'ablation')")
     return ap.parse_args()
@@ -279,12 +281,13 @@ def run_native(args):
     if fz:
         kernels["frozen_run"]["frac_of_hbm"] = round(fz["bytes"] / (fz["ms"] / 1e3) / 1e9 / peaks["hbm"], 4)
 
-    # end to end through the C ABI with host buffers (pinned), copies inside the region
+    # end to end through the C ABI with host buffers (pinned): every step copies its
+    # inputs in and its whole output back; the output copy of step s overlaps step s + 1
     e2e = None
     if not args.no_e2e:
         import torch as _t
         xs_h = [x.cpu().pin_memory() for x in xs[:T]]
-        out_h = out_buffer(cfg, "cpu", pinned=True)
+        outs_h = [out_buffer(cfg, "cpu", pinned=True) for _ in range(2)]
         cls_h = None if inp.class_ids is None else inp.class_ids.cpu().pin_memory()
         ctx_h = None if inp.ctx is None else inp.ctx.cpu().pin_memory()
         model.reset()
@@ -293,13 +296,19 @@ def run_native(args):
         t0 = time.perf_counter()
         for i in range(K):
             s = i % T + 1
-            model.step_host(xs_h[s - 1], out_h, timestep(cfg, s, T), s, class_ids_host=cls_h,
-                            ctx_host=ctx_h, stream=stream)
+            model.step_host_async(xs_h[s - 1], outs_h[i % 2], timestep(cfg, s, T), s,
+                                  class_ids_host=cls_h, ctx_host=ctx_h, stream=stream)
+        model.host_wait()
         _t.cuda.synchronize()
         e2e_s = max_over_ranks(time.perf_counter() - t0, world)
         h2d = xs_h[0].numel() * xs_h[0].element_size() + (0 if cls_h is None else cls_h.numel() * 4)
         e2e = {"value": round(K * world / e2e_s, 3), "unit": "steps/s", "h2d_bytes_per_step": int(h2d),
-               "d2h_bytes_per_step": int(out_h.numel() * out_h.element_size())}
+               "d2h_bytes_per_step": int(outs_h[0].numel() * outs_h[0].element_size()),
+               "api": "sgd_step_host_async + sgd_host_wait (output copy overlaps the next step)"}
+
+    sweep = None
+    if args.sweep:
+        sweep = run_sweep(binding, model, cfg, T, weights, sched, xs, out, cls, ctx, stream, peaks)
 
     ablation = None
     if args.ablation:
@@ -327,7 +336,7 @@ def run_native(args):
                    "cache_gb": round(info["cache_bytes"] / 2 ** 30, 2), "setup": setup_t},
         "roofline": roofline, "step_roofline": step_roof, "kernels": kernels,
         "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(gpu_launches),
-        "ablation": ablation,
+        "ablation": ablation, "budget_sweep": sweep,
         "clocks": clk.summary(),
     }
     if rank == 0:
@@ -335,6 +344,44 @@ def run_native(args):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def run_sweep(binding, model, cfg, T, weights, sched, xs, out, cls, ctx, stream, peaks):
+    """One trajectory per budget (same weights and inputs): steps/s, tokens/s, and the
+    step roofline from the per-op records of one profiled trajectory."""
+    import torch
+    from paper_2609_29505_gb300 import schedule
+    from paper_2609_29505_gb300.synth import timestep
+    rows = []
+    bq = sched["branch_scores"]
+    for budget in (1.0, 0.5, 0.33):
+        sc = schedule.build_schedule(cfg, weights, T, budget=budget, branch_q=bq)
+        model.set_schedule(T, sc["lifetimes"], sc["groups"])
+        for rep in range(2):
+            model.reset()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for s in range(1, T + 1):
+                model.step(xs[s - 1], out, timestep(cfg, s, T), s, class_ids=cls, ctx=ctx, stream=stream)
+            e1.record(stream)
+            torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        model.reset()
+        fl = by = 0.0
+        for s in range(1, T + 1):
+            for r in model.profile_step(xs[s - 1], out, timestep(cfg, s, T), s, class_ids=cls,
+                                        ctx=ctx, stream=stream):
+                fl += r["flops"]
+                by += r["bytes"]
+        t_roof = max(fl / (peaks["bf16_sus"] * 1e12), by / (peaks["hbm"] * 1e9))
+        sps = T / (ms / 1e3)
+        rows.append({"budget": budget, "achieved_ratio": round(sc["ratio"], 4),
+                     "steps_per_s": round(sps, 2), "tokens_per_s": round(sps * cfg.batch * cfg.n_tokens, 1),
+                     "ms_per_step": round(ms / T, 3), "roofline_steps_per_s": round(T / t_roof, 2),
+                     "roofline_frac": round(t_roof * 1e3 / ms, 4)})
+    model.set_schedule(T, sched["lifetimes"], sched["groups"])
+    return rows
 
 
 def run_ablation(binding, model, cfg, T, weights, sched, xs, out, cls, ctx, stream):

@@ -99,6 +99,8 @@ typedef enum {
 #define SGD_FLAG_MMA_SYNC_ATTENTION 2
 /* Run the tcgen05 GEMMs as 2-CTA clusters that multicast the shared B tile. */
 #define SGD_FLAG_GEMM_CLUSTER2 4
+/* Use 64-element K-blocks (4 stages, 128-byte swizzle) in the tcgen05 GEMMs. */
+#define SGD_FLAG_GEMM_BK64 8
 
 typedef struct {
   int stem, block, norm, mlp, head;   /* enums above                                   */
@@ -208,6 +210,21 @@ SGD_API int sgd_step(sgd_ctx* ctx, const void* state_in_dev, void* out_dev, floa
  */
 SGD_API int sgd_step_host(sgd_ctx* ctx, const void* state_in_host, void* out_host, float timestep,
                   const int32_t* class_ids_host, const void* ctx_host, int step, void* stream);
+
+/*
+ * sgd_step_host_async — sgd_step_host without the final wait: the input copy and the
+ * step are queued on `stream`, the output copy on a library-owned copy stream, so the
+ * copy of step s overlaps the compute of step s + 1 (the device output is
+ * double-buffered).  in_host / out_host should be pinned; in_host must stay unchanged
+ * until the step's input copy has run and out_host must not be read (or reused for
+ * another step) until sgd_host_wait returns.
+ */
+SGD_API int sgd_step_host_async(sgd_ctx* ctx, const void* state_in_host, void* out_host,
+                                float timestep, const int32_t* class_ids_host, const void* ctx_host,
+                                int step, void* stream);
+
+/* sgd_host_wait — wait until every output copy queued by sgd_step_host_async is done. */
+SGD_API int sgd_host_wait(sgd_ctx* ctx);
 
 /* sgd_get_active_mask — mask_host[u] = 1 iff unit u is evaluated at `step` (1..T). */
 SGD_API int sgd_get_active_mask(const sgd_ctx* ctx, int step, uint8_t* mask_host, int n_units);

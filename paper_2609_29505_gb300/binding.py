@@ -38,6 +38,7 @@ HEAD = {"linear": 0, "adaln_linear": 1, "identity": 2, "logits": 3}
 FLAG_SIMT_GEMM = 1
 FLAG_MMA_SYNC_ATTENTION = 2
 FLAG_GEMM_CLUSTER2 = 4
+FLAG_GEMM_BK64 = 8
 
 EPI_F16, EPI_F32, EPI_DELTA, EPI_GATED, EPI_GELU, EPI_ROPE = range(6)
 KERNEL_NAMES = ["gemm_tc", "gemm_simt", "attention", "norm", "frozen_run", "small"]
@@ -48,7 +49,7 @@ EXPORTED = [
     "sgd_get_info", "sgd_reset", "sgd_check_device", "sgd_destroy", "sgd_last_error",
     "sgd_compile_schedule", "sgd_step_profile", "sgd_sampler_update", "sgd_kernel_gemm",
     "sgd_kernel_attention", "sgd_kernel_norm", "sgd_kernel_frozen_run", "sgd_kernel_status",
-    "sgd_set_exec_mode",
+    "sgd_set_exec_mode", "sgd_step_host_async", "sgd_host_wait",
 ]
 EXEC_JAGGED_GRAPH, EXEC_EAGER, EXEC_PADDED_GRAPH = 0, 1, 2
 
@@ -131,6 +132,8 @@ def lib() -> C.CDLL:
             "sgd_kernel_frozen_run": (i, [vp, C.POINTER(vp), i, i64, vp]),
             "sgd_kernel_status": (i, [C.POINTER(C.c_int)]),
             "sgd_set_exec_mode": (i, [vp, i]),
+            "sgd_step_host_async": (i, [vp, vp, vp, f, vp, vp, i, vp]),
+            "sgd_host_wait": (i, [vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -287,6 +290,16 @@ class Denoiser:
         return check(lib().sgd_step_host(self.handle, _ptr(state_host), _ptr(out_host),
                                          float(t), _ptr(class_ids_host), _ptr(ctx_host), step,
                                          _stream(stream)), "sgd_step_host")
+
+    def step_host_async(self, state_host, out_host, t: float, step: int, class_ids_host=None,
+                        ctx_host=None, stream=None):
+        """Queued host-buffer step; out_host is valid after host_wait()."""
+        return check(lib().sgd_step_host_async(self.handle, _ptr(state_host), _ptr(out_host),
+                                               float(t), _ptr(class_ids_host), _ptr(ctx_host),
+                                               step, _stream(stream)), "sgd_step_host_async")
+
+    def host_wait(self):
+        return check(lib().sgd_host_wait(self.handle), "sgd_host_wait")
 
     def profile_step(self, state, out, t: float, step: int, class_ids=None, ctx=None,
                      stream=None, max_records: int = 4096) -> List[dict]:

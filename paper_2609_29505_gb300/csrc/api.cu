@@ -126,6 +126,7 @@ struct sgd_ctx {
   int device = 0;
   int M = 0, U = 0, nbr = 0;
   int attn_impl = 0;  // 1: mma.sync attention everywhere (SGD_FLAG_MMA_SYNC_ATTENTION)
+  int gemm_bk = 64;   // default K-block of the tcgen05 GEMM
   int exec_mode = SGD_EXEC_JAGGED_GRAPH;
   float* h_pad = nullptr;  // padded mode: residual that discarded branch updates land in
   // buffers
@@ -163,8 +164,20 @@ struct sgd_ctx {
   void* st_out = nullptr;
   int32_t* st_cls = nullptr;
   void* st_ctx = nullptr;
+  // asynchronous host-buffer steps: double-buffered device output, copy stream, events
+  void* st_out2[2] = {nullptr, nullptr};
+  cudaStream_t copy_stream = nullptr;
+  cudaEvent_t ev_done[2] = {nullptr, nullptr};
+  cudaEvent_t ev_copied[2] = {nullptr, nullptr};
+  int async_slot = 0;
 
   ~sgd_ctx() {
+    if (copy_stream) cudaStreamSynchronize(copy_stream);
+    for (int i = 0; i < 2; ++i) {
+      if (ev_done[i]) cudaEventDestroy(ev_done[i]);
+      if (ev_copied[i]) cudaEventDestroy(ev_copied[i]);
+    }
+    if (copy_stream) cudaStreamDestroy(copy_stream);
     for (auto e : execs) cudaGraphExecDestroy(e);
     for (auto g : graphs) cudaGraphDestroy(g);
     if (cap_stream) cudaStreamDestroy(cap_stream);
@@ -219,6 +232,7 @@ int make_gemm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, cons
   plan->epi = epi;
   plan->simt = (c->d.flags & SGD_FLAG_SIMT_GEMM) != 0;
   plan->cluster = (c->d.flags & SGD_FLAG_GEMM_CLUSTER2) ? 2 : 1;
+  plan->bk = (c->d.flags & SGD_FLAG_GEMM_BK64) ? 64 : c->gemm_bk;
   const char* why = "";
   if (gemm_plan(*plan, &why) != 0) return fail(SGD_ERR_SHAPE, std::string(name) + ": " + why);
   const bool gated = epi.kind == SGD_EPI_GATED;
@@ -1042,6 +1056,52 @@ int sgd_step_host(sgd_ctx* c, const void* in_host, void* out_host, float t, cons
   return SGD_OK;
 }
 
+int sgd_step_host_async(sgd_ctx* c, const void* in_host, void* out_host, float t, const int32_t* cls_host,
+                        const void* ctx_host, int step, void* stream) {
+  if (!c) return fail(SGD_ERR_ARG, "null context");
+  if (!in_host || !out_host) return fail(SGD_ERR_ARG, "null host buffer");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int rc;
+  if (!c->copy_stream) {
+    CUDA_TRY(cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking));
+    for (int i = 0; i < 2; ++i) {
+      CUDA_TRY(cudaEventCreateWithFlags(&c->ev_done[i], cudaEventDisableTiming));
+      CUDA_TRY(cudaEventCreateWithFlags(&c->ev_copied[i], cudaEventDisableTiming));
+      if ((rc = c->alloc(reinterpret_cast<uint8_t**>(&c->st_out2[i]), c->out_bytes(), &c->ws_bytes))) return rc;
+    }
+    if (!c->st_in && (rc = c->alloc(reinterpret_cast<uint8_t**>(&c->st_in), c->in_bytes(), &c->ws_bytes))) return rc;
+  }
+  const int k = c->async_slot;
+  sgd_cond cond{};
+  if (cls_host) {
+    if (!c->st_cls && (rc = c->alloc(&c->st_cls, c->d.batch, &c->ws_bytes))) return rc;
+    CUDA_TRY(cudaMemcpyAsync(c->st_cls, cls_host, c->d.batch * 4, cudaMemcpyHostToDevice, s));
+    cond.class_ids = c->st_cls;
+  }
+  if (ctx_host && step == 1) {
+    const size_t cb = static_cast<size_t>(c->d.batch) * c->d.ctx_len * c->d.d_ctx * 2;
+    if (!c->st_ctx && (rc = c->alloc(reinterpret_cast<uint8_t**>(&c->st_ctx), cb, &c->ws_bytes))) return rc;
+    CUDA_TRY(cudaMemcpyAsync(c->st_ctx, ctx_host, cb, cudaMemcpyHostToDevice, s));
+  }
+  if (ctx_host) cond.ctx = c->st_ctx;
+  CUDA_TRY(cudaMemcpyAsync(c->st_in, in_host, c->in_bytes(), cudaMemcpyHostToDevice, s));
+  // the output buffer of slot k is free once its previous copy to the host has finished
+  CUDA_TRY(cudaStreamWaitEvent(s, c->ev_copied[k], 0));
+  if ((rc = sgd_step(c, c->st_in, c->st_out2[k], t, &cond, step, stream))) return rc;
+  CUDA_TRY(cudaEventRecord(c->ev_done[k], s));
+  CUDA_TRY(cudaStreamWaitEvent(c->copy_stream, c->ev_done[k], 0));
+  CUDA_TRY(cudaMemcpyAsync(out_host, c->st_out2[k], c->out_bytes(), cudaMemcpyDeviceToHost, c->copy_stream));
+  CUDA_TRY(cudaEventRecord(c->ev_copied[k], c->copy_stream));
+  c->async_slot ^= 1;
+  return SGD_OK;
+}
+
+int sgd_host_wait(sgd_ctx* c) {
+  if (!c) return fail(SGD_ERR_ARG, "null context");
+  if (c->copy_stream) CUDA_TRY(cudaStreamSynchronize(c->copy_stream));
+  return SGD_OK;
+}
+
 int sgd_get_active_mask(const sgd_ctx* c, int step, uint8_t* mask, int n_units) {
   if (!c || !mask) return fail(SGD_ERR_ARG, "null argument");
   if (!c->scheduled) return fail(SGD_ERR_STATE, "no schedule installed");
@@ -1107,9 +1167,10 @@ int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N
   p.M = M;
   p.N = N;
   p.K = K;
-  if (use_simt < 0 || use_simt > 2) return fail(SGD_ERR_ARG, "gemm: use_simt must be 0, 1 or 2");
+  if (use_simt < 0 || use_simt > 4) return fail(SGD_ERR_ARG, "gemm: use_simt must be in 0..4");
   p.simt = use_simt == 1;
-  p.cluster = use_simt == 2 ? 2 : 1;
+  p.cluster = (use_simt == 2 || use_simt == 4) ? 2 : 1;
+  p.bk = use_simt >= 3 ? 32 : 64;
   EpiParams& e = p.epi;
   e = EpiParams{};
   e.kind = ea->kind;

@@ -314,6 +314,18 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
   return d;
 }
 
+// Same for 64-byte rows written with 64-byte swizzling (8-row groups 512 B apart,
+// layout SWIZZLE_64B); the K slice k of a 32-element row starts 32 k bytes further.
+__device__ __forceinline__ uint64_t smem_desc_sw64(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(1) << 16;
+  d |= static_cast<uint64_t>(512 >> 4) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(4) << 61;                   // SWIZZLE_64B
+  return d;
+}
+
 // Shared-memory descriptor for an MN-major operand (the N index contiguous) stored as
 // 128-byte swizzle atoms of 8 K-rows x 64 fp16: `lbo` = bytes between atoms along N,
 // `sbo` = bytes between 8-row groups along K.

@@ -31,14 +31,27 @@ namespace {
 
 constexpr int kBM = 128;
 constexpr int kBN = 256;        // accumulator columns per tile
-constexpr int kBK = 64;         // fp16 elements per 128-byte row
-constexpr int kStages = 4;
-constexpr int kTileA = kBM * kBK * 2;          // 16 KB
-constexpr int kTileBHalf = 128 * kBK * 2;      // 16 KB
-constexpr int kStageBytes = kTileA + 2 * kTileBHalf;  // 48 KB
 constexpr int kTmemCols = 512;
 constexpr int kThreads = 192;
-constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+
+// K-block geometry.  BK = 64: 128-byte rows, 128-byte swizzle, 4 stages of 48 KB.
+// BK = 32: 64-byte rows, 64-byte swizzle, 9 stages of 24 KB — the same MMA work per
+// byte but a third more bytes in flight, to cover more of the TMA refill latency.
+template <int BK>
+struct TileCfg {
+  static constexpr int kBK = BK;
+  static constexpr int kStages = BK == 64 ? 4 : 9;
+  static constexpr int kTileA = kBM * BK * 2;
+  static constexpr int kTileBHalf = 128 * BK * 2;
+  static constexpr int kStageBytes = kTileA + 2 * kTileBHalf;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+  static_assert(kSmemBytes <= 232448, "shared memory");
+};
+
+template <int BK>
+__device__ __forceinline__ uint64_t operand_desc(uint32_t saddr) {
+  return BK == 64 ? smem_desc_sw128(saddr) : smem_desc_sw64(saddr);
+}
 
 struct TcArgs {
   CUtensorMap tmap_a;
@@ -212,8 +225,11 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
 // the same 256 output columns; each loads its own A box and one of the two B halves,
 // multicast into both CTAs, so every B byte is read from L2 once per pair.  Each CTA's
 // MMA commits the release of a stage to both CTAs (empty barriers count 2 arrivals).
-template <int CLUSTER>
+template <int CLUSTER, int BK>
 __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcArgs a) {
+  using C = TileCfg<BK>;
+  constexpr int kBK = C::kBK, kStages = C::kStages, kTileA = C::kTileA;
+  constexpr int kTileBHalf = C::kTileBHalf, kStageBytes = C::kStageBytes;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -317,7 +333,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
           const uint32_t b_addr = a_addr + kTileA;
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k) {
-            umma_f16(d_tmem, smem_desc_sw128(a_addr + 32 * k), smem_desc_sw128(b_addr + 32 * k),
+            umma_f16(d_tmem, operand_desc<BK>(a_addr + 32 * k), operand_desc<BK>(b_addr + 32 * k),
                       idesc, (kb | k) != 0 ? 1u : 0u);
           }
           if (CLUSTER == 1)
@@ -459,17 +475,19 @@ EncodeTiledFn get_encode_fn() {
 
 }  // namespace
 
-// fp16 [rows, cols] with row stride ld elements; box = 64 columns x box_rows rows,
-// 128-byte swizzle, out-of-range elements read as zero.
-bool make_tmap_f16(CUtensorMap* m, const void* base, int rows, int cols, int ld, int box_rows) {
+// fp16 [rows, cols] with row stride ld elements; box = box_cols (64 or 32) columns x
+// box_rows rows, 128- or 64-byte swizzle to match, out-of-range elements read as zero.
+bool make_tmap_f16(CUtensorMap* m, const void* base, int rows, int cols, int ld, int box_rows,
+                   int box_cols) {
   EncodeTiledFn fn = get_encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
   cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
-  cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(box_cols), static_cast<cuuint32_t>(box_rows)};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides,
-                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  box_cols == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
@@ -499,13 +517,15 @@ int* device_status_ptr() {
 }
 
 // Clusters of two that can be resident at once (pairs must share a GPC), cached per device.
+template <int BK>
 int max_active_pairs() {
+  constexpr int kSmemBytes = TileCfg<BK>::kSmemBytes;
   static int cached[64] = {0};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return 0;
   if (!cached[dev]) {
-    if (cudaFuncSetAttribute(gemm_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(gemm_tc_kernel<2, BK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              kSmemBytes) != cudaSuccess)
       return 0;
     cudaLaunchConfig_t cfg = {};
@@ -520,7 +540,7 @@ int max_active_pairs() {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<2>, &cfg) != cudaSuccess || n < 1) {
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<2, BK>, &cfg) != cudaSuccess || n < 1) {
       cudaGetLastError();
       n = -1;
     }
@@ -561,8 +581,9 @@ int gemm_plan(GemmPlan& p, const char** why) {
   }
   if (p.simt) return 0;
   const int b_rows = gated ? 2 * p.N : p.N;
-  if (!make_tmap_f16(&p.tmap_a, p.A, p.M, p.K, p.lda, 128) ||
-      !make_tmap_f16(&p.tmap_b, p.B, b_rows, p.K, p.ldb, 128)) {
+  if (p.bk != 64 && p.bk != 32) p.bk = 64;
+  if (!make_tmap_f16(&p.tmap_a, p.A, p.M, p.K, p.lda, 128, p.bk) ||
+      !make_tmap_f16(&p.tmap_b, p.B, b_rows, p.K, p.ldb, 128, p.bk)) {
     *why = "gemm: cuTensorMapEncodeTiled failed (driver entry point unavailable or bad layout)";
     return -5;
   }
@@ -573,7 +594,7 @@ int gemm_plan(GemmPlan& p, const char** why) {
   if (p.cluster == 2 && num_m < 2) p.cluster = 1;  // nothing to share
   int max_units = sms;
   if (p.cluster == 2) {
-    max_units = max_active_pairs();
+    max_units = p.bk == 32 ? max_active_pairs<32>() : max_active_pairs<64>();
     if (max_units < 1) {
       p.cluster = 1;
       max_units = sms;
@@ -584,24 +605,43 @@ int gemm_plan(GemmPlan& p, const char** why) {
   return 0;
 }
 
+template <int CLUSTER, int BK>
+cudaError_t launch_tc(const GemmPlan& p, const TcArgs& a, cudaStream_t s) {
+  constexpr int kSmemBytes = TileCfg<BK>::kSmemBytes;
+  static bool attr_done[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<CLUSTER, BK>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    if (err != cudaSuccess) return err;
+    attr_done[dev] = true;
+  }
+  if (CLUSTER == 2) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(p.grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<CLUSTER, BK>, a);
+  }
+  gemm_tc_kernel<CLUSTER, BK><<<p.grid, kThreads, kSmemBytes, s>>>(a);
+  return cudaGetLastError();
+}
+
 cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s) {
   if (p.simt) {
     SimtArgs a{p.A, p.lda, p.B, p.ldb, p.M, p.N, p.K, p.epi};
     dim3 grid((p.N + 127) / 128, p.M);
     gemm_simt_kernel<<<grid, 128, 0, s>>>(a);
     return cudaGetLastError();
-  }
-  static bool attr_done[64] = {false};
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<1>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-    if (err == cudaSuccess)
-      err = cudaFuncSetAttribute(gemm_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 kSmemBytes);
-    if (err != cudaSuccess) return err;
-    attr_done[dev] = true;
   }
   TcArgs a;
   memcpy(&a.tmap_a, &p.tmap_a, sizeof(CUtensorMap));
@@ -615,25 +655,11 @@ cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s) {
   a.gated = p.epi.kind == SGD_EPI_GATED;
   a.num_m = (p.M + kBM - 1) / kBM;
   a.num_n = a.gated ? (p.N + 127) / 128 : (p.N + kBN - 1) / kBN;
-  a.num_k = (p.K + kBK - 1) / kBK;
+  a.num_k = (p.K + p.bk - 1) / p.bk;
   a.status = device_status_ptr();
-  if (p.cluster == 2) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(p.grid);
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = kSmemBytes;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 2;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<2>, a);
-  }
-  gemm_tc_kernel<1><<<p.grid, kThreads, kSmemBytes, s>>>(a);
-  return cudaGetLastError();
+  if (p.bk == 32)
+    return p.cluster == 2 ? launch_tc<2, 32>(p, a, s) : launch_tc<1, 32>(p, a, s);
+  return p.cluster == 2 ? launch_tc<2, 64>(p, a, s) : launch_tc<1, 64>(p, a, s);
 }
 
 }  // namespace sgd

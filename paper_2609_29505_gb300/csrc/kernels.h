@@ -50,6 +50,7 @@ struct GemmPlan {
   EpiParams epi{};
   bool simt = false;
   int cluster = 1;           // 2: pairs of CTAs share (multicast) the B tile
+  int bk = 64;               // K elements per stage: 64 (128-byte swizzle) or 32 (64-byte)
   CUtensorMap tmap_a;
   CUtensorMap tmap_b;
   int grid = 0;
@@ -62,7 +63,8 @@ int* device_status_ptr();  // device address of the shared status word
 int num_sms();
 // 2-D fp16 tensor map: [rows, cols] with row stride ld elements, box 64 x box_rows,
 // 128-byte swizzle (defined in gemm.cu).
-bool make_tmap_f16(CUtensorMap* m, const void* base, int rows, int cols, int ld, int box_rows);
+bool make_tmap_f16(CUtensorMap* m, const void* base, int rows, int cols, int ld, int box_rows,
+                   int box_cols = 64);
 
 // Attention.
 struct AttnParams {

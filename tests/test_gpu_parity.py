@@ -235,3 +235,24 @@ def test_mma_sync_attention_path_within_parity(B, name):
         m.step(x, out, otj.timestep(c.T, s), s, class_ids=c.cls, ctx=c.ctx)
         assert rel(out.float().cpu().numpy(), c.ref["outputs"][s - 1]) <= STEP_TOL
     m.close()
+
+
+def test_async_host_steps_equal_device_steps(B):
+    """Queued host-buffer steps (output copy overlapping the next step) return the same
+    bytes as device steps once sgd_host_wait has returned."""
+    c = case("llada_small", 0.5)
+    m = c.model(B)
+    out_d = c.out_buffer()
+    want = []
+    for s in range(1, c.T + 1):
+        m.step(c.ids_at(s).cuda(), out_d, otj.timestep(c.T, s), s)
+        want.append(out_d.cpu().clone())
+    m.reset()
+    outs = [torch.empty(out_d.shape, dtype=out_d.dtype).pin_memory() for _ in range(c.T)]
+    ins = [c.ids_at(s).pin_memory() for s in range(1, c.T + 1)]
+    for s in range(1, c.T + 1):
+        m.step_host_async(ins[s - 1], outs[s - 1], otj.timestep(c.T, s), s)
+    m.host_wait()
+    for a, b in zip(outs, want):
+        assert torch.equal(a, b)
+    m.close()
