@@ -422,7 +422,8 @@ def run_ablation(binding, model, cfg, T, weights, sched, xs, out, cls, ctx, stre
 
 def workload_name(cfg, T, budget):
     names = {"llada": "LLaDA-8B-shaped", "dit": "DiT-XL/2-shaped", "uvit": "U-ViT-L-shaped",
-             "sdxl": "SDXL-transformer-shaped", "tiny": "tiny pre-norm"}
+             "sdxl": "SDXL-transformer-shaped", "tiny": "tiny pre-norm",
+             "llada_4k": "LLaDA-8B-shaped 4K-context"}
     return (f"{names.get(cfg.name, cfg.name)} B={cfg.batch} N={cfg.n_tokens} d={cfg.d} "
             f"L={cfg.n_blocks} T={T} budget={budget:.0%}")
 

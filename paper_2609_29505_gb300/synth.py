@@ -157,7 +157,13 @@ SMALL_CONFIGS: Dict[str, ModelConfig] = {
                                           d_out=1000, out_channels=1000, T=8, horizons=[8]),
 }
 
-ALL_CONFIGS: Dict[str, ModelConfig] = {**CONFIGS, **SMALL_CONFIGS}
+# Longer context: the LLaDA-8B-shaped model on one 4096-token sequence (the length of the
+# paper's Needle-in-a-Haystack 4K setting), same weights seed as "llada".
+EXTRA_CONFIGS: Dict[str, ModelConfig] = {
+    "llada_4k": CONFIGS["llada"].with_(name="llada_4k", batch=1, n_tokens=4096, horizons=[64]),
+}
+
+ALL_CONFIGS: Dict[str, ModelConfig] = {**CONFIGS, **SMALL_CONFIGS, **EXTRA_CONFIGS}
 
 BUDGETS = (1.0, 0.5, 0.33)
 

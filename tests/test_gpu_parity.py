@@ -256,3 +256,26 @@ def test_async_host_steps_equal_device_steps(B):
     for a, b in zip(outs, want):
         assert torch.equal(a, b)
     m.close()
+
+
+def test_long_context_4096_tokens(B):
+    """LLaDA-structured model on one 4096-token sequence (32 key tiles per query tile,
+    RoPE over 4096 positions): bit-exact active sets, per-step relative L2 <= 5e-3."""
+    cfg = synth.get_config("llada_small").with_(name="llada_small_4k", batch=1, n_tokens=4096,
+                                                T=4, horizons=[4])
+    w_cpu = synth.make_weights(cfg, "cpu")
+    inp = synth.make_inputs(cfg, "cpu")
+    W = odn.to_numpy_weights(w_cpu)
+    sched = schedule.build_schedule(cfg, w_cpu, cfg.T, budget=0.5)
+    ref = otj.run(cfg, W, sched["lifetimes"], cfg.T,
+                  ids_at=lambda s: synth.token_ids_at(cfg, inp, s).numpy())
+    m = B.Denoiser(cfg, {k: v.cuda() for k, v in w_cpu.items()})
+    m.set_schedule(cfg.T, sched["lifetimes"], sched["groups"])
+    masks = osp.active_sets(sched["lifetimes"], cfg.T)
+    out = torch.empty(1, cfg.n_tokens, cfg.d_out, dtype=torch.float16, device="cuda")
+    for s in range(1, cfg.T + 1):
+        np.testing.assert_array_equal(m.active_mask(s), masks[s - 1])
+        m.step(synth.token_ids_at(cfg, inp, s).cuda(), out, otj.timestep(cfg.T, s), s)
+        assert rel(out.float().cpu().numpy(), ref["outputs"][s - 1]) <= STEP_TOL
+    m.check_device()
+    m.close()
