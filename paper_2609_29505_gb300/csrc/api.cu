@@ -137,6 +137,7 @@ struct sgd_ctx {
   f16* act = nullptr;
   float* t_hidden = nullptr;
   float* cond_c = nullptr;
+  float* cond_silu = nullptr;
   float* mod = nullptr;
   float* modf = nullptr;
   float* rope_cos = nullptr;
@@ -454,6 +455,7 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
     g2.rows = d.batch;
     g2.add_class = B16(c->w.class_emb);
     g2.n_classes = d.n_classes;
+    g2.out_silu = c->cond_silu;
     make_gemv_op(ops, "cond.t2", g2);
     for (int b = 0; b < d.n_blocks; ++b) {
       bool any = false;
@@ -462,10 +464,10 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
       GemvParams gm{};
       gm.out = c->mod + static_cast<size_t>(b) * d.batch * 6 * D;
       gm.ldo = 6 * D;
-      gm.x = c->cond_c;
+      gm.x = c->cond_silu;
       gm.ldx = D;
       gm.slot = c->slot;
-      gm.in_silu = 1;
+      gm.in_silu = 0;
       gm.W = B16(c->blk[b].w_mod);
       gm.N = 6 * D;
       gm.K = D;
@@ -546,10 +548,10 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
     GemvParams g{};
     g.out = c->modf;
     g.ldo = 2 * D;
-    g.x = c->cond_c;
+    g.x = c->cond_silu;
     g.ldx = D;
     g.slot = c->slot;
-    g.in_silu = 1;
+    g.in_silu = 0;
     g.W = B16(c->w.w_modf);
     g.N = 2 * D;
     g.K = D;
@@ -685,6 +687,7 @@ int ensure_alloc(sgd_ctx* c) {
   if (d.block == SGD_BLOCK_ADALN) {
     if ((rc = c->alloc(&c->t_hidden, D, &c->ws_bytes))) return rc;
     if ((rc = c->alloc(&c->cond_c, d.batch * D, &c->ws_bytes))) return rc;
+    if ((rc = c->alloc(&c->cond_silu, d.batch * D, &c->ws_bytes))) return rc;
     if ((rc = c->alloc(&c->mod, static_cast<size_t>(d.n_blocks) * d.batch * 6 * D, &c->ws_bytes))) return rc;
     if ((rc = c->alloc(&c->modf, d.batch * 2 * D, &c->ws_bytes))) return rc;
   }
@@ -1167,10 +1170,13 @@ int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N
   p.M = M;
   p.N = N;
   p.K = K;
-  if (use_simt < 0 || use_simt > 4) return fail(SGD_ERR_ARG, "gemm: use_simt must be in 0..4");
+  if (use_simt < 0 || use_simt > 7) return fail(SGD_ERR_ARG, "gemm: variant must be in 0..7");
   p.simt = use_simt == 1;
   p.cluster = (use_simt == 2 || use_simt == 4) ? 2 : 1;
-  p.bk = use_simt >= 3 ? 32 : 64;
+  p.bk = (use_simt == 3 || use_simt == 4) ? 32 : 64;
+  if (use_simt == 5) { p.bn = 256; p.epiw = 4; }
+  if (use_simt == 6) { p.bn = 256; p.epiw = 8; }
+  if (use_simt == 7) { p.bn = 128; p.epiw = 8; }
   EpiParams& e = p.epi;
   e = EpiParams{};
   e.kind = ea->kind;

@@ -111,6 +111,73 @@ __global__ void __launch_bounds__(kNormThreads) norm_kernel(const NormParams p) 
   }
 }
 
+// Same normalisation with one warp per row (d <= 2048: at most 16 float4 per lane), eight
+// rows per block: for the 1-2 k-wide rows of the mid-size models a 128-thread block per row
+// leaves each thread two vectors of work.
+constexpr int kNormWarpMaxVec = 16;
+__global__ void __launch_bounds__(256) norm_warp_kernel(const NormParams p) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row = blockIdx.x * 8 + warp;
+  if (row >= p.rows) return;
+  const int nv = p.d >> 2;
+  const float4* hr = reinterpret_cast<const float4*>(p.h + static_cast<int64_t>(row) * p.d);
+  float4 v[kNormWarpMaxVec];
+  float sum = 0.f, sq = 0.f;
+#pragma unroll
+  for (int j = 0; j < kNormWarpMaxVec; ++j) {
+    const int i = lane + 32 * j;
+    if (i < nv) {
+      v[j] = hr[i];
+      sum += (v[j].x + v[j].y) + (v[j].z + v[j].w);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+  const float mean = p.kind == SGD_NORM_RMS ? 0.f : sum / p.d;
+#pragma unroll
+  for (int j = 0; j < kNormWarpMaxVec; ++j) {
+    const int i = lane + 32 * j;
+    if (i < nv) {
+      const float a = v[j].x - mean, b = v[j].y - mean, c = v[j].z - mean, d = v[j].w - mean;
+      sq += (a * a + b * b) + (c * c + d * d);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+  const float rstd = rsqrtf(sq / p.d + p.eps);
+  const float* sh = p.shift ? p.shift + static_cast<int64_t>(row / p.rows_per_batch) * p.ld_mod : nullptr;
+  const float* sc = p.scale ? p.scale + static_cast<int64_t>(row / p.rows_per_batch) * p.ld_mod : nullptr;
+  f16* orow = p.out + static_cast<int64_t>(row) * p.d;
+#pragma unroll
+  for (int j = 0; j < kNormWarpMaxVec; ++j) {
+    const int i = lane + 32 * j;
+    if (i < nv) {
+      float y[4] = {(v[j].x - mean) * rstd, (v[j].y - mean) * rstd, (v[j].z - mean) * rstd,
+                    (v[j].w - mean) * rstd};
+      if (p.g) {
+        float g[4];
+        load_bf16x4(p.g + 4 * i, g);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) y[k] *= g[k];
+      }
+      if (p.b) {
+        float b[4];
+        load_bf16x4(p.b + 4 * i, b);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) y[k] += b[k];
+      }
+      if (sc) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) y[k] = y[k] * (1.f + sc[4 * i + k]) + sh[4 * i + k];
+      }
+      uint2 u;
+      u.x = pack_f16x2(y[0], y[1]);
+      u.y = pack_f16x2(y[2], y[3]);
+      *reinterpret_cast<uint2*>(orow + 4 * i) = u;
+    }
+  }
+}
+
 __global__ void __launch_bounds__(256) frozen_kernel(const __grid_constant__ FrozenParams p) {
   const int64_t n8 = p.n >> 3;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -187,10 +254,14 @@ __global__ void stem_kernel(const StemParams p) {
   p.h[idx] = v;
 }
 
-// One warp per output column j; all rows (<= 16) share the weight row read.
-constexpr int kGemvMaxRows = 16;
+// out[r, j] = sum_k act(x[r, k]) W[j, k] for R <= RMAX rows (conditioning and AdaLN
+// modulation: a few rows against a large weight, bound by reading W once).  Each warp owns
+// 4 consecutive columns; a lane streams 16-byte chunks of the 4 weight rows and reuses
+// every x chunk (read once from shared memory per row) across the 4 columns.
+constexpr int kGemvCols = 4;
+template <int RMAX>
 __global__ void __launch_bounds__(256) gemv_kernel(const GemvParams p) {
-  extern __shared__ float xs[];  // [rows][K]
+  extern __shared__ float xs[];  // [xrows][K]
   const int xrows = p.x_sinusoid ? 1 : (p.ldx == 0 ? 1 : p.rows);
   for (int i = threadIdx.x; i < xrows * p.K; i += blockDim.x) {
     const int r = i / p.K, k = i % p.K;
@@ -200,40 +271,67 @@ __global__ void __launch_bounds__(256) gemv_kernel(const GemvParams p) {
   }
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int j = blockIdx.x * (blockDim.x >> 5) + warp;
-  if (j >= p.N) return;
-  float acc[kGemvMaxRows];
+  const int j0 = (blockIdx.x * (blockDim.x >> 5) + warp) * kGemvCols;
+  if (j0 >= p.N) return;
+  float acc[kGemvCols][RMAX];
 #pragma unroll
-  for (int r = 0; r < kGemvMaxRows; ++r) acc[r] = 0.f;
-  const bf16* w = p.W + static_cast<int64_t>(j) * p.K;
+  for (int c = 0; c < kGemvCols; ++c)
+#pragma unroll
+    for (int r = 0; r < RMAX; ++r) acc[c][r] = 0.f;
   for (int k = lane * 8; k < p.K; k += 256) {
-    float f[8];
-    unpack_bf16x8(*reinterpret_cast<const uint4*>(w + k), f);
+    float w[kGemvCols][8];
 #pragma unroll
-    for (int r = 0; r < kGemvMaxRows; ++r) {
+    for (int c = 0; c < kGemvCols; ++c) {
+      if (j0 + c < p.N)
+        unpack_bf16x8(*reinterpret_cast<const uint4*>(p.W + static_cast<int64_t>(j0 + c) * p.K + k), w[c]);
+      else
+#pragma unroll
+        for (int q = 0; q < 8; ++q) w[c][q] = 0.f;
+    }
+#pragma unroll
+    for (int r = 0; r < RMAX; ++r) {
       if (r < xrows) {
-        const float* x = xs + r * p.K + k;
+        const float4 xa = *reinterpret_cast<const float4*>(xs + r * p.K + k);
+        const float4 xb = *reinterpret_cast<const float4*>(xs + r * p.K + k + 4);
+        const float xv[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
 #pragma unroll
-        for (int q = 0; q < 8; ++q) acc[r] = fmaf(f[q], x[q], acc[r]);
+        for (int c = 0; c < kGemvCols; ++c)
+#pragma unroll
+          for (int q = 0; q < 8; ++q) acc[c][r] = fmaf(w[c][q], xv[q], acc[c][r]);
       }
     }
   }
 #pragma unroll
-  for (int r = 0; r < kGemvMaxRows; ++r) {
-    if (r < xrows) {
+  for (int c = 0; c < kGemvCols; ++c)
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) acc[r] += __shfl_xor_sync(0xffffffffu, acc[r], o);
+    for (int r = 0; r < RMAX; ++r) {
+      if (r < xrows) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) acc[c][r] += __shfl_xor_sync(0xffffffffu, acc[c][r], o);
+      }
     }
-  }
-  if (lane == 0) {
+  if (lane < kGemvCols && j0 + lane < p.N) {
+    const int j = j0 + lane;
+    // lane c stores column j0 + c; select chains keep acc in registers
+    float vals[RMAX];
+#pragma unroll
+    for (int rr = 0; rr < RMAX; ++rr) {
+      float v = acc[0][rr];
+#pragma unroll
+      for (int c = 1; c < kGemvCols; ++c) v = (lane == c) ? acc[c][rr] : v;
+      vals[rr] = v;
+    }
     for (int r = 0; r < p.rows; ++r) {
-      float v = acc[xrows == 1 ? 0 : r];
+      float v = vals[0];
+#pragma unroll
+      for (int rr = 1; rr < RMAX; ++rr) v = (xrows > 1 && rr == r) ? vals[rr] : v;
       if (p.add_class) {
         const int cls = min(max(p.slot->class_ids[r], 0), p.n_classes - 1);
         v += __bfloat162float(p.add_class[static_cast<int64_t>(cls) * p.N + j]);
       }
       if (p.add_vec) v += p.add_vec[j];
       p.out[static_cast<int64_t>(r) * p.ldo + j] = v;
+      if (p.out_silu) p.out_silu[static_cast<int64_t>(r) * p.ldo + j] = silu_f(v);
     }
   }
 }
@@ -331,7 +429,10 @@ int grid_for(int64_t work, int threads) {
 }  // namespace
 
 cudaError_t norm_launch(const NormParams& p, cudaStream_t s) {
-  norm_kernel<<<p.rows, kNormThreads, 0, s>>>(p);
+  if (p.d <= 32 * 4 * kNormWarpMaxVec)
+    norm_warp_kernel<<<(p.rows + 7) / 8, 256, 0, s>>>(p);
+  else
+    norm_kernel<<<p.rows, kNormThreads, 0, s>>>(p);
   return cudaGetLastError();
 }
 
@@ -351,17 +452,25 @@ cudaError_t stem_launch(const StemParams& p, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t gemv_launch(const GemvParams& p, cudaStream_t s) {
-  const int xrows = p.x_sinusoid ? 1 : (p.ldx == 0 ? 1 : p.rows);
-  const size_t smem = static_cast<size_t>(xrows) * p.K * sizeof(float);
-  if (p.rows > kGemvMaxRows || smem > 200 * 1024) return cudaErrorInvalidValue;
+template <int RMAX>
+cudaError_t gemv_launch_r(const GemvParams& p, size_t smem, cudaStream_t s) {
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(gemv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(gemv_kernel<RMAX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
   }
-  gemv_kernel<<<(p.N + 7) / 8, 256, smem, s>>>(p);
+  const int cols_per_block = 8 * kGemvCols;
+  gemv_kernel<RMAX><<<(p.N + cols_per_block - 1) / cols_per_block, 256, smem, s>>>(p);
   return cudaGetLastError();
+}
+
+cudaError_t gemv_launch(const GemvParams& p, cudaStream_t s) {
+  const int xrows = p.x_sinusoid ? 1 : (p.ldx == 0 ? 1 : p.rows);
+  const size_t smem = static_cast<size_t>(xrows) * p.K * sizeof(float);
+  if (p.rows > 16 || smem > 200 * 1024 || (p.K % 8)) return cudaErrorInvalidValue;
+  if (xrows == 1) return gemv_launch_r<1>(p, smem, s);
+  if (xrows <= 8) return gemv_launch_r<8>(p, smem, s);
+  return gemv_launch_r<16>(p, smem, s);
 }
 
 cudaError_t head_small_launch(const HeadParams& p, cudaStream_t s) {

@@ -13,9 +13,10 @@
 //   warp 1      allocates 512 TMEM columns (two 128x256 fp32 accumulators) and one
 //               elected lane issues tcgen05.mma (M=128, N=256, K=16) four times per
 //               stage, committing each stage back to the producer.
-//   warps 2-5   epilogue: tcgen05.ld rows out of TMEM (warp w owns TMEM lanes
-//               32 (w % 4) ...), apply the epilogue, store to global memory.  The two
-//               accumulators let the epilogue of tile i overlap the MMAs of tile i+1.
+//   warps 2-9   epilogue: tcgen05.ld rows out of TMEM (warp w owns TMEM lanes
+//               32 (w % 4) ..., warps w and w + 4 split the tile's columns), apply the
+//               epilogue, store to global memory.  The two accumulators let the epilogue
+//               of tile i overlap the MMAs of tile i+1.
 // Every wait is bounded (common.cuh); on expiry the CTA drains its own copies and
 // MMAs, frees TMEM and exits with the device status word set.
 #include <cstdio>
@@ -30,22 +31,27 @@ namespace sgd {
 namespace {
 
 constexpr int kBM = 128;
-constexpr int kBN = 256;        // accumulator columns per tile
-constexpr int kTmemCols = 512;
-constexpr int kThreads = 192;
 
 // K-block geometry.  BK = 64: 128-byte rows, 128-byte swizzle, 4 stages of 48 KB.
 // BK = 32: 64-byte rows, 64-byte swizzle, 9 stages of 24 KB — the same MMA work per
 // byte but a third more bytes in flight, to cover more of the TMA refill latency.
-template <int BK>
+// BN = 256 or 128 accumulator columns per tile (two accumulators in TMEM); EPIW = 4 or 8
+// epilogue warps (8: warps w and w + 4 split the tile's columns).
+template <int BK, int BN = 256, int EPIW = 8>
 struct TileCfg {
   static constexpr int kBK = BK;
-  static constexpr int kStages = BK == 64 ? 4 : 9;
+  static constexpr int kBN = BN;
+  static constexpr int kEpiWarps = EPIW;
+  static constexpr int kThreads = 64 + 32 * EPIW;
+  static constexpr int kTmemCols = 2 * BN;
   static constexpr int kTileA = kBM * BK * 2;
   static constexpr int kTileBHalf = 128 * BK * 2;
-  static constexpr int kStageBytes = kTileA + 2 * kTileBHalf;
+  static constexpr int kTileB = BN * BK * 2;
+  static constexpr int kStageBytes = kTileA + kTileB;
+  static constexpr int kStages = (192 * 1024) / kStageBytes;
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
   static_assert(kSmemBytes <= 232448, "shared memory");
+  static_assert(2 * kStages + 5 <= 30, "barrier block");
 };
 
 template <int BK>
@@ -122,20 +128,23 @@ __device__ __forceinline__ void u32_to_f32x16(const uint32_t* r, float* f, float
   for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(r[i]) * alpha;
 }
 
-// Epilogue of one 128 x 256 accumulator, executed by all 128 epilogue threads; this
-// thread owns tile row `row` (TMEM lane row - m0) and reads from `tbase`.
+// Epilogue of one 128 x BN accumulator: this thread owns tile row `row` (TMEM lane
+// row - m0), reads from `tbase` and handles accumulator columns [cb, ce) (gated:
+// output columns [cb, ce) of the BN / 2 the tile produces).
+template <int BN>
 __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int row, int n_blk,
-                                              uint32_t tbase) {
+                                              uint32_t tbase, int cb, int ce) {
+  constexpr int kBN = BN;
   const EpiParams& e = a.epi;
   const bool row_ok = row < a.M;
   uint32_t r0[16], r1[16];
   float x[16], y[16];
   if (a.gated) {
-    const int n0 = n_blk * 128;
-    for (int c = 0; c < 128; c += 16) {
+    const int n0 = n_blk * (kBN / 2);
+    for (int c = cb; c < ce; c += 16) {
       if (n0 + c >= a.N) break;
       tmem_ld16(tbase + c, r0);
-      tmem_ld16(tbase + 128 + c, r1);
+      tmem_ld16(tbase + kBN / 2 + c, r1);
       tmem_ld_wait16(r0);
       tmem_ld_wait16(r1);
       u32_to_f32x16(r0, x, e.alpha);
@@ -151,21 +160,21 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
   }
   const int n0 = n_blk * kBN;
   if (e.kind == SGD_EPI_ROPE) {
-    const int dh = e.d_head, half = dh >> 1;
+    const int dh = e.d_head, hd = dh >> 1;
     const int pos = row_ok ? row % e.rope_tokens : 0;
-    for (int hb = 0; hb < kBN; hb += dh) {
+    for (int hb = cb; hb < ce; hb += dh) {
       if (n0 + hb >= a.N) break;
       const bool rot = (n0 + hb) < e.rope_cols;
-      for (int j = 0; j < half; j += 16) {
+      for (int j = 0; j < hd; j += 16) {
         tmem_ld16(tbase + hb + j, r0);
-        tmem_ld16(tbase + hb + half + j, r1);
+        tmem_ld16(tbase + hb + hd + j, r1);
         tmem_ld_wait16(r0);
         tmem_ld_wait16(r1);
         u32_to_f32x16(r0, x, e.alpha);
         u32_to_f32x16(r1, y, e.alpha);
         if (rot && row_ok) {
-          const float* cs = e.rope_cos + static_cast<int64_t>(pos) * half + j;
-          const float* sn = e.rope_sin + static_cast<int64_t>(pos) * half + j;
+          const float* cs = e.rope_cos + static_cast<int64_t>(pos) * hd + j;
+          const float* sn = e.rope_sin + static_cast<int64_t>(pos) * hd + j;
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
             const float c_ = cs[i], s_ = sn[i];
@@ -175,7 +184,7 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
           }
         }
         if (row_ok) {
-          const int c1 = n0 + hb + j, c2 = c1 + half;
+          const int c1 = n0 + hb + j, c2 = c1 + hd;
           epi_store8(e, out, row, c1, x);
           epi_store8(e, out, row, c1 + 8, x + 8);
           epi_store8(e, out, row, c2, y);
@@ -185,7 +194,7 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
     }
     return;
   }
-  for (int c = 0; c < kBN; c += 32) {
+  for (int c = cb; c < ce; c += 32) {
     if (n0 + c >= a.N) break;
     tmem_ld16(tbase + c, r0);
     tmem_ld16(tbase + c + 16, r1);
@@ -225,11 +234,14 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
 // the same 256 output columns; each loads its own A box and one of the two B halves,
 // multicast into both CTAs, so every B byte is read from L2 once per pair.  Each CTA's
 // MMA commits the release of a stage to both CTAs (empty barriers count 2 arrivals).
-template <int CLUSTER, int BK>
-__global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcArgs a) {
-  using C = TileCfg<BK>;
+template <int CLUSTER, int BK, int BN, int EPIW>
+__global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
+    gemm_tc_kernel(const __grid_constant__ TcArgs a) {
+  using C = TileCfg<BK, BN, EPIW>;
   constexpr int kBK = C::kBK, kStages = C::kStages, kTileA = C::kTileA;
   constexpr int kTileBHalf = C::kTileBHalf, kStageBytes = C::kStageBytes;
+  constexpr int kBN = C::kBN, kTmemCols = C::kTmemCols, kEpiWarps = C::kEpiWarps;
+  static_assert(CLUSTER == 1 || BN == 256, "multicast splits a 256-row B tile");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -254,7 +266,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], 4);
+      mbar_init(&tempty[i], kEpiWarps);
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -282,7 +294,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       for (int tile = unit0; tile < num_tiles; tile += unit_step) {
         const int m_blk = (tile % num_mu) * CLUSTER + crank, n_blk = tile / num_mu;
         const int rb0 = a.gated ? n_blk * 128 : n_blk * kBN;
-        const int rb1 = a.gated ? a.N + n_blk * 128 : rb0 + 128;
+        const int rb1 = a.gated ? a.N + n_blk * 128 : rb0 + 128;  // BN = 256 only
         bool ok = true;
         for (int kb = 0; kb < a.num_k; ++kb, ++it) {
           const int s = it % kStages;
@@ -296,7 +308,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
           tma_load_2d(st, &a.tmap_a, &full[s], kb * kBK, m_blk * kBM);
           if (CLUSTER == 1) {
             tma_load_2d(st + kTileA, &a.tmap_b, &full[s], kb * kBK, rb0);
-            tma_load_2d(st + kTileA + kTileBHalf, &a.tmap_b, &full[s], kb * kBK, rb1);
+            if (kBN == 256) tma_load_2d(st + kTileA + kTileBHalf, &a.tmap_b, &full[s], kb * kBK, rb1);
           } else {
             tma_load_2d_mc(st + kTileA + crank * kTileBHalf, &a.tmap_b, &full[s], kb * kBK,
                            crank ? rb1 : rb0, cmask);
@@ -350,6 +362,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     }
   } else {
     const int q = warp & 3;
+    // column range of this warp: all of the tile (4 epilogue warps) or one half (8)
+    const int span = a.gated ? kBN / 2 : kBN;
+    const int part = kEpiWarps == 8 ? ((warp - 2) >> 2) : 0;
+    const int cb = kEpiWarps == 8 ? part * (span / 2) : 0;
+    const int ce = kEpiWarps == 8 ? cb + span / 2 : span;
     int lt = 0;
     void* out = a.epi.out_slot ? *a.epi.out_slot : a.epi.out;
     for (int tile = unit0; tile < num_tiles; tile += unit_step, ++lt) {
@@ -360,7 +377,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       tc_fence_after();
       const int row = m_blk * kBM + q * 32 + lane;
       const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * kBN;
-      epilogue_tile(a, out, row, n_blk, tbase);
+      epilogue_tile<kBN>(a, out, row, n_blk, tbase, cb, ce);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -520,12 +537,13 @@ int* device_status_ptr() {
 template <int BK>
 int max_active_pairs() {
   constexpr int kSmemBytes = TileCfg<BK>::kSmemBytes;
+  constexpr int kThreads = TileCfg<BK>::kThreads;
   static int cached[64] = {0};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) return 0;
   if (!cached[dev]) {
-    if (cudaFuncSetAttribute(gemm_tc_kernel<2, BK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(gemm_tc_kernel<2, BK, 256, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              kSmemBytes) != cudaSuccess)
       return 0;
     cudaLaunchConfig_t cfg = {};
@@ -540,7 +558,7 @@ int max_active_pairs() {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<2, BK>, &cfg) != cudaSuccess || n < 1) {
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<2, BK, 256, 8>, &cfg) != cudaSuccess || n < 1) {
       cudaGetLastError();
       n = -1;
     }
@@ -588,8 +606,21 @@ int gemm_plan(GemmPlan& p, const char** why) {
     return -5;
   }
   const int num_m = (p.M + kBM - 1) / kBM;
-  const int num_n = gated ? (p.N + 127) / 128 : (p.N + kBN - 1) / kBN;
   const int sms = num_sms();
+  // tile shape: 128-column tiles when they need clearly fewer tile-times than 256-column
+  // tiles (a 128-column tile takes half the time of a 256-column one, at about 3/4 of its
+  // efficiency, so: 2 * waves_128 < 3 * waves_256); they need a plain epilogue and
+  // one-CTA launches.  4 epilogue warps for RoPE and gated epilogues.
+  const bool small_ok = !gated && e.kind != SGD_EPI_ROPE && p.bk == 64 && p.cluster == 1;
+  if (p.bn == 0) {
+    const int w256 = (num_m * ((p.N + 255) / 256) + sms - 1) / sms;
+    const int w128 = (num_m * ((p.N + 127) / 128) + sms - 1) / sms;
+    p.bn = (small_ok && 2 * w128 < 3 * w256) ? 128 : 256;
+  }
+  if (p.bn != 128 || !small_ok) p.bn = 256;
+  if (p.epiw == 0) p.epiw = (e.kind == SGD_EPI_ROPE || gated) ? 4 : 8;
+  if (p.bn == 128 || p.cluster == 2 || p.bk == 32) p.epiw = 8;
+  const int num_n = gated ? (p.N + 127) / 128 : (p.N + p.bn - 1) / p.bn;
   if (p.cluster != 1 && p.cluster != 2) p.cluster = 1;
   if (p.cluster == 2 && num_m < 2) p.cluster = 1;  // nothing to share
   int max_units = sms;
@@ -605,14 +636,15 @@ int gemm_plan(GemmPlan& p, const char** why) {
   return 0;
 }
 
-template <int CLUSTER, int BK>
+template <int CLUSTER, int BK, int BN, int EPIW>
 cudaError_t launch_tc(const GemmPlan& p, const TcArgs& a, cudaStream_t s) {
-  constexpr int kSmemBytes = TileCfg<BK>::kSmemBytes;
+  constexpr int kSmemBytes = TileCfg<BK, BN, EPIW>::kSmemBytes;
+  constexpr int kThreads = TileCfg<BK, BN, EPIW>::kThreads;
   static bool attr_done[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<CLUSTER, BK>,
+    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<CLUSTER, BK, BN, EPIW>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (err != cudaSuccess) return err;
     attr_done[dev] = true;
@@ -630,9 +662,9 @@ cudaError_t launch_tc(const GemmPlan& p, const TcArgs& a, cudaStream_t s) {
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<CLUSTER, BK>, a);
+    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<CLUSTER, BK, BN, EPIW>, a);
   }
-  gemm_tc_kernel<CLUSTER, BK><<<p.grid, kThreads, kSmemBytes, s>>>(a);
+  gemm_tc_kernel<CLUSTER, BK, BN, EPIW><<<p.grid, kThreads, kSmemBytes, s>>>(a);
   return cudaGetLastError();
 }
 
@@ -654,12 +686,14 @@ cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s) {
   a.K = p.K;
   a.gated = p.epi.kind == SGD_EPI_GATED;
   a.num_m = (p.M + kBM - 1) / kBM;
-  a.num_n = a.gated ? (p.N + 127) / 128 : (p.N + kBN - 1) / kBN;
+  a.num_n = a.gated ? (p.N + 127) / 128 : (p.N + p.bn - 1) / p.bn;
   a.num_k = (p.K + p.bk - 1) / p.bk;
   a.status = device_status_ptr();
   if (p.bk == 32)
-    return p.cluster == 2 ? launch_tc<2, 32>(p, a, s) : launch_tc<1, 32>(p, a, s);
-  return p.cluster == 2 ? launch_tc<2, 64>(p, a, s) : launch_tc<1, 64>(p, a, s);
+    return p.cluster == 2 ? launch_tc<2, 32, 256, 8>(p, a, s) : launch_tc<1, 32, 256, 8>(p, a, s);
+  if (p.cluster == 2) return launch_tc<2, 64, 256, 8>(p, a, s);
+  if (p.bn == 128) return launch_tc<1, 64, 128, 8>(p, a, s);
+  return p.epiw == 4 ? launch_tc<1, 64, 256, 4>(p, a, s) : launch_tc<1, 64, 256, 8>(p, a, s);
 }
 
 }  // namespace sgd

@@ -51,6 +51,8 @@ struct GemmPlan {
   bool simt = false;
   int cluster = 1;           // 2: pairs of CTAs share (multicast) the B tile
   int bk = 64;               // K elements per stage: 64 (128-byte swizzle) or 32 (64-byte)
+  int bn = 0;                // output columns per tile: 256, 128, or 0 = choose by tile count
+  int epiw = 0;              // epilogue warps: 4, 8, or 0 = choose by epilogue kind
   CUtensorMap tmap_a;
   CUtensorMap tmap_b;
   int grid = 0;
@@ -153,6 +155,7 @@ struct GemvParams {
   const bf16* add_class;  // optional: + class_emb[class_ids[r]] (bf16 [n_classes, N])
   int n_classes;          // class ids are clamped into [0, n_classes)
   const float* add_vec;   // optional: + add_vec[j] (broadcast over rows)
+  float* out_silu;        // optional: silu(out) written alongside (same layout)
 };
 cudaError_t gemv_launch(const GemvParams& p, cudaStream_t s);
 

@@ -49,7 +49,7 @@ def _check_f16(got, want, extra_abs=0.0):
 GEMM_SHAPES = [(64, 256, 256), (300, 520, 688), (129, 264, 72), (1000, 1376, 512), (4128, 1024, 2048)]
 
 
-@pytest.mark.parametrize("simt", [0, 2, 3, 4, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "simt"])
+@pytest.mark.parametrize("simt", [0, 2, 3, 4, 5, 6, 7, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "tcgen05_epi4", "tcgen05_epi8", "tcgen05_bn128", "simt"])
 @pytest.mark.parametrize("M,N,K", GEMM_SHAPES)
 def test_gemm_bf16(B, M, N, K, simt):
     rng = np.random.default_rng(M + N + K)
@@ -63,7 +63,7 @@ def test_gemm_bf16(B, M, N, K, simt):
     _check_f16(out, odn.linear(_f(A), _f(W)))
 
 
-@pytest.mark.parametrize("simt", [0, 2, 3, 4, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "simt"])
+@pytest.mark.parametrize("simt", [0, 2, 3, 4, 5, 6, 7, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "tcgen05_epi4", "tcgen05_epi8", "tcgen05_bn128", "simt"])
 @pytest.mark.parametrize("gated", [False, True])
 def test_gemm_delta_residual_and_cache(B, simt, gated):
     rng = np.random.default_rng(5)
@@ -87,7 +87,7 @@ def test_gemm_delta_residual_and_cache(B, simt, gated):
     _check_f16(cache, delta)
 
 
-@pytest.mark.parametrize("simt", [0, 2, 3, 4, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "simt"])
+@pytest.mark.parametrize("simt", [0, 2, 3, 4, 5, 6, 7, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "tcgen05_epi4", "tcgen05_epi8", "tcgen05_bn128", "simt"])
 @pytest.mark.parametrize("act", [0, 1])
 def test_gemm_gated_activation(B, simt, act):
     rng = np.random.default_rng(6)
@@ -103,7 +103,7 @@ def test_gemm_gated_activation(B, simt, act):
     _check_f16(out, want, extra_abs=1e-4 * float(np.abs(want).max()))
 
 
-@pytest.mark.parametrize("simt", [0, 2, 3, 4, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "simt"])
+@pytest.mark.parametrize("simt", [0, 2, 3, 4, 5, 6, 7, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "tcgen05_epi4", "tcgen05_epi8", "tcgen05_bn128", "simt"])
 @pytest.mark.parametrize("act", [0, 1])
 def test_gemm_gelu(B, simt, act):
     rng = np.random.default_rng(7)
@@ -119,7 +119,7 @@ def test_gemm_gelu(B, simt, act):
     _check_f16(out, want, extra_abs=1e-4 * float(np.abs(want).max()))
 
 
-@pytest.mark.parametrize("simt", [0, 2, 3, 4, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "simt"])
+@pytest.mark.parametrize("simt", [0, 2, 3, 4, 5, 6, 7, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "tcgen05_epi4", "tcgen05_epi8", "tcgen05_bn128", "simt"])
 @pytest.mark.parametrize("dh", [64, 128])
 def test_gemm_rope_epilogue(B, simt, dh):
     rng = np.random.default_rng(8)
@@ -170,7 +170,8 @@ def test_attention(B, dh, H, nq, nkv, bsz, impl):
     assert B.sgd_kernel_status() == 0
 
 
-@pytest.mark.parametrize("kind,d", [(0, 256), (0, 4096), (1, 1280), (2, 1152), (1, 1024)])
+@pytest.mark.parametrize("kind,d", [(0, 256), (0, 4096), (1, 1280), (2, 1152), (1, 1024), (0, 2048),
+                                    (1, 2056), (2, 12)])
 def test_norm(B, kind, d):
     rng = np.random.default_rng(kind * 10000 + d)
     rows, rpb = 260, 130
