@@ -67,12 +67,17 @@ typedef struct {
  * (row stride ldb).  K, lda, ldb multiples of 8; N multiple of 8; pointers 16-byte
  * aligned.  use_simt = 1 runs the plain SIMT kernel (reference / debugging), 0 the
  * tcgen05 + TMA kernel (M = 128, N = 256, K = 16 instructions, fp32 accumulators in
- * TMEM) with 64-element K-blocks, choosing 128 x 256 or (when 256-column tiles would not
- * fill one wave) 128 x 128 tiles and 4 or 8 epilogue warps by itself; 2 the same kernel as
- * 2-CTA clusters in which vertically adjacent tiles share one multicast load of their B
- * tile; 3 and 4 the forms of 0 and 2 with 32-element K-blocks (64-byte swizzle); 5, 6, 7
- * force 128 x 256 tiles with 4 epilogue warps, 128 x 256 with 8, and 128 x 128 with 8
- * (128 x 128 applies to plain, GELU and DELTA epilogues only).
+ * TMEM) with 64-element K-blocks, choosing by itself 128 x 256 or 128 x 128 tiles, 4 or 8
+ * epilogue warps, and whether the tiles left over after the last full wave of CTAs are
+ * split along K over all SMs ("stream-K": fp32 partial tiles in a workspace, summed in a
+ * fixed order by the CTA that finishes a tile last, so results are deterministic); 2 the
+ * same kernel as 2-CTA clusters in which vertically adjacent tiles share one multicast
+ * load of their B tile; 3 and 4 the forms of 0 and 2 with 32-element K-blocks (64-byte
+ * swizzle); 5, 6, 7 force 128 x 256 tiles with 4 epilogue warps, 128 x 256 with 8, and
+ * 128 x 128 with 8 and no stream-K (128 x 128 applies to plain, GELU and DELTA epilogues
+ * only); 8 is 0 without stream-K, 9 is 0 with stream-K whenever the last wave is partial.
+ * The stream-K workspace is owned by the library, one per (device, stream), allocated
+ * or grown by the first call that needs it (after synchronising that stream).
  */
 SGD_API int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
                     const sgd_epilogue_args* epi, int use_simt, void* stream);

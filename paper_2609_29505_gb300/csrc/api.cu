@@ -18,6 +18,7 @@
 #include <functional>
 #include <map>
 #include <memory>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -129,6 +130,13 @@ struct sgd_ctx {
   int gemm_bk = 64;   // default K-block of the tcgen05 GEMM
   int exec_mode = SGD_EXEC_JAGGED_GRAPH;
   float* h_pad = nullptr;  // padded mode: residual that discarded branch updates land in
+  // stream-K GEMM workspace, shared by every GEMM of this context (they run one after
+  // another on one stream); grown when a new plan needs more, the old buffers stay
+  // allocated for graphs captured with them
+  float* sk_ws = nullptr;
+  int* sk_cnt = nullptr;
+  size_t sk_ws_floats = 0, sk_need_floats = 0;
+  int sk_cnt_n = 0, sk_need_cnt = 0;
   // buffers
   float* h = nullptr;
   f16* xn = nullptr;
@@ -236,6 +244,10 @@ int make_gemm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, cons
   plan->bk = (c->d.flags & SGD_FLAG_GEMM_BK64) ? 64 : c->gemm_bk;
   const char* why = "";
   if (gemm_plan(*plan, &why) != 0) return fail(SGD_ERR_SHAPE, std::string(name) + ": " + why);
+  plan->ws_ref = &c->sk_ws;
+  plan->cnt_ref = &c->sk_cnt;
+  c->sk_need_floats = std::max(c->sk_need_floats, gemm_ws_floats(*plan));
+  c->sk_need_cnt = std::max(c->sk_need_cnt, plan->sk_tiles);
   const bool gated = epi.kind == SGD_EPI_GATED;
   const double nb = gated ? 2.0 * N : N;
   double out_b;
@@ -589,6 +601,22 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
   return make_gemm_op(c, ops, "head.linear", c->xn, D, c->pw_head, D, M, d.d_out, D, e);
 }
 
+// Stream-K workspace for the GEMM plans built so far (tickets zeroed once; every launch
+// that completes leaves them zero).
+int ensure_sk_ws(sgd_ctx* c) {
+  int rc;
+  if (c->sk_need_floats > c->sk_ws_floats) {
+    if ((rc = c->alloc(&c->sk_ws, c->sk_need_floats, &c->ws_bytes))) return rc;
+    c->sk_ws_floats = c->sk_need_floats;
+  }
+  if (c->sk_need_cnt > c->sk_cnt_n) {
+    if ((rc = c->alloc(&c->sk_cnt, static_cast<size_t>(c->sk_need_cnt), &c->ws_bytes))) return rc;
+    CUDA_TRY(cudaMemset(c->sk_cnt, 0, sizeof(int) * c->sk_need_cnt));
+    c->sk_cnt_n = c->sk_need_cnt;
+  }
+  return SGD_OK;
+}
+
 int run_ops(const std::vector<Op>& ops, cudaStream_t s) {
   for (const Op& op : ops) {
     cudaError_t e = op.run(s);
@@ -829,7 +857,7 @@ int prepare_step(sgd_ctx* c, const void* in, void* out, float t, const sgd_cond*
     std::vector<Op> ops;
     int rc = ctx_kv_ops(c, cond->ctx, ops);
     if (rc) return rc;
-    if ((rc = run_ops(ops, s))) return rc;
+    if ((rc = ensure_sk_ws(c)) || (rc = run_ops(ops, s))) return rc;
   }
   return SGD_OK;
 }
@@ -912,7 +940,7 @@ static int build_graphs(sgd_ctx* c) {
     std::vector<uint8_t> write(c->U, 0);
     for (int u = 0; u < c->U; ++u) write[u] = (c->S[u] == s && s < T) ? 1 : 0;
     std::vector<Op> ops;
-    if ((rc = build_program(c, c->patterns[pid], write, ops))) return rc;
+    if ((rc = build_program(c, c->patterns[pid], write, ops)) || (rc = ensure_sk_ws(c))) return rc;
     cudaGraph_t g = nullptr;
     CUDA_TRY(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeRelaxed));
     rc = run_ops(ops, c->cap_stream);
@@ -1135,6 +1163,11 @@ int sgd_get_info(const sgd_ctx* c, sgd_info* info) {
 int sgd_reset(sgd_ctx* c) {
   if (!c) return fail(SGD_ERR_ARG, "null context");
   c->last_step = 0;
+  // a GEMM that stopped on an expired wait may have left stream-K tickets behind
+  if (c->sk_cnt) {
+    CUDA_TRY(cudaSetDevice(c->device));
+    CUDA_TRY(cudaMemset(c->sk_cnt, 0, sizeof(int) * c->sk_cnt_n));
+  }
   return SGD_OK;
 }
 
@@ -1158,6 +1191,49 @@ int sgd_sampler_update(float* z, const float* eps, float alpha, float beta, int6
 
 // ----- kernel-level entry points (include/sgd_kernels.h) -----
 
+namespace {
+
+// Stream-K workspace of the kernel-level GEMM entry, one per (device, stream): launches on
+// one stream run in order, so they can share it.  Grown on demand (after the stream has
+// finished with the old one).
+struct KernelWs {
+  float* ws = nullptr;
+  size_t floats = 0;
+  int* cnt = nullptr;
+  int n_cnt = 0;
+};
+std::mutex g_kws_mu;
+std::map<std::pair<int, void*>, KernelWs> g_kws;
+
+int kernel_ws(int dev, void* stream, size_t floats, int n_cnt, KernelWs** out) {
+  std::lock_guard<std::mutex> lk(g_kws_mu);
+  KernelWs& w = g_kws[{dev, stream}];
+  if (floats > w.floats || n_cnt > w.n_cnt) {
+    CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+    if (floats > w.floats) {
+      if (w.ws) cudaFree(w.ws);
+      w.ws = nullptr;
+      w.floats = 0;
+      cudaError_t e = cudaMalloc(&w.ws, floats * sizeof(float));
+      if (e != cudaSuccess) return fail(SGD_ERR_OOM, std::string("cudaMalloc: ") + cudaGetErrorString(e));
+      w.floats = floats;
+    }
+    if (n_cnt > w.n_cnt) {
+      if (w.cnt) cudaFree(w.cnt);
+      w.cnt = nullptr;
+      w.n_cnt = 0;
+      cudaError_t e = cudaMalloc(&w.cnt, n_cnt * sizeof(int));
+      if (e != cudaSuccess) return fail(SGD_ERR_OOM, std::string("cudaMalloc: ") + cudaGetErrorString(e));
+      CUDA_TRY(cudaMemset(w.cnt, 0, n_cnt * sizeof(int)));
+      w.n_cnt = n_cnt;
+    }
+  }
+  *out = &w;
+  return SGD_OK;
+}
+
+}  // namespace
+
 int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
                     const sgd_epilogue_args* ea, int use_simt, void* stream) {
   if (!ea) return fail(SGD_ERR_ARG, "null epilogue");
@@ -1170,13 +1246,15 @@ int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N
   p.M = M;
   p.N = N;
   p.K = K;
-  if (use_simt < 0 || use_simt > 7) return fail(SGD_ERR_ARG, "gemm: variant must be in 0..7");
+  if (use_simt < 0 || use_simt > 9) return fail(SGD_ERR_ARG, "gemm: variant must be in 0..9");
   p.simt = use_simt == 1;
   p.cluster = (use_simt == 2 || use_simt == 4) ? 2 : 1;
   p.bk = (use_simt == 3 || use_simt == 4) ? 32 : 64;
   if (use_simt == 5) { p.bn = 256; p.epiw = 4; }
   if (use_simt == 6) { p.bn = 256; p.epiw = 8; }
-  if (use_simt == 7) { p.bn = 128; p.epiw = 8; }
+  if (use_simt == 7) { p.bn = 128; p.epiw = 8; p.sk = 0; }
+  if (use_simt == 8) p.sk = 0;
+  if (use_simt == 9) p.sk = 1;
   EpiParams& e = p.epi;
   e = EpiParams{};
   e.kind = ea->kind;
@@ -1201,6 +1279,17 @@ int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N
   const char* why = "";
   const int rc = gemm_plan(p, &why);
   if (rc) return fail(rc == -5 ? SGD_ERR_CUDA : (rc == -1 ? SGD_ERR_ARG : SGD_ERR_SHAPE), why);
+  if (p.sk_tiles > 0) {
+    int dev = 0;
+    CUDA_TRY(cudaGetDevice(&dev));
+    KernelWs* w = nullptr;
+    const int wrc = kernel_ws(dev, stream, gemm_ws_floats(p), p.sk_tiles, &w);
+    if (wrc) return wrc;
+    p.ws_ref = &w->ws;
+    p.cnt_ref = &w->cnt;
+    // a launch that stopped on an expired wait can leave counters behind; start from zero
+    CUDA_TRY(cudaMemsetAsync(w->cnt, 0, sizeof(int) * p.sk_tiles, static_cast<cudaStream_t>(stream)));
+  }
   CUDA_TRY(gemm_launch(p, static_cast<cudaStream_t>(stream)));
   return SGD_OK;
 }

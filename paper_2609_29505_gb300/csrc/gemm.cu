@@ -19,6 +19,7 @@
 //               of tile i overlap the MMAs of tile i+1.
 // Every wait is bounded (common.cuh); on expiry the CTA drains its own copies and
 // MMAs, frees TMEM and exits with the device status word set.
+#include <algorithm>
 #include <cstdio>
 #include <cstring>
 #include <mutex>
@@ -51,7 +52,7 @@ struct TileCfg {
   static constexpr int kStages = (192 * 1024) / kStageBytes;
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
   static_assert(kSmemBytes <= 232448, "shared memory");
-  static_assert(2 * kStages + 5 <= 30, "barrier block");
+  static_assert((2 * kStages + 5) * 8 + 3 * 4 <= 256, "barrier block");
 };
 
 template <int BK>
@@ -67,6 +68,10 @@ struct TcArgs {
   int num_m, num_n, num_k;
   int gated;    // B second half starts at row N (= f)
   int* status;
+  // stream-K (0 tiles: data-parallel only)
+  int sk_tiles, sk_ctas, max_seg;
+  float* ws;    // [sk_tiles][max_seg][128 * BN] fp32 partial accumulators (max_seg <= kMaxSeg)
+  int* sk_cnt;  // [sk_tiles] tickets, zero between launches
 };
 
 __device__ int g_status;  // device status word (bounded-wait expiry codes)
@@ -128,27 +133,116 @@ __device__ __forceinline__ void u32_to_f32x16(const uint32_t* r, float* f, float
   for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(r[i]) * alpha;
 }
 
-// Epilogue of one 128 x BN accumulator: this thread owns tile row `row` (TMEM lane
-// row - m0), reads from `tbase` and handles accumulator columns [cb, ce) (gated:
-// output columns [cb, ce) of the BN / 2 the tile produces).
+// Accumulator sources for the epilogue.  load2(c0, c1, x, y) returns alpha times the
+// accumulator at tile columns [c0, c0 + 16) and [c1, c1 + 16) of this thread's row.
+// TmemSrc reads the tile's TMEM accumulator; every lane of the warp must call it together
+// (tcgen05.ld is .sync.aligned).
+struct TmemSrc {
+  uint32_t tbase;
+  float alpha;
+  __device__ __forceinline__ void load2(int c0, int c1, float* x, float* y) const {
+    uint32_t r0[16], r1[16];
+    tmem_ld16(tbase + c0, r0);
+    tmem_ld16(tbase + c1, r1);
+    tmem_ld_wait16(r0);
+    tmem_ld_wait16(r1);
+    u32_to_f32x16(r0, x, alpha);
+    u32_to_f32x16(r1, y, alpha);
+  }
+};
+
+// Stream-K partial tiles in the workspace: slot j of a tile holds the raw fp32
+// accumulator of its j-th K segment (at most kMaxSeg segments), laid out
+// [BN / 4][128 rows] x float4 so that a warp's 32 rows are one contiguous 512-byte run.
+// WsSrc, used by the CTA that finishes a tile, adds the slots in slot order (a fixed
+// order, so the result does not depend on which CTA finishes last), loading two slots
+// at a time.
+constexpr int kMaxSeg = 4;
+
 template <int BN>
+struct WsSrc {
+  const float* slot0;
+  int nseg;
+  int r;  // row within the tile
+  float alpha;
+  __device__ __forceinline__ void load16(int c, float* x) const {
+    const float4* p = reinterpret_cast<const float4*>(slot0) + (c >> 2) * kBM + r;
+    constexpr size_t kSlot = static_cast<size_t>(kBM) * BN / 4;  // float4 per slot
+#pragma unroll
+    for (int i = 0; i < 16; ++i) x[i] = 0.f;
+#pragma unroll
+    for (int j = 0; j < kMaxSeg; j += 2) {
+      if (j < nseg) {
+        // the second slot's loads are unconditional (a predicated load makes the compiler
+        // spill); past the last slot they repeat the first slot's addresses, unused
+        const int j1 = j + 1 < nseg ? j + 1 : j;
+        float4 u[4], w[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          u[i] = __ldcg(p + j * kSlot + i * kBM);
+          w[i] = __ldcg(p + j1 * kSlot + i * kBM);
+        }
+        const bool two = j + 1 < nseg;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          x[4 * i] += u[i].x;
+          x[4 * i + 1] += u[i].y;
+          x[4 * i + 2] += u[i].z;
+          x[4 * i + 3] += u[i].w;
+          x[4 * i] = two ? x[4 * i] + w[i].x : x[4 * i];
+          x[4 * i + 1] = two ? x[4 * i + 1] + w[i].y : x[4 * i + 1];
+          x[4 * i + 2] = two ? x[4 * i + 2] + w[i].z : x[4 * i + 2];
+          x[4 * i + 3] = two ? x[4 * i + 3] + w[i].w : x[4 * i + 3];
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 16; ++i) x[i] *= alpha;
+  }
+  __device__ __forceinline__ void load2(int c0, int c1, float* x, float* y) const {
+    load16(c0, x);
+    load16(c1, y);
+  }
+};
+
+// Store the raw TMEM accumulator columns [c0, c1) of this thread's row r into a
+// workspace slot (layout of WsSrc).
+template <int BN>
+__device__ __forceinline__ void store_partial(float* slot, int r, uint32_t tbase, int c0, int c1) {
+  uint32_t v0[16], v1[16];
+  for (int c = c0; c < c1; c += 32) {
+    tmem_ld16(tbase + c, v0);
+    tmem_ld16(tbase + c + 16, v1);
+    tmem_ld_wait16(v0);
+    tmem_ld_wait16(v1);
+    float4* p = reinterpret_cast<float4*>(slot) + (c >> 2) * kBM + r;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      __stcg(p + i * kBM, make_float4(__uint_as_float(v0[4 * i]), __uint_as_float(v0[4 * i + 1]),
+                                      __uint_as_float(v0[4 * i + 2]), __uint_as_float(v0[4 * i + 3])));
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      __stcg(p + (4 + i) * kBM,
+             make_float4(__uint_as_float(v1[4 * i]), __uint_as_float(v1[4 * i + 1]),
+                         __uint_as_float(v1[4 * i + 2]), __uint_as_float(v1[4 * i + 3])));
+  }
+}
+
+// Epilogue of one 128 x BN accumulator: this thread owns tile row `row` and handles
+// accumulator columns [cb, ce) (gated: output columns [cb, ce) of the BN / 2 the tile
+// produces), reading the accumulator through `src`.
+template <int BN, class Src>
 __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int row, int n_blk,
-                                              uint32_t tbase, int cb, int ce) {
+                                              const Src& src, int cb, int ce) {
   constexpr int kBN = BN;
   const EpiParams& e = a.epi;
   const bool row_ok = row < a.M;
-  uint32_t r0[16], r1[16];
   float x[16], y[16];
   if (a.gated) {
     const int n0 = n_blk * (kBN / 2);
     for (int c = cb; c < ce; c += 16) {
       if (n0 + c >= a.N) break;
-      tmem_ld16(tbase + c, r0);
-      tmem_ld16(tbase + kBN / 2 + c, r1);
-      tmem_ld_wait16(r0);
-      tmem_ld_wait16(r1);
-      u32_to_f32x16(r0, x, e.alpha);
-      u32_to_f32x16(r1, y, e.alpha);
+      src.load2(c, kBN / 2 + c, x, y);
 #pragma unroll
       for (int i = 0; i < 16; ++i) x[i] = e.act ? x[i] * gelu_erf_f(y[i]) : silu_f(x[i]) * y[i];
       if (row_ok) {
@@ -166,12 +260,7 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
       if (n0 + hb >= a.N) break;
       const bool rot = (n0 + hb) < e.rope_cols;
       for (int j = 0; j < hd; j += 16) {
-        tmem_ld16(tbase + hb + j, r0);
-        tmem_ld16(tbase + hb + hd + j, r1);
-        tmem_ld_wait16(r0);
-        tmem_ld_wait16(r1);
-        u32_to_f32x16(r0, x, e.alpha);
-        u32_to_f32x16(r1, y, e.alpha);
+        src.load2(hb + j, hb + hd + j, x, y);
         if (rot && row_ok) {
           const float* cs = e.rope_cos + static_cast<int64_t>(pos) * hd + j;
           const float* sn = e.rope_sin + static_cast<int64_t>(pos) * hd + j;
@@ -196,12 +285,7 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
   }
   for (int c = cb; c < ce; c += 32) {
     if (n0 + c >= a.N) break;
-    tmem_ld16(tbase + c, r0);
-    tmem_ld16(tbase + c + 16, r1);
-    tmem_ld_wait16(r0);
-    tmem_ld_wait16(r1);
-    u32_to_f32x16(r0, x, e.alpha);
-    u32_to_f32x16(r1, y, e.alpha);
+    src.load2(c, c + 16, x, y);
     if (row_ok) {
 #pragma unroll
       for (int q = 0; q < 2; ++q) {
@@ -230,10 +314,86 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
   }
 }
 
+// Named barrier 1 over the epilogue warps, returning the AND of `v` over them.
+__device__ __forceinline__ bool epi_bar_and(bool v, int nthreads) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.and.pred q, 1, %2, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(v)), "r"(nthreads)
+      : "memory");
+  return r != 0;
+}
+
+__device__ __forceinline__ void epi_bar(int nthreads) {
+  asm volatile("bar.sync 1, %0;" ::"r"(nthreads) : "memory");
+}
+
+// Stream-K split of the K iterations of tiles [0, sk_tiles): CTA c < sk_ctas owns the
+// contiguous iterations [start(c), start(c + 1)) of the sk_tiles * num_k iteration space,
+// start(c) = floor(c * total / sk_ctas); every CTA owns at least one iteration (the host
+// keeps sk_ctas <= total).  The CTA owning iteration i is the largest c with start(c) <= i.
+__device__ __forceinline__ int sk_start(int c, int total, int ctas) {
+  return static_cast<int>(static_cast<int64_t>(c) * total / ctas);
+}
+__device__ __forceinline__ int sk_owner(int i, int total, int ctas) {
+  return static_cast<int>((static_cast<int64_t>(i + 1) * ctas - 1) / total);
+}
+
+// The work of one CTA: first its stream-K segments (tiles t_sk0 .., K iterations clipped to
+// [sk_s, sk_e)), then the data-parallel tiles sk_tiles + unit0 + d * unit_step, full K.
+struct CtaWork {
+  int sk_s, sk_e, t_sk0, n_sk;
+  int unit0, unit_step, n_units;
+};
+
+__device__ __forceinline__ CtaWork cta_work(const TcArgs& a, int num_tiles, int unit0, int unit_step) {
+  CtaWork w;
+  w.unit0 = unit0;
+  w.unit_step = unit_step;
+  w.sk_s = w.sk_e = w.t_sk0 = w.n_sk = 0;
+  if (a.sk_tiles > 0 && static_cast<int>(blockIdx.x) < a.sk_ctas) {
+    const int total = a.sk_tiles * a.num_k;
+    w.sk_s = sk_start(blockIdx.x, total, a.sk_ctas);
+    w.sk_e = sk_start(blockIdx.x + 1, total, a.sk_ctas);
+    w.t_sk0 = w.sk_s / a.num_k;
+    w.n_sk = (w.sk_e - 1) / a.num_k - w.t_sk0 + 1;
+  }
+  const int dp = num_tiles - a.sk_tiles;
+  const int n_dp = unit0 < dp ? (dp - unit0 + unit_step - 1) / unit_step : 0;
+  w.n_units = w.n_sk + n_dp;
+  return w;
+}
+
+__device__ __forceinline__ void unit_at(const TcArgs& a, const CtaWork& w, int u, int& tile, int& k0,
+                                        int& k1) {
+  if (u < w.n_sk) {
+    tile = w.t_sk0 + u;
+    const int base = tile * a.num_k;
+    k0 = max(w.sk_s - base, 0);
+    k1 = min(w.sk_e - base, a.num_k);
+  } else {
+    tile = a.sk_tiles + w.unit0 + (u - w.n_sk) * w.unit_step;
+    k0 = 0;
+    k1 = a.num_k;
+  }
+}
+
 // CLUSTER = 2: the two CTAs of a cluster compute vertically adjacent 128-row tiles of
 // the same 256 output columns; each loads its own A box and one of the two B halves,
 // multicast into both CTAs, so every B byte is read from L2 once per pair.  Each CTA's
 // MMA commits the release of a stage to both CTAs (empty barriers count 2 arrivals).
+//
+// Stream-K (CLUSTER = 1, sk_tiles > 0): the K iterations of the first sk_tiles tiles are
+// spread evenly over sk_ctas CTAs (at most kMaxSeg per tile), so that the tiles left over
+// after the last full wave do not leave most SMs idle.  A CTA whose segment does not cover
+// a tile's whole K range stores its raw accumulator in its workspace slot, then draws a
+// ticket from the tile's counter; the CTA that draws the last ticket sums the slots in
+// order, runs the epilogue and puts the counter back to zero.  No CTA ever waits for
+// another.
 template <int CLUSTER, int BK, int BN, int EPIW>
 __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ TcArgs a) {
@@ -253,6 +413,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* last_flag = reinterpret_cast<volatile int*>(tmem_slot + 2);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -286,17 +447,19 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
   // work units: CLUSTER vertically adjacent tiles that share their B columns
   const int num_mu = (a.num_m + CLUSTER - 1) / CLUSTER;
   const int num_tiles = num_mu * a.num_n;
-  const int unit0 = blockIdx.x / CLUSTER, unit_step = gridDim.x / CLUSTER;
+  const CtaWork w = cta_work(a, num_tiles, blockIdx.x / CLUSTER, gridDim.x / CLUSTER);
 
   if (warp == 0) {
     if (lane == 0) {
       int it = 0;
-      for (int tile = unit0; tile < num_tiles; tile += unit_step) {
+      for (int u = 0; u < w.n_units; ++u) {
+        int tile, k0, k1;
+        unit_at(a, w, u, tile, k0, k1);
         const int m_blk = (tile % num_mu) * CLUSTER + crank, n_blk = tile / num_mu;
         const int rb0 = a.gated ? n_blk * 128 : n_blk * kBN;
         const int rb1 = a.gated ? a.N + n_blk * 128 : rb0 + 128;  // BN = 256 only
         bool ok = true;
-        for (int kb = 0; kb < a.num_k; ++kb, ++it) {
+        for (int kb = k0; kb < k1; ++kb, ++it) {
           const int s = it % kStages;
           const uint32_t ph = (it / kStages) & 1;
           if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, a.status, 1)) {
@@ -325,15 +488,17 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = umma_idesc_f16(kBM, kBN);
-      int it = 0, lt = 0;
+      int it = 0;
       bool ok = true;
-      for (int tile = unit0; tile < num_tiles && ok; tile += unit_step, ++lt) {
-        const int acc = lt & 1;
-        const uint32_t aph = (lt >> 1) & 1;
+      for (int u = 0; u < w.n_units && ok; ++u) {
+        int tile, k0, k1;
+        unit_at(a, w, u, tile, k0, k1);
+        const int acc = u & 1;
+        const uint32_t aph = (u >> 1) & 1;
         if (!mbar_wait(&tempty[acc], aph ^ 1u, abort_flag, a.status, 2)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * kBN;
-        for (int kb = 0; kb < a.num_k; ++kb, ++it) {
+        for (int kb = k0; kb < k1; ++kb, ++it) {
           const int s = it % kStages;
           const uint32_t ph = (it / kStages) & 1;
           if (!mbar_wait(&full[s], ph, abort_flag, a.status, 3)) {
@@ -346,7 +511,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k) {
             umma_f16(d_tmem, operand_desc<BK>(a_addr + 32 * k), operand_desc<BK>(b_addr + 32 * k),
-                      idesc, (kb | k) != 0 ? 1u : 0u);
+                      idesc, (kb != k0 || k != 0) ? 1u : 0u);
           }
           if (CLUSTER == 1)
             umma_commit(&empty[s]);
@@ -362,25 +527,75 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
     }
   } else {
     const int q = warp & 3;
+    constexpr int kEpiThreads = 32 * kEpiWarps;
     // column range of this warp: all of the tile (4 epilogue warps) or one half (8)
     const int span = a.gated ? kBN / 2 : kBN;
     const int part = kEpiWarps == 8 ? ((warp - 2) >> 2) : 0;
     const int cb = kEpiWarps == 8 ? part * (span / 2) : 0;
     const int ce = kEpiWarps == 8 ? cb + span / 2 : span;
-    int lt = 0;
+    // accumulator columns this warp stores for a stream-K partial
+    const int pb = kEpiWarps == 8 ? part * (kBN / 2) : 0;
+    const int pe = kEpiWarps == 8 ? pb + kBN / 2 : kBN;
+    const int total = a.sk_tiles * a.num_k;
     void* out = a.epi.out_slot ? *a.epi.out_slot : a.epi.out;
-    for (int tile = unit0; tile < num_tiles; tile += unit_step, ++lt) {
+    for (int u = 0; u < w.n_units; ++u) {
+      int tile, k0, k1;
+      unit_at(a, w, u, tile, k0, k1);
       const int m_blk = (tile % num_mu) * CLUSTER + crank, n_blk = tile / num_mu;
-      const int acc = lt & 1;
-      const uint32_t aph = (lt >> 1) & 1;
-      if (!warp_wait(&tfull[acc], aph, abort_flag, a.status, 4)) break;
-      tc_fence_after();
+      const int acc = u & 1;
+      const uint32_t aph = (u >> 1) & 1;
       const int row = m_blk * kBM + q * 32 + lane;
       const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * kBN;
-      epilogue_tile<kBN>(a, out, row, n_blk, tbase, cb, ce);
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[acc]);
+      if (u >= w.n_sk) {  // data-parallel tile
+        if (!warp_wait(&tfull[acc], aph, abort_flag, a.status, 4)) break;
+        tc_fence_after();
+        epilogue_tile<kBN>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[acc]);
+        continue;
+      }
+      // stream-K unit: every epilogue warp reaches each barrier below, also after an
+      // expired wait, so that they leave the loop together
+      const bool ok = warp_wait(&tfull[acc], aph, abort_flag, a.status, 4);
+      if (k0 == 0 && k1 == a.num_k) {  // the whole K range of the tile lies in this CTA's share
+        if (ok) {
+          tc_fence_after();
+          epilogue_tile<kBN>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&tempty[acc]);
+        }
+        if (!epi_bar_and(ok, kEpiThreads)) break;
+        continue;
+      }
+      // partial: store it, then draw a ticket; the CTA that draws the last one has every
+      // other partial in the workspace already and finishes the tile.  No CTA waits.
+      const int first = sk_owner(tile * a.num_k, total, a.sk_ctas);
+      const int nseg = sk_owner(tile * a.num_k + a.num_k - 1, total, a.sk_ctas) - first + 1;
+      float* slot0 = a.ws + static_cast<size_t>(tile) * a.max_seg * (kBM * kBN);
+      if (ok) {
+        tc_fence_after();
+        store_partial<kBN>(slot0 + static_cast<size_t>(blockIdx.x - first) * (kBM * kBN), q * 32 + lane,
+                           tbase, pb, pe);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[acc]);
+        __threadfence();
+      }
+      if (!epi_bar_and(ok, kEpiThreads)) break;
+      // last_flag is rewritten (next stream-K unit) only after every epilogue thread has
+      // read it, since each reads it before reaching the next epi_bar_and
+      if (threadIdx.x == 64) {
+        __threadfence();
+        *last_flag = atomicAdd(&a.sk_cnt[tile], 1) == nseg - 1 ? 1 : 0;
+      }
+      epi_bar(kEpiThreads);
+      if (*last_flag != 0) {
+        __threadfence();
+        epilogue_tile<kBN>(a, out, row, n_blk, WsSrc<kBN>{slot0, nseg, q * 32 + lane, a.epi.alpha}, cb, ce);
+        if (threadIdx.x == 64) a.sk_cnt[tile] = 0;
+      }
     }
   }
 
@@ -567,6 +782,42 @@ int max_active_pairs() {
   return cached[dev] > 0 ? cached[dev] : 0;
 }
 
+// Stream-K split of the tiles left after the last full wave of `sms` CTAs: their
+// tiles * num_k K iterations go to up to `sms` CTAs, at least a third of a tile's K range
+// each, so that no tile is shared by more than kMaxSeg = 4 CTAs.  Measured on GB300 under
+// its power cap, the split pays only where the last wave leaves much of the GPU idle
+// (>= 12% of the tile slots of the launch), K is long enough (>= 48 K-blocks) for the
+// partial stores and sums to be small next to a tile, and at least one full wave of
+// data-parallel tiles follows to hide them; `force` takes any valid split.  max_seg:
+// most CTAs sharing a tile, with the kernel's owner arithmetic.
+struct SkSplit {
+  int tiles = 0, ctas = 0, max_seg = 0;
+};
+
+SkSplit sk_split(int num_tiles, int num_k, int sms, bool force = false) {
+  SkSplit r;
+  const int rem = num_tiles % sms;
+  if (rem == 0 || num_k < 2) return r;
+  const int total = rem * num_k;
+  const int min_iters = (num_k + 2) / 3;
+  const int ctas = std::min(sms, total / min_iters);
+  if (ctas <= rem) return r;
+  const int slots = (num_tiles / sms + 1) * sms;
+  const bool gain = num_k >= 48 && num_tiles >= sms && (slots - num_tiles) >= 0.12 * slots;
+  if (!gain && !force) return r;
+  auto owner = [&](int64_t i) { return static_cast<int>(((i + 1) * ctas - 1) / total); };
+  int max_seg = 0;
+  for (int t = 0; t < rem; ++t) {
+    const int nseg = owner(static_cast<int64_t>(t) * num_k + num_k - 1) - owner(static_cast<int64_t>(t) * num_k) + 1;
+    max_seg = std::max(max_seg, nseg);
+  }
+  if (max_seg > kMaxSeg) return r;
+  r.tiles = rem;
+  r.ctas = ctas;
+  r.max_seg = max_seg;
+  return r;
+}
+
 int gemm_plan(GemmPlan& p, const char** why) {
   const EpiParams& e = p.epi;
   const bool gated = e.kind == SGD_EPI_GATED;
@@ -607,21 +858,26 @@ int gemm_plan(GemmPlan& p, const char** why) {
   }
   const int num_m = (p.M + kBM - 1) / kBM;
   const int sms = num_sms();
+  const int num_k = (p.K + p.bk - 1) / p.bk;
+  if (p.cluster != 1 && p.cluster != 2) p.cluster = 1;
   // tile shape: 128-column tiles when they need clearly fewer tile-times than 256-column
   // tiles (a 128-column tile takes half the time of a 256-column one, at about 3/4 of its
-  // efficiency, so: 2 * waves_128 < 3 * waves_256); they need a plain epilogue and
-  // one-CTA launches.  4 epilogue warps for RoPE and gated epilogues.
+  // efficiency, so: 2 * waves_128 < 3 * waves_256) and stream-K does not already even out
+  // the last wave; they need a plain epilogue and one-CTA launches.  4 epilogue warps for
+  // RoPE and gated epilogues.
   const bool small_ok = !gated && e.kind != SGD_EPI_ROPE && p.bk == 64 && p.cluster == 1;
   if (p.bn == 0) {
-    const int w256 = (num_m * ((p.N + 255) / 256) + sms - 1) / sms;
+    const int t256 = num_m * (gated ? (p.N + 127) / 128 : (p.N + 255) / 256);
+    const int w256 = (t256 + sms - 1) / sms;
     const int w128 = (num_m * ((p.N + 127) / 128) + sms - 1) / sms;
-    p.bn = (small_ok && 2 * w128 < 3 * w256) ? 128 : 256;
+    SkSplit sk256 = sk_split(t256, num_k, sms);
+    const bool sk_on = p.cluster == 1 && p.sk != 0 && sk256.tiles > 0;
+    p.bn = (small_ok && !sk_on && 2 * w128 < 3 * w256) ? 128 : 256;
   }
   if (p.bn != 128 || !small_ok) p.bn = 256;
   if (p.epiw == 0) p.epiw = (e.kind == SGD_EPI_ROPE || gated) ? 4 : 8;
   if (p.bn == 128 || p.cluster == 2 || p.bk == 32) p.epiw = 8;
   const int num_n = gated ? (p.N + 127) / 128 : (p.N + p.bn - 1) / p.bn;
-  if (p.cluster != 1 && p.cluster != 2) p.cluster = 1;
   if (p.cluster == 2 && num_m < 2) p.cluster = 1;  // nothing to share
   int max_units = sms;
   if (p.cluster == 2) {
@@ -633,7 +889,21 @@ int gemm_plan(GemmPlan& p, const char** why) {
   }
   const int units = ((num_m + p.cluster - 1) / p.cluster) * num_n;
   p.grid = (units < max_units ? units : max_units) * p.cluster;
+  p.sk_tiles = p.sk_ctas = p.max_seg = 0;
+  if (p.cluster == 1 && p.sk != 0) {
+    const SkSplit k = sk_split(units, num_k, sms, p.sk == 1);
+    if (k.tiles > 0) {
+      p.sk_tiles = k.tiles;
+      p.sk_ctas = k.ctas;
+      p.max_seg = k.max_seg;
+      p.grid = units >= sms ? sms : k.ctas;
+    }
+  }
   return 0;
+}
+
+size_t gemm_ws_floats(const GemmPlan& p) {
+  return p.sk_tiles > 0 ? static_cast<size_t>(p.sk_tiles) * p.max_seg * kBM * p.bn : 0;
 }
 
 template <int CLUSTER, int BK, int BN, int EPIW>
@@ -689,6 +959,12 @@ cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s) {
   a.num_n = a.gated ? (p.N + 127) / 128 : (p.N + p.bn - 1) / p.bn;
   a.num_k = (p.K + p.bk - 1) / p.bk;
   a.status = device_status_ptr();
+  a.sk_tiles = p.sk_tiles;
+  a.sk_ctas = p.sk_ctas;
+  a.max_seg = p.max_seg;
+  a.ws = p.ws_ref ? *p.ws_ref : nullptr;
+  a.sk_cnt = p.cnt_ref ? *p.cnt_ref : nullptr;
+  if (p.sk_tiles > 0 && (!a.ws || !a.sk_cnt || p.cluster != 1)) return cudaErrorInvalidValue;
   if (p.bk == 32)
     return p.cluster == 2 ? launch_tc<2, 32, 256, 8>(p, a, s) : launch_tc<1, 32, 256, 8>(p, a, s);
   if (p.cluster == 2) return launch_tc<2, 64, 256, 8>(p, a, s);

@@ -53,14 +53,23 @@ struct GemmPlan {
   int bk = 64;               // K elements per stage: 64 (128-byte swizzle) or 32 (64-byte)
   int bn = 0;                // output columns per tile: 256, 128, or 0 = choose by tile count
   int epiw = 0;              // epilogue warps: 4, 8, or 0 = choose by epilogue kind
+  int sk = -1;               // stream-K for the tiles after the last full wave: -1 choose, 0 off, 1 on
   CUtensorMap tmap_a;
   CUtensorMap tmap_b;
   int grid = 0;
+  int sk_tiles = 0, sk_ctas = 0, max_seg = 0;  // stream-K split (set by gemm_plan)
+  // stream-K workspace, read at launch time through these (so that a plan built before its
+  // workspace exists stays valid): fp32 [gemm_ws_floats] and int [sk_tiles] tickets that
+  // must be zero before the first launch; a launch leaves them zero when it completes.
+  float* const* ws_ref = nullptr;
+  int* const* cnt_ref = nullptr;
 };
 
 // Validates shapes and builds the tensor maps; returns an sgd_status.
 int gemm_plan(GemmPlan& p, const char** why);
 cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s);
+// fp32 elements of stream-K workspace a planned GEMM needs (0: data-parallel only).
+size_t gemm_ws_floats(const GemmPlan& p);
 int* device_status_ptr();  // device address of the shared status word
 int num_sms();
 // 2-D fp16 tensor map: [rows, cols] with row stride ld elements, box 64 x box_rows,

@@ -46,10 +46,15 @@ def _check_f16(got, want, extra_abs=0.0):
                            f"{np.max(np.abs(got - want)):.3e}, rms(want) {scale:.3e}")
 
 
+# sgd_kernel_gemm variant codes (include/sgd_kernels.h)
+VARIANTS = [0, 2, 3, 4, 5, 6, 7, 8, 9, 1]
+VARIANT_IDS = ["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "tcgen05_epi4",
+               "tcgen05_epi8", "tcgen05_bn128", "tcgen05_dp", "tcgen05_streamk", "simt"]
+
 GEMM_SHAPES = [(64, 256, 256), (300, 520, 688), (129, 264, 72), (1000, 1376, 512), (4128, 1024, 2048)]
 
 
-@pytest.mark.parametrize("simt", [0, 2, 3, 4, 5, 6, 7, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "tcgen05_epi4", "tcgen05_epi8", "tcgen05_bn128", "simt"])
+@pytest.mark.parametrize("simt", VARIANTS, ids=VARIANT_IDS)
 @pytest.mark.parametrize("M,N,K", GEMM_SHAPES)
 def test_gemm_bf16(B, M, N, K, simt):
     rng = np.random.default_rng(M + N + K)
@@ -63,7 +68,7 @@ def test_gemm_bf16(B, M, N, K, simt):
     _check_f16(out, odn.linear(_f(A), _f(W)))
 
 
-@pytest.mark.parametrize("simt", [0, 2, 3, 4, 5, 6, 7, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "tcgen05_epi4", "tcgen05_epi8", "tcgen05_bn128", "simt"])
+@pytest.mark.parametrize("simt", VARIANTS, ids=VARIANT_IDS)
 @pytest.mark.parametrize("gated", [False, True])
 def test_gemm_delta_residual_and_cache(B, simt, gated):
     rng = np.random.default_rng(5)
@@ -87,7 +92,7 @@ def test_gemm_delta_residual_and_cache(B, simt, gated):
     _check_f16(cache, delta)
 
 
-@pytest.mark.parametrize("simt", [0, 2, 3, 4, 5, 6, 7, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "tcgen05_epi4", "tcgen05_epi8", "tcgen05_bn128", "simt"])
+@pytest.mark.parametrize("simt", VARIANTS, ids=VARIANT_IDS)
 @pytest.mark.parametrize("act", [0, 1])
 def test_gemm_gated_activation(B, simt, act):
     rng = np.random.default_rng(6)
@@ -103,7 +108,7 @@ def test_gemm_gated_activation(B, simt, act):
     _check_f16(out, want, extra_abs=1e-4 * float(np.abs(want).max()))
 
 
-@pytest.mark.parametrize("simt", [0, 2, 3, 4, 5, 6, 7, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "tcgen05_epi4", "tcgen05_epi8", "tcgen05_bn128", "simt"])
+@pytest.mark.parametrize("simt", VARIANTS, ids=VARIANT_IDS)
 @pytest.mark.parametrize("act", [0, 1])
 def test_gemm_gelu(B, simt, act):
     rng = np.random.default_rng(7)
@@ -119,7 +124,7 @@ def test_gemm_gelu(B, simt, act):
     _check_f16(out, want, extra_abs=1e-4 * float(np.abs(want).max()))
 
 
-@pytest.mark.parametrize("simt", [0, 2, 3, 4, 5, 6, 7, 1], ids=["tcgen05", "tcgen05_cluster2", "tcgen05_bk32", "tcgen05_bk32_cluster2", "tcgen05_epi4", "tcgen05_epi8", "tcgen05_bn128", "simt"])
+@pytest.mark.parametrize("simt", VARIANTS, ids=VARIANT_IDS)
 @pytest.mark.parametrize("dh", [64, 128])
 def test_gemm_rope_epilogue(B, simt, dh):
     rng = np.random.default_rng(8)
@@ -227,3 +232,45 @@ def test_gemm_large_sampled_rows_tcgen05(B):
     rows = np.sort(rng.choice(M, 96, replace=False))
     want = odn.linear(_f(A[rows]), _f(W))
     _check_f16(out[rows], want)
+
+
+@pytest.mark.parametrize("M,N,K,epi", [(4096, 4096, 4096, "f16"), (2048, 1152, 1152, "delta"),
+                                       (1000, 1376, 512, "gelu"), (4096, 4096, 1024, "gated")])
+def test_gemm_streamk_repeatable(B, M, N, K, epi):
+    """Stream-K (leftover tiles split along K over all SMs, partial sums in a workspace):
+    two launches in a row give identical bits (the partials are summed in a fixed order and
+    the tile tickets are back at zero after each launch), and agree with the
+    data-parallel schedule to fp16 rounding and with the oracle on sampled rows."""
+    rng = np.random.default_rng(M + N + K + 1)
+    gated = epi == "gated"
+    A = _rand(rng, (M, K)).cuda()
+    W = _rand(rng, (2 * N if gated else N, K), 1 / math.sqrt(K)).cuda()
+    kind = {"f16": B.EPI_F16, "delta": B.EPI_DELTA, "gelu": B.EPI_GELU, "gated": B.EPI_GATED}[epi]
+
+    def run(variant):
+        if epi == "delta":
+            h = torch.zeros(M, N, device="cuda")
+            e = B.sgd_epilogue_args(kind=kind, h=h.data_ptr(), ldh=N)
+            B.sgd_kernel_gemm(A, W, M, N, K, e, use_simt=variant)
+            return h
+        out = torch.empty(M, N, dtype=torch.float16, device="cuda")
+        e = B.sgd_epilogue_args(kind=kind, out=out.data_ptr(), ldo=N)
+        B.sgd_kernel_gemm(A, W, M, N, K, e, use_simt=variant)
+        return out
+
+    first, second, dp = run(9), run(9), run(8)
+    torch.cuda.synchronize()
+    assert B.sgd_kernel_status() == 0
+    assert torch.equal(first, second)
+    rows = np.sort(rng.choice(M, 64, replace=False))
+    u = odn.linear(_f(A[rows]), _f(W))
+    want = {"f16": u, "delta": u, "gelu": odn.gelu_tanh(u),
+            "gated": odn.silu(u[:, :N]) * u[:, N:] if gated else None}[epi]
+    if epi == "delta":
+        np.testing.assert_allclose(_f(first[rows]), want, rtol=2e-5, atol=2e-5)
+        np.testing.assert_allclose(_f(first), _f(dp), rtol=2e-5, atol=2e-5)
+    else:
+        extra = 1e-4 * float(np.abs(want).max())
+        _check_f16(first[rows], want, extra_abs=extra)
+        a, b = _f(first), _f(dp)  # two fp16 roundings of nearly equal sums: 1 ulp apart at most
+        assert np.all(np.abs(a - b) <= 2.0 ** -10 * np.abs(b) + extra)
