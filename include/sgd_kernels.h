@@ -83,6 +83,27 @@ SGD_API int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int 
                     const sgd_epilogue_args* epi, int use_simt, void* stream);
 
 /*
+ * sgd_kernel_gemm without any device memory allocation.  The paper has no counterpart:
+ * this is an interface for callers that cannot let the library allocate, such as a
+ * process whose device memory is all reserved by its own pool allocator, or one that
+ * cannot take the device-wide synchronisation that cudaMalloc / cudaFree may imply while
+ * its other streams run.  Same arguments, variant codes (`variant` = use_simt above),
+ * kernels and results bit for bit as sgd_kernel_gemm; the only difference is where a
+ * stream-K split keeps its partial tiles and tile tickets: in one fixed array compiled
+ * into the library (32 MiB of fp32 partial tiles, then 1024 tickets) instead of a
+ * workspace the library allocates.
+ * Limit: a problem whose stream-K split needs more than the array holds is rejected
+ * with SGD_ERR_SHAPE before anything is launched (variant 8, or sgd_kernel_gemm, runs it).
+ * The tickets are cleared (cudaMemsetAsync on `stream`) before each stream-K launch; the
+ * partial tiles need no clearing (each is written before it is read within one launch).
+ * Every call on a device uses the same array: calls that can overlap in time (launched
+ * on different streams without ordering, or from several host threads at once) race on
+ * it and can produce wrong results, so order them on one stream or with events.
+ */
+SGD_API int sgd_kernel_gemm_static_ws(const void* A, int lda, const void* B, int ldb, int M, int N,
+                              int K, const sgd_epilogue_args* epi, int variant, void* stream);
+
+/*
  * O = softmax(Q K^T / sqrt(d_head)) V per (sample, head), non-causal, keys beyond n_kv
  * masked.  Row r = b * n_q + i of q / o, row b * n_kv + j of k / v; head h occupies
  * columns [h d_head, (h+1) d_head).  fp16 in and out; d_head in {64, 72, 128};

@@ -49,7 +49,7 @@ EXPORTED = [
     "sgd_get_info", "sgd_reset", "sgd_check_device", "sgd_destroy", "sgd_last_error",
     "sgd_compile_schedule", "sgd_step_profile", "sgd_sampler_update", "sgd_kernel_gemm",
     "sgd_kernel_attention", "sgd_kernel_norm", "sgd_kernel_frozen_run", "sgd_kernel_status",
-    "sgd_set_exec_mode", "sgd_step_host_async", "sgd_host_wait",
+    "sgd_set_exec_mode", "sgd_step_host_async", "sgd_host_wait", "sgd_kernel_gemm_static_ws",
 ]
 EXEC_JAGGED_GRAPH, EXEC_EAGER, EXEC_PADDED_GRAPH = 0, 1, 2
 
@@ -127,6 +127,7 @@ def lib() -> C.CDLL:
                                      C.POINTER(sgd_op_record), i, C.POINTER(C.c_int)]),
             "sgd_sampler_update": (i, [vp, vp, f, f, i64, vp]),
             "sgd_kernel_gemm": (i, [vp, i, vp, i, i, i, i, C.POINTER(sgd_epilogue_args), i, vp]),
+            "sgd_kernel_gemm_static_ws": (i, [vp, i, vp, i, i, i, i, C.POINTER(sgd_epilogue_args), i, vp]),
             "sgd_kernel_attention": (i, [vp, i, vp, vp, i, vp, i, i, i, i, i, i, i, vp]),
             "sgd_kernel_norm": (i, [vp, vp, i, i, i, vp, vp, vp, vp, i, i, f, vp]),
             "sgd_kernel_frozen_run": (i, [vp, C.POINTER(vp), i, i64, vp]),
@@ -188,6 +189,14 @@ def sgd_kernel_gemm(A, B, M, N, K, epi: sgd_epilogue_args, use_simt=False, lda=N
     return check(lib().sgd_kernel_gemm(_ptr(A), lda or K, _ptr(B), ldb or K, M, N, K,
                                        C.byref(epi), int(use_simt), _stream(stream)),
                  "sgd_kernel_gemm")
+
+
+def sgd_kernel_gemm_static_ws(A, B, M, N, K, epi: sgd_epilogue_args, variant=0, lda=None, ldb=None,
+                              stream=None):
+    """sgd_kernel_gemm that allocates no device memory (stream-K scratch in a fixed array)."""
+    return check(lib().sgd_kernel_gemm_static_ws(_ptr(A), lda or K, _ptr(B), ldb or K, M, N, K,
+                                                 C.byref(epi), int(variant), _stream(stream)),
+                 "sgd_kernel_gemm_static_ws")
 
 
 def sgd_kernel_attention(q, ldq, k, v, ldkv, o, ldo, batch, n_q, n_kv, n_heads, d_head,

@@ -1294,6 +1294,71 @@ int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N
   return SGD_OK;
 }
 
+int sgd_kernel_gemm_static_ws(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
+                              const sgd_epilogue_args* ea, int variant, void* stream) {
+  if (!ea) return fail(SGD_ERR_ARG, "null epilogue");
+  if (ea->kind < 0 || ea->kind > SGD_EPI_ROPE) return fail(SGD_ERR_ARG, "bad epilogue kind");
+  if (variant < 0 || variant > 9) return fail(SGD_ERR_ARG, "gemm: variant must be in 0..9");
+  GemmPlan p;
+  p.A = H16(A);
+  p.lda = lda;
+  p.B = H16(B);
+  p.ldb = ldb;
+  p.M = M;
+  p.N = N;
+  p.K = K;
+  p.simt = variant == 1;
+  p.cluster = (variant == 2 || variant == 4) ? 2 : 1;
+  p.bk = (variant == 3 || variant == 4) ? 32 : 64;
+  if (variant == 5) { p.bn = 256; p.epiw = 4; }
+  if (variant == 6) { p.bn = 256; p.epiw = 8; }
+  if (variant == 7) { p.bn = 128; p.epiw = 8; p.sk = 0; }
+  if (variant == 8) p.sk = 0;
+  if (variant == 9) p.sk = 1;
+  EpiParams& e = p.epi;
+  e = EpiParams{};
+  e.kind = ea->kind;
+  e.alpha = ea->alpha != 0.f ? ea->alpha : 1.f;
+  e.out = ea->out;
+  e.ldo = ea->ldo;
+  e.h = ea->h;
+  e.ldh = ea->ldh;
+  e.cache = static_cast<f16*>(ea->cache);
+  e.ld_cache = ea->ld_cache;
+  e.gate = ea->gate;
+  e.ld_gate = ea->ld_gate;
+  e.rows_per_batch = ea->rows_per_batch > 0 ? ea->rows_per_batch : 1;
+  e.act = ea->act;
+  e.rope_cos = ea->rope_cos;
+  e.rope_sin = ea->rope_sin;
+  e.rope_tokens = ea->rope_tokens;
+  e.d_head = ea->d_head;
+  e.rope_cols = ea->rope_cols;
+  e.M = M;
+  e.N = N;
+  const char* why = "";
+  const int rc = gemm_plan(p, &why);
+  if (rc) return fail(rc == -5 ? SGD_ERR_CUDA : (rc == -1 ? SGD_ERR_ARG : SGD_ERR_SHAPE), why);
+  float* ws = nullptr;
+  int* tickets = nullptr;
+  if (p.sk_tiles > 0) {
+    size_t cap = 0;
+    int n_cap = 0;
+    if (gemm_static_scratch(&ws, &cap, &tickets, &n_cap, &why)) return fail(SGD_ERR_CUDA, why);
+    if (gemm_ws_floats(p) > cap || p.sk_tiles > n_cap)
+      return fail(SGD_ERR_SHAPE, "gemm: the stream-K split of this problem needs " +
+                                     std::to_string(gemm_ws_floats(p) * sizeof(float)) +
+                                     " bytes of partial tiles, more than the " + std::to_string(cap * sizeof(float)) +
+                                     "-byte static scratch (use sgd_kernel_gemm, or variant 8)");
+    p.ws_ref = &ws;
+    p.cnt_ref = &tickets;
+    // the tickets must start at zero (a launch stopped on an expired wait can leave some)
+    CUDA_TRY(cudaMemsetAsync(tickets, 0, sizeof(int) * p.sk_tiles, static_cast<cudaStream_t>(stream)));
+  }
+  CUDA_TRY(gemm_launch(p, static_cast<cudaStream_t>(stream)));
+  return SGD_OK;
+}
+
 int sgd_kernel_attention(const void* q, int ldq, const void* k, const void* v, int ldkv, void* o,
                          int ldo, int batch, int n_q, int n_kv, int n_heads, int d_head, int impl,
                          void* stream) {

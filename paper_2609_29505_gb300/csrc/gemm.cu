@@ -735,6 +735,45 @@ int num_sms() {
   return n > 0 ? n : 1;
 }
 
+// ----------------------------------------------------------------------------
+// Static stream-K scratch of sgd_kernel_gemm_static_ws: callers of that entry cannot
+// have the library allocate device memory, so its stream-K partial tiles and tickets
+// live in this fixed array instead: kStaticWsBytes of fp32 partials (enough for the
+// 4096 x 4096 projections at K >= 3072 on 152 SMs, 56 tiles x 4 segments x 128 KB), then
+// kStaticTickets tile tickets.  The array is zero when the module loads; the entry
+// clears the tickets before each launch and the partials need no clearing.
+// ----------------------------------------------------------------------------
+constexpr size_t kStaticWsBytes = static_cast<size_t>(32) << 20;
+constexpr int kStaticTickets = 1024;
+static __device__ __align__(256) uint8_t g_static_scratch[kStaticWsBytes + kStaticTickets * sizeof(int)];
+
+int gemm_static_scratch(float** ws, size_t* ws_floats, int** tickets, int* n_tickets, const char** why) {
+  constexpr int kMaxDevices = 64;
+  static std::mutex mu;
+  static uint8_t* addr[kMaxDevices] = {nullptr};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+    *why = "gemm: no current CUDA device";
+    return -1;
+  }
+  std::lock_guard<std::mutex> lk(mu);
+  if (!addr[dev]) {
+    // once per device, with that device current (the symbol has one instance per device)
+    void* q = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&q, g_static_scratch);
+    if (e != cudaSuccess || !q) {
+      *why = "gemm: cudaGetSymbolAddress of the static stream-K scratch failed";
+      return -1;
+    }
+    addr[dev] = static_cast<uint8_t*>(q);
+  }
+  *ws = reinterpret_cast<float*>(addr[dev]);
+  *ws_floats = kStaticWsBytes / sizeof(float);
+  *tickets = reinterpret_cast<int*>(addr[dev] + kStaticWsBytes);
+  *n_tickets = kStaticTickets;
+  return 0;
+}
+
 int* device_status_ptr() {
   static int* ptr[64] = {nullptr};
   int dev = 0;

@@ -70,6 +70,9 @@ int gemm_plan(GemmPlan& p, const char** why);
 cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s);
 // fp32 elements of stream-K workspace a planned GEMM needs (0: data-parallel only).
 size_t gemm_ws_floats(const GemmPlan& p);
+// The fixed stream-K scratch of the current device (partials, then tickets) and its
+// capacity; returns 0, or -1 with `why` set when its address cannot be obtained.
+int gemm_static_scratch(float** ws, size_t* ws_floats, int** tickets, int* n_tickets, const char** why);
 int* device_status_ptr();  // device address of the shared status word
 int num_sms();
 // 2-D fp16 tensor map: [rows, cols] with row stride ld elements, box 64 x box_rows,
