@@ -257,12 +257,16 @@ class Trace:
 
 
 def denoise(cfg, weights, state, t: float, s: int, S_units: Sequence[int], cache: Dict,
-            class_ids=None, ctx=None, trace: Optional[Trace] = None) -> np.ndarray:
+            class_ids=None, ctx=None, trace: Optional[Trace] = None,
+            active_units: Optional[Sequence[bool]] = None) -> np.ndarray:
     """One denoiser evaluation at step s (1-based) under lifetimes S_units.
 
     ``cache`` maps unit index -> stored Delta and is updated in place: an active unit
     (s <= S_u) computes Delta_{u,s} and refreshes its entry, a frozen unit (s > S_u)
     adds the entry written at its last active step.  Units are visited in graph order.
+    ``active_units``, when given, replaces the lifetime rule (unit u is active iff
+    active_units[u]):
+    the input-aware policy of App. B.1 chooses the active set per step.
     """
     h = stem(cfg, weights, state, t, class_ids)
     c = conditioning(cfg, weights, t, class_ids)
@@ -274,7 +278,7 @@ def denoise(cfg, weights, state, t: float, s: int, S_units: Sequence[int], cache
             h = skip_combine(weights, j, h, skips.pop())
         for kind in cfg.branches:
             h_in = h
-            if s <= S_units[u]:
+            if (active_units[u] if active_units is not None else s <= S_units[u]):
                 delta = branch(cfg, weights, b, kind, h, c, ctx)
                 cache[u] = delta
                 h = (h + delta).astype(F32)
