@@ -42,6 +42,9 @@ def parse():
                     help="also time one trajectory at 100/50/33%% budgets (adds key 'budget_sweep')")
     ap.add_argument("--ablation", action="store_true",
                     help="also time the execution modes of Table tab:kernel (adds key 'ablation')")
+    ap.add_argument("--policies", action="store_true",
+                    help="also time the static schedule against the activation-drift policy of "
+                         "App. B.1 at the same budget (adds key 'policies')")
     return ap.parse_args()
 
 
@@ -264,7 +267,10 @@ def run_native(args):
                 "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
                 "frac": round(achieved / peaks["bf16_sus"], 4),
                 "peak_source": f"{peaks['source']} bf16 sustained x 1 (fp16 and bf16 share the "
-                               "kind::f16 dense rate)", "traffic": None,
+                               "kind::f16 dense rate)", "traffic": gemm_traffic(cfg, T, args.budget),
+                "traffic_unit": "DRAM bytes per launch (ncu launch list in profiles/, averaged over "
+                                "the step's GEMM launches)",
+                "algorithmic_bytes_per_launch": round(gemm["bytes"] / gemm["launches"]),
                 "launches_per_trajectory": gemm["launches"],
                 "share_of_step": round(gemm["ms"] / tot_ms, 3)}
     fz = by_kernel.get("frozen_run")
@@ -314,6 +320,10 @@ def run_native(args):
     if args.ablation:
         ablation = run_ablation(binding, model, cfg, T, weights, sched, xs, out, cls, ctx, stream)
 
+    policies = None
+    if args.policies:
+        policies = run_policies(binding, model, cfg, T, xs, out, cls, ctx, stream)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(cfg, T, weights, inp, sched, n_steps=8)
@@ -336,7 +346,7 @@ def run_native(args):
                    "cache_gb": round(info["cache_bytes"] / 2 ** 30, 2), "setup": setup_t},
         "roofline": roofline, "step_roofline": step_roof, "kernels": kernels,
         "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(gpu_launches),
-        "ablation": ablation, "budget_sweep": sweep,
+        "ablation": ablation, "budget_sweep": sweep, "policies": policies,
         "clocks": clk.summary(),
     }
     if rank == 0:
@@ -418,6 +428,59 @@ def run_ablation(binding, model, cfg, T, weights, sched, xs, out, cls, ctx, stre
     for r in rows:
         r["speedup_vs_eager_full"] = round(base / r["trajectory_ms"], 3)
     return rows
+
+
+def run_policies(binding, model, cfg, T, xs, out, cls, ctx, stream):
+    """Latency side of Table tab:input-aware: whole trajectories under the static schedule
+    and under the causal activation-drift policy (same per-step active counts; drift
+    reductions, host routing after every step, graph lookup and eager fallback included).
+    Two trajectories each after one warm-up trajectory, CUDA events on the stream."""
+    import torch
+    from paper_2609_29505_gb300.synth import timestep
+    rows = {}
+    for name, pol in (("static", binding.POLICY_STATIC), ("drift", binding.POLICY_DRIFT)):
+        model.set_policy(pol)
+        i0 = model.info()
+        times = []
+        for rep in range(3):  # the first pass warms the policy up
+            model.reset()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for s in range(1, T + 1):
+                model.step(xs[s - 1], out, timestep(cfg, s, T), s, class_ids=cls, ctx=ctx, stream=stream)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if rep:
+                times.append(e0.elapsed_time(e1))
+        i1 = model.info()
+        ms = sum(times) / len(times)
+        rows[name] = {"trajectory_ms": round(ms, 2), "steps_per_s": round(T / (ms / 1e3), 3)}
+        if pol == binding.POLICY_DRIFT:
+            rows[name]["graph_steps"] = int(i1["graph_steps"] - i0["graph_steps"])
+            rows[name]["eager_steps"] = int(i1["eager_steps"] - i0["eager_steps"])
+    model.set_policy(binding.POLICY_STATIC)
+    rows["drift_slowdown"] = round(rows["drift"]["trajectory_ms"] / rows["static"]["trajectory_ms"], 3)
+    return rows
+
+
+def gemm_traffic(cfg, T, budget):
+    """DRAM bytes per GEMM launch (read + write, averaged over the step's GEMM launches) from
+    the committed ncu launch list of this workload, or None when the workload differs or the
+    GEMM sources changed since the counters were taken."""
+    import hashlib
+    import re
+    path = os.path.join(ROOT, "profiles", "launches_llada_b4_n1024_T64_budget50.md")
+    if cfg.name != "llada" or T != 64 or abs(budget - 0.5) > 1e-9 or not os.path.exists(path):
+        return None
+    m = re.search(r"traffic_bytes_per_launch: (\d+) sources: ([0-9a-f]{16})", open(path).read())
+    if not m:
+        return None
+    h = hashlib.sha256()
+    for f in ("gemm.cu", "common.cuh"):
+        with open(os.path.join(ROOT, "paper_2609_29505_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return int(m.group(1)) if h.hexdigest()[:16] == m.group(2) else None
 
 
 def workload_name(cfg, T, budget):

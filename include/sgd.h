@@ -162,6 +162,10 @@ typedef struct {
   size_t cache_bytes;   /* device bytes of the per-unit update caches (fp16)      */
   size_t workspace_bytes;
   size_t weight_bytes;  /* device bytes of the library's fp16 projection weights  */
+  int policy;           /* SGD_POLICY_STATIC or SGD_POLICY_DRIFT                  */
+  int n_groups;         /* scheduled (atomic) groups of the current schedule      */
+  int64_t graph_steps;  /* drift policy: steps replayed from the graph library    */
+  int64_t eager_steps;  /* drift policy: steps run op by op (pattern not in it)   */
 } sgd_info;
 
 typedef struct sgd_ctx sgd_ctx;
@@ -226,7 +230,8 @@ SGD_API int sgd_step_host_async(sgd_ctx* ctx, const void* state_in_host, void* o
 /* sgd_host_wait — wait until every output copy queued by sgd_step_host_async is done. */
 SGD_API int sgd_host_wait(sgd_ctx* ctx);
 
-/* sgd_get_active_mask — mask_host[u] = 1 iff unit u is evaluated at `step` (1..T). */
+/* sgd_get_active_mask — mask_host[u] = 1 iff unit u is evaluated at `step` (1..T).  Under
+ * the drift policy: the mask step `step` ran with (steps run since the last reset). */
 SGD_API int sgd_get_active_mask(const sgd_ctx* ctx, int step, uint8_t* mask_host, int n_units);
 
 /* sgd_get_info — sizes and schedule statistics. */
@@ -246,6 +251,35 @@ SGD_API int sgd_get_info(const sgd_ctx* ctx, sgd_info* info);
  */
 enum { SGD_EXEC_JAGGED_GRAPH = 0, SGD_EXEC_EAGER = 1, SGD_EXEC_PADDED_GRAPH = 2 };
 SGD_API int sgd_set_exec_mode(sgd_ctx* ctx, int mode);
+
+/*
+ * Active-set policies:
+ *   SGD_POLICY_STATIC  default: unit u is active at step s iff s <= S_u (Algorithm 2).
+ *   SGD_POLICY_DRIFT   the causal activation-drift baseline of App. B.1: after step s-1
+ *                      the library has the lagged drift of every scheduled group's input,
+ *                      d_g = ||h_{s-1} - h_{s-2}||_2 / (||h_{s-1}||_2 + 1e-8) (the residual
+ *                      stream entering the group's first branch, over the whole batch),
+ *                      and step s runs the m_s groups with the largest drift, m_s being the
+ *                      static schedule's active count at s (ties to the lower group
+ *                      index, groups numbered by their first unit).  Step 1 is full; at
+ *                      step 2 no lagged drift exists yet and the m_2 lowest-indexed groups
+ *                      run.  A frozen unit adds the update of its last active step, so
+ *                      every active unit stores its update.  Each step s >= 3 waits on the
+ *                      host for step s-1's drift sums (the routing is on the host, as in
+ *                      the paper); a step whose active set is one of the static schedule's
+ *                      patterns replays that pattern's graph, any other runs op by op.
+ *                      Needs SGD_EXEC_JAGGED_GRAPH or SGD_EXEC_EAGER.
+ * Changing the policy resets the trajectory.
+ */
+enum { SGD_POLICY_STATIC = 0, SGD_POLICY_DRIFT = 1 };
+SGD_API int sgd_set_policy(sgd_ctx* ctx, int policy);
+
+/*
+ * sgd_get_drift — the lagged drifts the drift policy ranked to choose step `step`'s
+ * active set, drift_host[g] for the n_groups groups (0 at steps 1 and 2).  Valid for
+ * steps run since the last reset; SGD_ERR_STATE otherwise or under the static policy.
+ */
+SGD_API int sgd_get_drift(const sgd_ctx* ctx, int step, double* drift_host, int n_groups);
 
 /* sgd_reset — start a new trajectory: the next step must be 1 (caches invalidated). */
 SGD_API int sgd_reset(sgd_ctx* ctx);

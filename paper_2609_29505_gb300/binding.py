@@ -50,8 +50,10 @@ EXPORTED = [
     "sgd_compile_schedule", "sgd_step_profile", "sgd_sampler_update", "sgd_kernel_gemm",
     "sgd_kernel_attention", "sgd_kernel_norm", "sgd_kernel_frozen_run", "sgd_kernel_status",
     "sgd_set_exec_mode", "sgd_step_host_async", "sgd_host_wait", "sgd_kernel_gemm_static_ws",
+    "sgd_set_policy", "sgd_get_drift",
 ]
 EXEC_JAGGED_GRAPH, EXEC_EAGER, EXEC_PADDED_GRAPH = 0, 1, 2
+POLICY_STATIC, POLICY_DRIFT = 0, 1
 
 
 class sgd_model_desc(C.Structure):
@@ -83,7 +85,9 @@ class sgd_cond(C.Structure):
 class sgd_info(C.Structure):
     _fields_ = [("n_units", C.c_int), ("n_patterns", C.c_int), ("n_graphs", C.c_int),
                 ("T", C.c_int), ("layer_steps", C.c_int64), ("cache_bytes", C.c_size_t),
-                ("workspace_bytes", C.c_size_t), ("weight_bytes", C.c_size_t)]
+                ("workspace_bytes", C.c_size_t), ("weight_bytes", C.c_size_t),
+                ("policy", C.c_int), ("n_groups", C.c_int), ("graph_steps", C.c_int64),
+                ("eager_steps", C.c_int64)]
 
 
 class sgd_op_record(C.Structure):
@@ -135,6 +139,8 @@ def lib() -> C.CDLL:
             "sgd_set_exec_mode": (i, [vp, i]),
             "sgd_step_host_async": (i, [vp, vp, vp, f, vp, vp, i, vp]),
             "sgd_host_wait": (i, [vp]),
+            "sgd_set_policy": (i, [vp, i]),
+            "sgd_get_drift": (i, [vp, i, vp, i]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -338,6 +344,17 @@ class Denoiser:
 
     def set_exec_mode(self, mode: int):
         check(lib().sgd_set_exec_mode(self.handle, mode), "sgd_set_exec_mode")
+
+    def set_policy(self, policy: int):
+        """POLICY_STATIC (lifetimes) or POLICY_DRIFT (the input-aware baseline of App. B.1)."""
+        check(lib().sgd_set_policy(self.handle, policy), "sgd_set_policy")
+
+    def drift(self, step: int) -> np.ndarray:
+        """Lagged drifts the drift policy ranked to choose `step`'s active groups."""
+        n = self.info()["n_groups"]
+        d = np.zeros(n, np.float64)
+        check(lib().sgd_get_drift(self.handle, step, d.ctypes.data, n), "sgd_get_drift")
+        return d
 
     def check_device(self, stream=None):
         return check(lib().sgd_check_device(self.handle, _stream(stream)), "sgd_check_device")

@@ -179,9 +179,28 @@ struct sgd_ctx {
   cudaEvent_t ev_done[2] = {nullptr, nullptr};
   cudaEvent_t ev_copied[2] = {nullptr, nullptr};
   int async_slot = 0;
+  // input-aware (drift) policy, App. B.1
+  int policy = SGD_POLICY_STATIC;
+  int n_groups = 0;
+  std::vector<int> group_of_unit;    // group index (groups numbered by their first unit)
+  std::vector<uint8_t> group_start;  // 1 for the first unit of each group
+  std::vector<int> m_of_step;        // static active-group count at steps 1..T
+  float* snap = nullptr;             // [G][M d] fp32: each group's input at the last step
+  float* drift_part = nullptr;       // [G][kDriftBlocks][2]
+  double* drift_sums = nullptr;      // [G][2]: sum (h - snap)^2, sum h^2
+  double* drift_host = nullptr;      // pinned copy of drift_sums
+  size_t drift_alloc_groups = 0;
+  cudaEvent_t ev_drift = nullptr;    // recorded after the copy of a step's drift sums
+  std::map<std::vector<uint8_t>, int> drift_graph_of;            // library: pattern -> graph
+  std::map<std::vector<uint8_t>, std::vector<Op>> drift_eager;   // patterns outside it
+  std::vector<std::vector<double>> drift_used;  // [T + 1]: drifts ranked at each step
+  std::vector<std::vector<uint8_t>> mask_used;  // [T + 1]: unit mask each step ran
+  int64_t graph_steps = 0, eager_steps = 0;
 
   ~sgd_ctx() {
     if (copy_stream) cudaStreamSynchronize(copy_stream);
+    if (ev_drift) cudaEventDestroy(ev_drift);
+    if (drift_host) cudaFreeHost(drift_host);
     for (int i = 0; i < 2; ++i) {
       if (ev_done[i]) cudaEventDestroy(ev_done[i]);
       if (ev_copied[i]) cudaEventDestroy(ev_copied[i]);
@@ -513,6 +532,20 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
     }
     for (int k = 0; k < c->nbr; ++k, ++u) {
       const int kind = d.block == SGD_BLOCK_XATTN ? k : (k == 0 ? 0 : 2);
+      if (c->policy == SGD_POLICY_DRIFT && c->group_start[u]) {
+        // App. B.1: lagged drift of the group's input (the stream entering its first branch)
+        flush_run(c, ops, run, run_first);
+        const int g = c->group_of_unit[u];
+        DriftParams dp{c->h, c->snap + static_cast<size_t>(g) * M * D, static_cast<int64_t>(M) * D,
+                       c->drift_part + static_cast<size_t>(g) * 2 * kDriftBlocks};
+        Op op;
+        op.name = "g" + std::to_string(g) + ".drift";
+        op.kernel = SGD_KERNEL_SMALL;
+        op.flops = 4.0 * M * D;
+        op.bytes = 12.0 * M * D;
+        op.run = [dp](cudaStream_t s) { return drift_launch(dp, s); };
+        ops.push_back(std::move(op));
+      }
       if (active[u]) {
         flush_run(c, ops, run, run_first);
         if ((rc = build_branch(c, ops, b, kind, write[u] != 0, u))) return rc;
@@ -541,6 +574,18 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
     }
   }
   flush_run(c, ops, run, run_first);
+  if (c->policy == SGD_POLICY_DRIFT) {
+    const float* part = c->drift_part;
+    double* sums = c->drift_sums;
+    const int G = c->n_groups;
+    Op op;
+    op.name = "drift.reduce";
+    op.kernel = SGD_KERNEL_SMALL;
+    op.flops = 0;
+    op.bytes = 8.0 * G * kDriftBlocks;
+    op.run = [part, G, sums](cudaStream_t s) { return drift_reduce_launch(part, G, sums, s); };
+    ops.push_back(std::move(op));
+  }
   // head
   void* const* out_slot = reinterpret_cast<void* const*>(&c->slot->out);
   if (d.head == SGD_HEAD_IDENTITY) {
@@ -805,6 +850,8 @@ void drop_graphs(sgd_ctx* c) {
   c->execs.clear();
   c->graphs.clear();
   c->programs.clear();
+  c->drift_graph_of.clear();
+  c->drift_eager.clear();
   c->scheduled = false;
 }
 
@@ -921,10 +968,76 @@ int sgd_compile_schedule(int T, int n_units, const int32_t* lifetimes, const int
   return SGD_OK;
 }
 
+// Capture `ops` into a graph; the program, graph and executable are kept in the context.
+static int capture_program(sgd_ctx* c, std::vector<Op>&& ops, int* gid) {
+  cudaGraph_t g = nullptr;
+  CUDA_TRY(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeRelaxed));
+  int rc = run_ops(ops, c->cap_stream);
+  cudaError_t ce = cudaStreamEndCapture(c->cap_stream, &g);
+  if (rc) {
+    if (g) cudaGraphDestroy(g);
+    return rc;
+  }
+  if (ce != cudaSuccess) return fail(SGD_ERR_CUDA, std::string("graph capture: ") + cudaGetErrorString(ce));
+  cudaGraphExec_t ex = nullptr;
+  ce = cudaGraphInstantiate(&ex, g, 0);
+  if (ce != cudaSuccess) {
+    cudaGraphDestroy(g);
+    return fail(SGD_ERR_CUDA, std::string("graph instantiate: ") + cudaGetErrorString(ce));
+  }
+  *gid = static_cast<int>(c->graphs.size());
+  c->graphs.push_back(g);
+  c->execs.push_back(ex);
+  c->programs.push_back(std::move(ops));
+  return SGD_OK;
+}
+
+// Buffers of the drift policy: every unit's cache (any active step may be a unit's last),
+// the per-group input snapshots, partial and final drift sums, and their host copy.
+static int ensure_drift_buffers(sgd_ctx* c) {
+  int rc;
+  for (int u = 0; u < c->U; ++u)
+    if (!c->cache[u] && (rc = c->alloc(&c->cache[u], static_cast<size_t>(c->M) * c->d.d, &c->cache_bytes)))
+      return rc;
+  const size_t G = static_cast<size_t>(c->n_groups);
+  if (c->drift_alloc_groups < G) {
+    const size_t n = static_cast<size_t>(c->M) * c->d.d;
+    if ((rc = c->alloc(&c->snap, G * n, &c->ws_bytes)) ||
+        (rc = c->alloc(&c->drift_part, G * 2 * kDriftBlocks, &c->ws_bytes)) ||
+        (rc = c->alloc(&c->drift_sums, G * 2, &c->ws_bytes)))
+      return rc;
+    CUDA_TRY(cudaMemset(c->snap, 0, G * n * sizeof(float)));
+    if (c->drift_host) cudaFreeHost(c->drift_host);
+    c->drift_host = nullptr;
+    CUDA_TRY(cudaHostAlloc(reinterpret_cast<void**>(&c->drift_host), G * 2 * sizeof(double), cudaHostAllocDefault));
+    c->drift_alloc_groups = G;
+  }
+  if (!c->ev_drift) CUDA_TRY(cudaEventCreateWithFlags(&c->ev_drift, cudaEventDisableTiming));
+  return SGD_OK;
+}
+
 static int build_graphs(sgd_ctx* c) {
   const int T = c->T;
   int rc;
   drop_graphs(c);
+  if (c->policy == SGD_POLICY_DRIFT) {
+    // the graph library: one graph per active set of the static schedule, in which every
+    // active unit stores its update and every group's drift is reduced
+    if ((rc = ensure_drift_buffers(c))) return rc;
+    for (const auto& pat : c->patterns) {
+      std::vector<Op> ops;
+      if ((rc = build_program(c, pat, pat, ops)) || (rc = ensure_sk_ws(c))) return rc;
+      int gid = -1;
+      if ((rc = capture_program(c, std::move(ops), &gid))) return rc;
+      c->drift_graph_of[pat] = gid;
+    }
+    c->graph_of_step.assign(T + 1, -1);
+    c->drift_used.assign(T + 1, {});
+    c->mask_used.assign(T + 1, {});
+    c->last_step = 0;
+    c->scheduled = true;
+    return SGD_OK;
+  }
   // graph variants: (pattern, cache-store set); the store set is non-empty only at steps
   // s = S_u < T, so each such step gets its own variant.
   std::map<std::pair<int, int>, int> key_to_graph;
@@ -941,25 +1054,8 @@ static int build_graphs(sgd_ctx* c) {
     for (int u = 0; u < c->U; ++u) write[u] = (c->S[u] == s && s < T) ? 1 : 0;
     std::vector<Op> ops;
     if ((rc = build_program(c, c->patterns[pid], write, ops)) || (rc = ensure_sk_ws(c))) return rc;
-    cudaGraph_t g = nullptr;
-    CUDA_TRY(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeRelaxed));
-    rc = run_ops(ops, c->cap_stream);
-    cudaError_t ce = cudaStreamEndCapture(c->cap_stream, &g);
-    if (rc) {
-      if (g) cudaGraphDestroy(g);
-      return rc;
-    }
-    if (ce != cudaSuccess) return fail(SGD_ERR_CUDA, std::string("graph capture: ") + cudaGetErrorString(ce));
-    cudaGraphExec_t ex = nullptr;
-    ce = cudaGraphInstantiate(&ex, g, 0);
-    if (ce != cudaSuccess) {
-      cudaGraphDestroy(g);
-      return fail(SGD_ERR_CUDA, std::string("graph instantiate: ") + cudaGetErrorString(ce));
-    }
-    const int gid = static_cast<int>(c->graphs.size());
-    c->graphs.push_back(g);
-    c->execs.push_back(ex);
-    c->programs.push_back(std::move(ops));
+    int gid = -1;
+    if ((rc = capture_program(c, std::move(ops), &gid))) return rc;
     key_to_graph[{pid, key2}] = gid;
     c->graph_of_step[s] = gid;
   }
@@ -978,6 +1074,29 @@ int sgd_set_schedule(sgd_ctx* c, int T, int n_units, const int32_t* lifetimes, c
   c->S.assign(lifetimes, lifetimes + n_units);
   c->groups.assign(groups, groups + n_units);
   compile_patterns(T, n_units, lifetimes, c->pattern_of_step, c->writes, c->patterns);
+  // groups numbered by their first unit; the static schedule's active-group count per step
+  {
+    std::map<int32_t, int> index;
+    c->group_of_unit.assign(n_units, 0);
+    c->group_start.assign(n_units, 0);
+    std::vector<int32_t> life;
+    for (int u = 0; u < n_units; ++u) {
+      auto it = index.find(groups[u]);
+      if (it == index.end()) {
+        const int g = static_cast<int>(index.size());
+        index[groups[u]] = g;
+        c->group_start[u] = 1;
+        life.push_back(lifetimes[u]);
+        c->group_of_unit[u] = g;
+      } else {
+        c->group_of_unit[u] = it->second;
+      }
+    }
+    c->n_groups = static_cast<int>(index.size());
+    c->m_of_step.assign(T + 1, 0);
+    for (int s = 1; s <= T; ++s)
+      for (int32_t l : life) c->m_of_step[s] += l >= s ? 1 : 0;
+  }
   // caches only for units that are ever frozen
   for (int u = 0; u < c->U; ++u)
     if (c->S[u] < T && !c->cache[u]) {
@@ -992,6 +1111,8 @@ int sgd_set_exec_mode(sgd_ctx* c, int mode) {
   if (!c) return fail(SGD_ERR_ARG, "null context");
   if (mode < SGD_EXEC_JAGGED_GRAPH || mode > SGD_EXEC_PADDED_GRAPH)
     return fail(SGD_ERR_ARG, "unknown execution mode");
+  if (mode == SGD_EXEC_PADDED_GRAPH && c->policy == SGD_POLICY_DRIFT)
+    return fail(SGD_ERR_STATE, "the drift policy runs with jagged graphs or eagerly, not padded graphs");
   int rc;
   if (mode == SGD_EXEC_PADDED_GRAPH && !c->h_pad &&
       (rc = c->alloc(&c->h_pad, static_cast<size_t>(c->M) * c->d.d, &c->ws_bytes)))
@@ -1006,12 +1127,95 @@ int sgd_set_exec_mode(sgd_ctx* c, int mode) {
   return SGD_OK;
 }
 
+int sgd_set_policy(sgd_ctx* c, int policy) {
+  if (!c) return fail(SGD_ERR_ARG, "null context");
+  if (policy != SGD_POLICY_STATIC && policy != SGD_POLICY_DRIFT) return fail(SGD_ERR_ARG, "unknown policy");
+  if (policy == SGD_POLICY_DRIFT && c->exec_mode == SGD_EXEC_PADDED_GRAPH)
+    return fail(SGD_ERR_STATE, "the drift policy runs with jagged graphs or eagerly, not padded graphs");
+  const bool rebuild = policy != c->policy;
+  c->policy = policy;
+  if (rebuild && c->scheduled) {
+    CUDA_TRY(cudaSetDevice(c->device));
+    int rc;
+    if ((rc = build_graphs(c))) return rc;
+  }
+  c->last_step = 0;
+  return SGD_OK;
+}
+
+namespace {
+
+// App. B.1 routing for step `step`: the active groups (step 1 all, step 2 the m_2 lowest,
+// later the m_s with the largest lagged drift of step - 1, ties to the lower index),
+// recorded with the drifts they were ranked by; returns the unit mask.
+int drift_route(sgd_ctx* c, int step, std::vector<uint8_t>& mask) {
+  const int G = c->n_groups;
+  const int m = c->m_of_step[step];
+  if (step == 1) {  // a new trajectory: forget the previous one's records
+    for (auto& v : c->drift_used) v.clear();
+    for (auto& v : c->mask_used) v.clear();
+  }
+  std::vector<double> dv(G, 0.0);
+  std::vector<int> order(G);
+  for (int g = 0; g < G; ++g) order[g] = g;
+  if (step >= 3) {
+    CUDA_TRY(cudaEventSynchronize(c->ev_drift));  // step - 1's sums are on the host
+    for (int g = 0; g < G; ++g)
+      dv[g] = std::sqrt(c->drift_host[2 * g]) / (std::sqrt(c->drift_host[2 * g + 1]) + 1e-8);
+    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return dv[a] > dv[b]; });
+  }
+  std::vector<uint8_t> on(G, 0);
+  for (int i = 0; i < (step == 1 ? G : m); ++i) on[order[i]] = 1;
+  mask.assign(c->U, 0);
+  for (int u = 0; u < c->U; ++u) mask[u] = on[c->group_of_unit[u]];
+  c->drift_used[step] = dv;
+  c->mask_used[step] = mask;
+  return SGD_OK;
+}
+
+// One step under the drift policy: route, replay the library graph of the chosen active set
+// or run its op list eagerly, then queue the copy of this step's drift sums to the host.
+int drift_step(sgd_ctx* c, int step, cudaStream_t s) {
+  std::vector<uint8_t> mask;
+  int rc;
+  if ((rc = drift_route(c, step, mask))) return rc;
+  auto it = c->drift_graph_of.find(mask);
+  if (it != c->drift_graph_of.end() && c->exec_mode == SGD_EXEC_JAGGED_GRAPH) {
+    CUDA_TRY(cudaGraphLaunch(c->execs[it->second], s));
+    ++c->graph_steps;
+  } else {
+    if (it != c->drift_graph_of.end()) {
+      if ((rc = run_ops(c->programs[it->second], s))) return rc;
+    } else {
+      auto e = c->drift_eager.find(mask);
+      if (e == c->drift_eager.end()) {
+        std::vector<Op> ops;
+        if ((rc = build_program(c, mask, mask, ops)) || (rc = ensure_sk_ws(c))) return rc;
+        e = c->drift_eager.emplace(mask, std::move(ops)).first;
+      }
+      if ((rc = run_ops(e->second, s))) return rc;
+    }
+    ++c->eager_steps;
+  }
+  CUDA_TRY(cudaMemcpyAsync(c->drift_host, c->drift_sums, sizeof(double) * 2 * c->n_groups,
+                           cudaMemcpyDeviceToHost, s));
+  CUDA_TRY(cudaEventRecord(c->ev_drift, s));
+  return SGD_OK;
+}
+
+}  // namespace
+
 int sgd_step(sgd_ctx* c, const void* in, void* out, float t, const sgd_cond* cond, int step,
              void* stream) {
   int rc = check_step_args(c, in, out, cond, step);
   if (rc) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if ((rc = prepare_step(c, in, out, t, cond, step, s))) return rc;
+  if (c->policy == SGD_POLICY_DRIFT) {
+    if ((rc = drift_step(c, step, s))) return rc;
+    c->last_step = step == c->T ? 0 : step;
+    return SGD_OK;
+  }
   if (c->exec_mode == SGD_EXEC_EAGER) {
     if ((rc = run_ops(c->programs[c->graph_of_step[step]], s))) return rc;  // one launch per op
   } else {
@@ -1025,6 +1229,7 @@ int sgd_step_profile(sgd_ctx* c, const void* in, void* out, float t, const sgd_c
                      void* stream, sgd_op_record* rec, int max_rec, int* n_rec) {
   int rc = check_step_args(c, in, out, cond, step);
   if (rc) return rc;
+  if (c->policy != SGD_POLICY_STATIC) return fail(SGD_ERR_STATE, "profiled steps need the static policy");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if ((rc = prepare_step(c, in, out, t, cond, step, s))) return rc;
   const std::vector<Op>& ops = c->programs[c->graph_of_step[step]];
@@ -1138,8 +1343,26 @@ int sgd_get_active_mask(const sgd_ctx* c, int step, uint8_t* mask, int n_units) 
   if (!c->scheduled) return fail(SGD_ERR_STATE, "no schedule installed");
   if (step < 1 || step > c->T) return fail(SGD_ERR_ARG, "step outside [1, T]");
   if (n_units != c->U) return fail(SGD_ERR_ARG, "n_units mismatch");
+  if (c->policy == SGD_POLICY_DRIFT) {
+    if (static_cast<size_t>(step) >= c->mask_used.size() || c->mask_used[step].empty())
+      return fail(SGD_ERR_STATE, "step " + std::to_string(step) + " has not run since the last reset");
+    for (int u = 0; u < n_units; ++u) mask[u] = c->mask_used[step][u];
+    return SGD_OK;
+  }
   const auto& m = c->patterns[c->pattern_of_step[step - 1]];
   for (int u = 0; u < n_units; ++u) mask[u] = m[u];
+  return SGD_OK;
+}
+
+int sgd_get_drift(const sgd_ctx* c, int step, double* drift, int n_groups) {
+  if (!c || !drift) return fail(SGD_ERR_ARG, "null argument");
+  if (c->policy != SGD_POLICY_DRIFT) return fail(SGD_ERR_STATE, "the static policy records no drift");
+  if (!c->scheduled) return fail(SGD_ERR_STATE, "no schedule installed");
+  if (step < 1 || step > c->T) return fail(SGD_ERR_ARG, "step outside [1, T]");
+  if (n_groups != c->n_groups) return fail(SGD_ERR_ARG, "n_groups mismatch");
+  if (static_cast<size_t>(step) >= c->drift_used.size() || c->drift_used[step].empty())
+    return fail(SGD_ERR_STATE, "step " + std::to_string(step) + " has not run since the last reset");
+  for (int g = 0; g < n_groups; ++g) drift[g] = c->drift_used[step][g];
   return SGD_OK;
 }
 
@@ -1150,6 +1373,10 @@ int sgd_get_info(const sgd_ctx* c, sgd_info* info) {
   info->n_patterns = static_cast<int>(c->patterns.size());
   info->n_graphs = static_cast<int>(c->graphs.size());
   info->T = c->scheduled ? c->T : 0;
+  info->policy = c->policy;
+  info->n_groups = c->scheduled ? c->n_groups : 0;
+  info->graph_steps = c->graph_steps;
+  info->eager_steps = c->eager_steps;
   int64_t ls = 0;
   if (c->scheduled)
     for (int u = 0; u < c->U; ++u) ls += c->S[u];
@@ -1163,6 +1390,8 @@ int sgd_get_info(const sgd_ctx* c, sgd_info* info) {
 int sgd_reset(sgd_ctx* c) {
   if (!c) return fail(SGD_ERR_ARG, "null context");
   c->last_step = 0;
+  for (auto& v : c->drift_used) v.clear();
+  for (auto& v : c->mask_used) v.clear();
   // a GEMM that stopped on an expired wait may have left stream-K tickets behind
   if (c->sk_cnt) {
     CUDA_TRY(cudaSetDevice(c->device));

@@ -178,6 +178,65 @@ __global__ void __launch_bounds__(256) norm_warp_kernel(const NormParams p) {
   }
 }
 
+// Lagged drift of one group's input (App. B.1): each of kDriftBlocks blocks strides over
+// float4s of h (two per iteration, to keep more loads in flight), accumulating (h - snap)^2
+// and h^2 per thread in fp32, reduces them in a fixed tree and writes its pair; snap takes
+// the current h for the next step.  The grid size is fixed, so the summation order (and
+// the result) is the same on every run.
+__device__ __forceinline__ void drift_acc(const float4 x, const float4 y, float& dd, float& hh) {
+  const float a = x.x - y.x, b = x.y - y.y, c = x.z - y.z, d = x.w - y.w;
+  dd += (a * a + b * b) + (c * c + d * d);
+  hh += (x.x * x.x + x.y * x.y) + (x.z * x.z + x.w * x.w);
+}
+
+__global__ void __launch_bounds__(256) drift_kernel(const DriftParams p) {
+  __shared__ float red[8];
+  const int64_t nv = p.n >> 2;
+  const float4* h4 = reinterpret_cast<const float4*>(p.h);
+  float4* s4 = reinterpret_cast<float4*>(p.snap);
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  float dd = 0.f, hh = 0.f;
+  int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  for (; i + stride < nv; i += 2 * stride) {
+    const float4 x0 = h4[i], y0 = s4[i], x1 = h4[i + stride], y1 = s4[i + stride];
+    drift_acc(x0, y0, dd, hh);
+    drift_acc(x1, y1, dd, hh);
+    s4[i] = x0;
+    s4[i + stride] = x1;
+  }
+  if (i < nv) {
+    const float4 x = h4[i], y = s4[i];
+    drift_acc(x, y, dd, hh);
+    s4[i] = x;
+  }
+  dd = block_sum(dd, red);
+  hh = block_sum(hh, red);
+  if (threadIdx.x == 0) {
+    p.partial[2 * blockIdx.x] = dd;
+    p.partial[2 * blockIdx.x + 1] = hh;
+  }
+}
+
+// One warp per group: lane l sums partials l, l + 32, ... in double, then a fixed xor tree
+// combines the lanes (the order is the same on every run).
+__global__ void drift_reduce_kernel(const float* partials, double* sums) {
+  const float* p = partials + static_cast<size_t>(blockIdx.x) * 2 * kDriftBlocks;
+  double dd = 0.0, hh = 0.0;
+  for (int b = threadIdx.x; b < kDriftBlocks; b += 32) {
+    dd += static_cast<double>(p[2 * b]);
+    hh += static_cast<double>(p[2 * b + 1]);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    dd += __shfl_xor_sync(0xffffffffu, dd, o);
+    hh += __shfl_xor_sync(0xffffffffu, hh, o);
+  }
+  if (threadIdx.x == 0) {
+    sums[2 * blockIdx.x] = dd;
+    sums[2 * blockIdx.x + 1] = hh;
+  }
+}
+
 __global__ void __launch_bounds__(256) frozen_kernel(const __grid_constant__ FrozenParams p) {
   const int64_t n8 = p.n >> 3;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -433,6 +492,16 @@ cudaError_t norm_launch(const NormParams& p, cudaStream_t s) {
     norm_warp_kernel<<<(p.rows + 7) / 8, 256, 0, s>>>(p);
   else
     norm_kernel<<<p.rows, kNormThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t drift_launch(const DriftParams& p, cudaStream_t s) {
+  drift_kernel<<<kDriftBlocks, 256, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t drift_reduce_launch(const float* partials, int n_groups, double* sums, cudaStream_t s) {
+  drift_reduce_kernel<<<n_groups, 32, 0, s>>>(partials, sums);
   return cudaGetLastError();
 }
 

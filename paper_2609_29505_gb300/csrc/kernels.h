@@ -128,6 +128,20 @@ struct FrozenParams {
 };
 cudaError_t frozen_launch(const FrozenParams& p, cudaStream_t s);
 
+// Lagged-drift reduction of the input-aware policy (App. B.1) for one scheduled group:
+// partial[b] = (sum (h - snap)^2, sum h^2) over block b's elements (fp32, fixed order),
+// then snap = h.  n % 4 == 0, 16-byte aligned.  drift_reduce sums each group's kDriftBlocks
+// partials in a fixed order, in double: sums[2 g], sums[2 g + 1].
+constexpr int kDriftBlocks = 1024;
+struct DriftParams {
+  const float* h;
+  float* snap;
+  int64_t n;
+  float* partial;  // [kDriftBlocks][2]
+};
+cudaError_t drift_launch(const DriftParams& p, cudaStream_t s);
+cudaError_t drift_reduce_launch(const float* partials, int n_groups, double* sums, cudaStream_t s);
+
 // Per-step I/O slot (device memory) read by graph kernels.
 struct IoSlot {
   const void* state;
