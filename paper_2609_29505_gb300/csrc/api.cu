@@ -1591,7 +1591,7 @@ int sgd_kernel_gemm_static_ws(const void* A, int lda, const void* B, int ldb, in
 int sgd_kernel_attention(const void* q, int ldq, const void* k, const void* v, int ldkv, void* o,
                          int ldo, int batch, int n_q, int n_kv, int n_heads, int d_head, int impl,
                          void* stream) {
-  if (impl < 0 || impl > 1) return fail(SGD_ERR_ARG, "attention: impl must be 0 or 1");
+  if (impl < 0 || impl > 3) return fail(SGD_ERR_ARG, "attention: impl must be in 0..3");
   AttnPlan plan;
   plan.p = AttnParams{H16(q), ldq, H16(k), H16(v), ldkv, static_cast<f16*>(o), ldo,
                       batch, n_q, n_kv, n_heads, d_head, impl};

@@ -521,6 +521,301 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const __grid_con
   }
 }
 
+// ----------------------------------------------------------------------------
+// attn_pp_kernel: two query tiles per CTA, ping-pong between two softmax warpgroups.
+//
+// One CTA = 256 queries (tiles 0 and 1) of one (sample, head); K/V tiles of 128 keys, shared
+// by both query tiles, through a 2-stage TMA ring.  TMEM holds S_0, S_1 (128 fp32 columns
+// each) and O_0, O_1 (d_h columns each).  Warps 2-5 run the softmax of tile 0, warps 6-9 of
+// tile 1: each reads its S from TMEM (a max pass, then an exp pass), writes P as fp16 pairs
+// over the first 64 columns of the same S, and the MMA warp computes O_t += P_t V from
+// Tensor Memory (A operand in TMEM), so P needs no shared memory.  The MMA warp issues, per
+// key tile j: PV_0(j), S_0(j+1), PV_1(j), S_1(j+1): while one warpgroup runs its softmax,
+// the tensor cores work on the other tile.  tcgen05.mma operations of one thread run in
+// issue order, so S_t(j+1) overwrites P_t(j) only after PV_t(j) has read it.
+// ----------------------------------------------------------------------------
+constexpr int kPpThreads = 320;
+constexpr int kPpBQ = 256;
+
+template <int DH>
+struct PpLayout {
+  static constexpr int kAtoms = DH / 64;
+  static constexpr int kQ = 0;                        // Q tile t: atoms at kQ + (t kAtoms + a) kAtom
+  static constexpr int kKV = 2 * kAtoms * kAtom;      // stage s: K atoms, then V atoms
+  static constexpr int kStage = 2 * kAtoms * kAtom;
+  static constexpr int kBar = kKV + 2 * kStage;
+  static constexpr int kBytes = kBar + 256 + 1024;
+  static constexpr uint32_t kTmemS = 0;               // S_t at columns 128 t
+  static constexpr uint32_t kTmemO = 256;             // O_t at columns 256 + DH t
+  static_assert(kBytes <= 232448, "shared memory");
+};
+
+template <int DH>
+__global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_constant__ AttnTcArgs a) {
+  using L = PpLayout<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L::kBar);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;
+  uint64_t* kv_empty = bars + 3;
+  uint64_t* s_full = bars + 5;   // per query tile
+  uint64_t* p_full = bars + 7;   // per query tile, 4 warps arrive
+  uint64_t* o_done = bars + 9;   // per query tile
+  uint64_t* drain = bars + 11;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qt = blockIdx.x, bh = blockIdx.y;
+  const int b = bh / a.n_heads, h = bh % a.n_heads;
+  const int nt = (a.n_kv + kTcBK - 1) / kTcBK;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&kv_full[i], 1);
+      mbar_init(&kv_empty[i], 1);
+      mbar_init(&s_full[i], 1);
+      mbar_init(&p_full[i], 4);
+      mbar_init(&o_done[i], 1);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&a.tmap_q);
+    tma_prefetch_desc(&a.tmap_k);
+    tma_prefetch_desc(&a.tmap_v);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      mbar_arrive_expect_tx(q_full, 2 * L::kAtoms * kAtom);
+      for (int t = 0; t < 2; ++t)
+        for (int at = 0; at < L::kAtoms; ++at)
+          tma_load_2d(sm + L::kQ + (t * L::kAtoms + at) * kAtom, &a.tmap_q, q_full, h * DH + at * 64,
+                      b * a.n_q + (2 * qt + t) * kTcBQ);
+      int j = 0;
+      for (; j < nt; ++j) {
+        const int s = j & 1;
+        if (!mbar_wait(&kv_empty[s], ((j >> 1) & 1) ^ 1u, abort_flag, a.status, 21)) break;
+        uint8_t* st = sm + L::kKV + s * L::kStage;
+        mbar_arrive_expect_tx(&kv_full[s], 2 * L::kAtoms * kAtom);
+        const int row = b * a.n_kv + j * kTcBK;
+        for (int at = 0; at < L::kAtoms; ++at) {
+          tma_load_2d(st + at * kAtom, &a.tmap_k, &kv_full[s], h * DH + at * 64, row);
+          tma_load_2d(st + (L::kAtoms + at) * kAtom, &a.tmap_v, &kv_full[s], h * DH + at * 64, row);
+        }
+      }
+      if (*abort_flag) {
+        drain_bar(q_full, 0);
+        for (int i = (j > 2 ? j - 2 : 0); i < j; ++i) drain_bar(&kv_full[i & 1], (i >> 1) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc_qk = umma_idesc_f16(kTcBQ, kTcBK);
+      const uint32_t idesc_pv = umma_idesc_f16_bmn(kTcBQ, DH);
+      bool ok = mbar_wait(q_full, 0, abort_flag, a.status, 22);
+      auto issue_qk = [&](int t, int j) {
+        const int s = j & 1;
+        const uint32_t qa = smem_u32(sm + L::kQ + t * L::kAtoms * kAtom);
+        const uint32_t ka = smem_u32(sm + L::kKV + s * L::kStage);
+#pragma unroll
+        for (int ks = 0; ks < DH / 16; ++ks) {
+          const uint32_t off = (ks >> 2) * kAtom + (ks & 3) * 32;
+          umma_f16(tmem + L::kTmemS + t * kTcBK, smem_desc_sw128(qa + off), smem_desc_sw128(ka + off),
+                   idesc_qk, ks > 0 ? 1u : 0u);
+        }
+        umma_commit(&s_full[t]);
+      };
+      auto issue_pv = [&](int t, int j) {
+        const int s = j & 1;
+        const uint32_t va = smem_u32(sm + L::kKV + s * L::kStage + L::kAtoms * kAtom);
+#pragma unroll
+        for (int ks = 0; ks < kTcBK / 16; ++ks) {
+          const uint64_t bd = smem_desc_sw128_mn(va + ks * 2048, kAtom, 1024);
+          umma_f16_ts(tmem + L::kTmemO + t * DH, tmem + L::kTmemS + t * kTcBK + 8 * ks, bd, idesc_pv,
+                      (j > 0 || ks > 0) ? 1u : 0u);
+        }
+        umma_commit(&o_done[t]);
+      };
+      if (ok && (ok = mbar_wait(&kv_full[0], 0, abort_flag, a.status, 23))) {
+        tc_fence_after();
+        issue_qk(0, 0);
+        issue_qk(1, 0);
+      }
+      for (int j = 0; j < nt && ok; ++j) {
+        const uint32_t ph = j & 1;
+        if (!(ok = mbar_wait(&p_full[0], ph, abort_flag, a.status, 24))) break;
+        tc_fence_after();
+        issue_pv(0, j);
+        if (j + 1 < nt) {
+          if (!(ok = mbar_wait(&kv_full[(j + 1) & 1], ((j + 1) >> 1) & 1, abort_flag, a.status, 25))) break;
+          tc_fence_after();
+          issue_qk(0, j + 1);
+        }
+        if (!(ok = mbar_wait(&p_full[1], ph, abort_flag, a.status, 26))) break;
+        tc_fence_after();
+        issue_pv(1, j);
+        umma_commit(&kv_empty[j & 1]);
+        if (j + 1 < nt) issue_qk(1, j + 1);
+      }
+      umma_commit(drain);
+      drain_bar(drain, 0);
+    }
+  } else {
+    const int t = (warp - 2) >> 2;   // query tile of this warpgroup
+    const int q = warp & 3;          // TMEM lane quarter
+    const int row = q * 32 + lane;
+    const uint32_t lane_base = static_cast<uint32_t>(q * 32) << 16;
+    const uint32_t s_col = tmem + lane_base + L::kTmemS + t * kTcBK;
+    const uint32_t o_col = tmem + lane_base + L::kTmemO + t * DH;
+    float m2 = -INFINITY, l = 0.f;
+    bool ok = true;
+    uint32_t r0[16], r1[16];
+    for (int j = 0; j < nt; ++j) {
+      if (!(ok = warp_wait_bar(&s_full[t], j & 1, abort_flag, a.status, 27))) break;
+      tc_fence_after();
+      const int kb = j * kTcBK;
+      const bool whole = kb + kTcBK <= a.n_kv;
+      // pass 1: the tile's row maximum (scores in log2 units)
+      float mx[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) mx[i] = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < kTcBK; c += 32) {
+        tmem_ld16(s_col + c, r0);
+        tmem_ld16(s_col + c + 16, r1);
+        tmem_ld_wait16(r0);
+        tmem_ld_wait16(r1);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float v0 = (whole || kb + c + i < a.n_kv) ? __uint_as_float(r0[i]) * a.scale_log2 : -INFINITY;
+          const float v1 = (whole || kb + c + 16 + i < a.n_kv) ? __uint_as_float(r1[i]) * a.scale_log2 : -INFINITY;
+          mx[i & 7] = fmaxf(mx[i & 7], fmaxf(v0, v1));
+        }
+      }
+      const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      if (j == 0) {
+        m2 = mt;
+      } else if (__any_sync(0xffffffffu, mt > m2 + kRescaleLog2)) {
+        // warp-uniform (the TMEM accesses are .sync.aligned); O_t must hold PV_t(j-1)
+        if (!(ok = warp_wait_bar(&o_done[t], (j - 1) & 1, abort_flag, a.status, 28))) break;
+        tc_fence_after();
+        const float mnew = fmaxf(m2, mt);
+        const float corr = exp2f(m2 - mnew);
+#pragma unroll
+        for (int c = 0; c < DH; c += 16) {
+          tmem_ld16(o_col + c, r0);
+          tmem_ld_wait16(r0);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) r0[i] = __float_as_uint(__uint_as_float(r0[i]) * corr);
+          tmem_st16(o_col + c, r0);
+        }
+        tmem_st_wait();
+        l *= corr;
+        m2 = mnew;
+      }
+      // pass 2: P = exp2(score - m2) as fp16 pairs over columns [0, 64) of this S; the 16
+      // packed columns of scores [c, c + 32) land on scores already read
+      float ls[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ls[i] = 0.f;
+#pragma unroll
+      for (int c = 0; c < kTcBK; c += 32) {
+        tmem_ld16(s_col + c, r0);
+        tmem_ld16(s_col + c + 16, r1);
+        tmem_ld_wait16(r0);
+        tmem_ld_wait16(r1);
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          float p[4];
+          const int c0 = c + 2 * i;
+          p[0] = (whole || kb + c0 < a.n_kv) ? exp2f(__uint_as_float(r0[2 * i]) * a.scale_log2 - m2) : 0.f;
+          p[1] = (whole || kb + c0 + 1 < a.n_kv) ? exp2f(__uint_as_float(r0[2 * i + 1]) * a.scale_log2 - m2) : 0.f;
+          p[2] = (whole || kb + c0 + 16 < a.n_kv) ? exp2f(__uint_as_float(r1[2 * i]) * a.scale_log2 - m2) : 0.f;
+          p[3] = (whole || kb + c0 + 17 < a.n_kv) ? exp2f(__uint_as_float(r1[2 * i + 1]) * a.scale_log2 - m2) : 0.f;
+          ls[i] += (p[0] + p[1]) + (p[2] + p[3]);
+          pk[i] = pack_f16x2(p[0], p[1]);
+          pk[8 + i] = pack_f16x2(p[2], p[3]);
+        }
+        tmem_st16(s_col + c / 2, pk);
+      }
+      l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
+      tmem_st_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[t]);
+    }
+    if (ok && warp_wait_bar(&o_done[t], (nt - 1) & 1, abort_flag, a.status, 29)) {
+      tc_fence_after();
+      const float inv = 1.f / l;
+      const int qrow = (2 * qt + t) * kTcBQ + row;
+      f16* orow = a.o + (static_cast<int64_t>(b) * a.n_q + qrow) * a.ldo + h * DH;
+#pragma unroll
+      for (int c = 0; c < DH; c += 16) {
+        tmem_ld16(o_col + c, r0);
+        tmem_ld_wait16(r0);
+        float f[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(r0[i]) * inv;
+        if (qrow < a.n_q) {
+          reinterpret_cast<uint4*>(orow + c)[0] = pack_f16x8(f);
+          reinterpret_cast<uint4*>(orow + c)[1] = pack_f16x8(f + 8);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+template <int DH>
+cudaError_t launch_pp(const AttnPlan& plan, cudaStream_t s) {
+  using L = PpLayout<DH>;
+  static bool done[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !done[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(attn_pp_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         L::kBytes);
+    if (e != cudaSuccess) return e;
+    done[dev] = true;
+  }
+  const AttnParams& p = plan.p;
+  AttnTcArgs a;
+  memcpy(&a.tmap_q, &plan.tmap_q, sizeof(CUtensorMap));
+  memcpy(&a.tmap_k, &plan.tmap_kv, sizeof(CUtensorMap));
+  memcpy(&a.tmap_v, &plan.tmap_v, sizeof(CUtensorMap));
+  a.o = p.o;
+  a.ldo = p.ldo;
+  a.n_q = p.n_q;
+  a.n_kv = p.n_kv;
+  a.n_heads = p.n_heads;
+  a.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(DH));
+  a.status = device_status_ptr();
+  dim3 grid((p.n_q + kPpBQ - 1) / kPpBQ, p.batch * p.n_heads);
+  attn_pp_kernel<DH><<<grid, kPpThreads, L::kBytes, s>>>(a);
+  return cudaGetLastError();
+}
+
 template <int DH>
 cudaError_t launch_tc(const AttnPlan& plan, cudaStream_t s) {
   using L = TcLayout<DH>;
@@ -597,8 +892,11 @@ int attn_plan(AttnPlan& plan, const char** why) {
   const AttnParams& p = plan.p;
   int rc = attn_check(p, why);
   if (rc) return rc;
-  plan.tc = p.impl == 0 && (p.d_head == 64 || p.d_head == 128);
+  const bool tc_dh = p.d_head == 64 || p.d_head == 128;
+  plan.tc = (p.impl == 0 || p.impl == 2 || p.impl == 3) && tc_dh;
   if (!plan.tc) return 0;
+  // two query tiles per CTA (ping-pong) where the second tile is rarely padding
+  plan.pp = p.impl == 3 || (p.impl == 0 && p.n_q >= 512);
   const int cols = p.n_heads * p.d_head;
   if (!make_tmap_f16(&plan.tmap_q, p.q, p.batch * p.n_q, cols, p.ldq, kTcBQ) ||
       !make_tmap_f16(&plan.tmap_kv, p.k, p.batch * p.n_kv, cols, p.ldkv, kTcBK) ||
@@ -611,6 +909,7 @@ int attn_plan(AttnPlan& plan, const char** why) {
 
 cudaError_t attn_launch(const AttnPlan& plan, cudaStream_t s) {
   const AttnParams& p = plan.p;
+  if (plan.tc && plan.pp) return p.d_head == 64 ? launch_pp<64>(plan, s) : launch_pp<128>(plan, s);
   if (plan.tc) return p.d_head == 64 ? launch_tc<64>(plan, s) : launch_tc<128>(plan, s);
   switch (p.d_head) {
     case 64: return launch_dh<64, 64>(p, s);

@@ -90,12 +90,15 @@ struct AttnParams {
   f16* o;
   int ldo;
   int batch, n_q, n_kv, n_heads, d_head;
-  int impl;  // 0: tcgen05 where d_head is 64 or 128, else mma.sync; 1: mma.sync
+  int impl;  // 0: tcgen05 where d_head is 64 or 128 (two query tiles per CTA when n_q >= 512),
+             //    else mma.sync; 1: mma.sync; 2: tcgen05, one query tile per CTA; 3: tcgen05,
+             //    two query tiles per CTA
 };
 // A planned attention launch: parameters plus TMA descriptors for the tcgen05 kernel.
 struct AttnPlan {
   AttnParams p{};
   bool tc = false;
+  bool pp = false;  // two query tiles per CTA (attn_pp_kernel)
   CUtensorMap tmap_q;
   CUtensorMap tmap_kv;
   CUtensorMap tmap_v;

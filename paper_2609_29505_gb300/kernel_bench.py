@@ -78,7 +78,7 @@ def case_attention(a):
     ms = _time(lambda: binding.sgd_kernel_attention(q, 3 * d, k, v, 3 * d, o, d, B, N, N, H, dh,
                                                     impl=a.impl), a.iters, a.warmup)
     flops = 4.0 * B * H * N * N * dh
-    return dict(case="attention", impl=["tcgen05", "mma_sync"][a.impl], batch=B, heads=H,
+    return dict(case="attention", impl=["tcgen05", "mma_sync", "tcgen05_1tile", "tcgen05_2tile"][a.impl], batch=B, heads=H,
                 tokens=N, dh=dh, ms=ms, tflops=flops / ms / 1e9)
 
 
@@ -115,7 +115,8 @@ def main():
     ap.add_argument("--batch", type=int, default=4)
     ap.add_argument("--heads", type=int, default=32)
     ap.add_argument("--dh", type=int, default=128)
-    ap.add_argument("--impl", type=int, default=0, help="attention: 0 tcgen05, 1 mma.sync")
+    ap.add_argument("--impl", type=int, default=0, help="attention: 0 tcgen05 (auto), 1 mma.sync, 2 tcgen05 one query tile per CTA, "
+                         "3 tcgen05 two query tiles per CTA")
     ap.add_argument("--rows", type=int, default=4096)
     ap.add_argument("--d", type=int, default=4096)
     ap.add_argument("--caches", type=int, default=8)

@@ -151,11 +151,12 @@ def test_gemm_rope_epilogue(B, simt, dh):
     _check_f16(out, want.reshape(M, N), extra_abs=1e-4)
 
 
-@pytest.mark.parametrize("impl", [0, 1], ids=["tcgen05", "mma_sync"])
+@pytest.mark.parametrize("impl", [0, 1, 2, 3], ids=["tcgen05", "mma_sync", "tcgen05_1tile", "tcgen05_2tile"])
 @pytest.mark.parametrize("dh,H,nq,nkv,bsz", [(64, 4, 64, 64, 1), (72, 3, 136, 136, 2),
                                               (128, 2, 192, 192, 2), (64, 5, 200, 77, 2),
                                               (64, 4, 258, 258, 2), (128, 2, 33, 5, 3),
-                                              (128, 3, 1024, 1024, 1), (64, 2, 300, 700, 2)])
+                                              (128, 3, 1024, 1024, 1), (64, 2, 300, 700, 2),
+                                              (128, 2, 600, 333, 2), (64, 3, 512, 1024, 1)])
 def test_attention(B, dh, H, nq, nkv, bsz, impl):
     rng = np.random.default_rng(dh + nq + nkv)
     d = H * dh
@@ -172,6 +173,30 @@ def test_attention(B, dh, H, nq, nkv, bsz, impl):
     err = np.linalg.norm(got - want) / np.linalg.norm(want)
     assert err < 1.5e-3, err
     assert np.max(np.abs(got - want)) < 5e-3 * float(np.abs(want).max())
+    assert B.sgd_kernel_status() == 0
+
+
+@pytest.mark.parametrize("impl", [0, 2, 3], ids=["tcgen05", "tcgen05_1tile", "tcgen05_2tile"])
+@pytest.mark.parametrize("dh", [64, 128])
+def test_attention_growing_row_maxima(B, dh, impl):
+    """Later key tiles carry larger scores, so row maxima grow by more than 2^8 from tile to
+    tile and the accumulated O is rescaled in TMEM (the lazy-rescale path)."""
+    rng = np.random.default_rng(dh + impl)
+    H, nq, nkv, bsz = 2, 640, 640, 1
+    d = H * dh
+    q = _rand(rng, (bsz * nq, d), 1.0).cuda()
+    kk = rng.standard_normal((bsz * nkv, d)).astype(np.float32)
+    kk *= (1.0 + 1.5 * (np.arange(bsz * nkv) // 128))[:, None]  # tile j scaled by 1 + 1.5 j
+    k = torch.from_numpy(kk).half().cuda()
+    v = _rand(rng, (bsz * nkv, d)).cuda()
+    o = torch.empty(bsz * nq, d, dtype=torch.float16, device="cuda")
+    B.sgd_kernel_attention(q, d, k, v, d, o, d, bsz, nq, nkv, H, dh, impl=impl)
+    torch.cuda.synchronize()
+    want = odn.attention(_f(q).reshape(bsz, nq, d), _f(k).reshape(bsz, nkv, d),
+                         _f(v).reshape(bsz, nkv, d), H).reshape(bsz * nq, d)
+    got = _f(o)
+    err = np.linalg.norm(got - want) / np.linalg.norm(want)
+    assert err < 1.5e-3, err
     assert B.sgd_kernel_status() == 0
 
 
