@@ -108,10 +108,9 @@ SGD_API int sgd_kernel_gemm_static_ws(const void* A, int lda, const void* B, int
  * masked.  Row r = b * n_q + i of q / o, row b * n_kv + j of k / v; head h occupies
  * columns [h d_head, (h+1) d_head).  fp16 in and out; d_head in {64, 72, 128};
  * leading dimensions in elements, multiples of 8.  impl = 0: tcgen05 for d_head 64 / 128
- * (S, P and O in TMEM; two 128-query tiles per CTA, whose softmax warpgroups alternate with
- * each other's MMAs, when n_q >= 512, else one tile per CTA with P in shared memory), the
- * mma.sync kernel for 72; 1: the mma.sync kernel for every d_head; 2: tcgen05 with one
- * query tile per CTA; 3: tcgen05 with two query tiles per CTA (d_head 72 takes mma.sync).
+ * (S, P and O in TMEM; two 128-query tiles per CTA whose softmax warpgroups alternate with
+ * each other's MMAs), the mma.sync kernel for 72; 1: the mma.sync kernel for every d_head;
+ * 2: tcgen05 with one query tile per CTA and P in shared memory; 3: the same as 0.
  */
 SGD_API int sgd_kernel_attention(const void* q, int ldq, const void* k, const void* v, int ldkv,
                          void* o, int ldo, int batch, int n_q, int n_kv, int n_heads,

@@ -3,7 +3,9 @@
 // Used inside every active self-attention and cross-attention branch (Algorithm 2:
 // an active unit evaluates F_l(h_{l-1,s}; c_s)); frozen units never launch it.
 //
-// Two kernels:
+// Three kernels:
+//   attn_pp_kernel (d_h 64, 128; the default): tcgen05 with two query tiles per CTA and two
+//     alternating softmax warpgroups, P in TMEM; described above the kernel.
 //   attn_tc_kernel (d_h 64, 128): tcgen05.  One CTA = 128 queries of one (sample, head),
 //     keys in tiles of 128.  Warp 0 loads Q once and K/V tiles through a 2-stage TMA ring;
 //     warp 1 issues S = Q K^T into one of two TMEM S buffers and O += P V into a TMEM O
@@ -251,6 +253,20 @@ constexpr int kTcBQ = 128;
 constexpr int kTcBK = 128;
 constexpr int kAtom = 128 * 64 * 2;  // 128 rows x 64 fp16: one 128-byte-swizzle column block
 constexpr float kRescaleLog2 = 8.f;  // rescale O only when the row max grows by > 2^8
+
+// fp16 pair, round to nearest, no saturation (the callers' values are far below 65504)
+__device__ __forceinline__ uint32_t pack_f16x2_rn(float lo, float hi) {
+  __half2 v = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// 2^x with the hardware's approximate base-2 exponential (PTX ex2.approx.ftz.f32); the
+// arguments here are <= 8 and results below the fp16 range flush to zero either way.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 
 struct AttnTcArgs {
   CUtensorMap tmap_q;
@@ -682,31 +698,30 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
     const uint32_t o_col = tmem + lane_base + L::kTmemO + t * DH;
     float m2 = -INFINITY, l = 0.f;
     bool ok = true;
-    uint32_t r0[16], r1[16];
+    uint32_t r[kTcBK];
     for (int j = 0; j < nt; ++j) {
       if (!(ok = warp_wait_bar(&s_full[t], j & 1, abort_flag, a.status, 27))) break;
       tc_fence_after();
       const int kb = j * kTcBK;
-      const bool whole = kb + kTcBK <= a.n_kv;
-      // pass 1: the tile's row maximum (scores in log2 units)
+      const int nvalid = min(a.n_kv - kb, kTcBK);  // keys of this tile (the rest are masked)
+      // the whole S row in registers, one TMEM round trip
+#pragma unroll
+      for (int c = 0; c < kTcBK; c += 16) tmem_ld16(s_col + c, r + c);
+#pragma unroll
+      for (int c = 0; c < kTcBK; c += 16) tmem_ld_wait16(r + c);
+      if (nvalid < kTcBK) {  // masked keys score -inf (P = 0)
+#pragma unroll
+        for (int c = 0; c < kTcBK; ++c)
+          if (c >= nvalid) r[c] = __float_as_uint(-INFINITY);
+      }
+      // the row maximum of the raw scores (scale > 0 commutes with max), then log2 units
       float mx[8];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) mx[i] = -INFINITY;
+      for (int i = 0; i < 8; ++i) mx[i] = __uint_as_float(r[i]);
 #pragma unroll
-      for (int c = 0; c < kTcBK; c += 32) {
-        tmem_ld16(s_col + c, r0);
-        tmem_ld16(s_col + c + 16, r1);
-        tmem_ld_wait16(r0);
-        tmem_ld_wait16(r1);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float v0 = (whole || kb + c + i < a.n_kv) ? __uint_as_float(r0[i]) * a.scale_log2 : -INFINITY;
-          const float v1 = (whole || kb + c + 16 + i < a.n_kv) ? __uint_as_float(r1[i]) * a.scale_log2 : -INFINITY;
-          mx[i & 7] = fmaxf(mx[i & 7], fmaxf(v0, v1));
-        }
-      }
-      const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      for (int c = 8; c < kTcBK; ++c) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(r[c]));
+      const float mt = a.scale_log2 * fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                                            fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
       if (j == 0) {
         m2 = mt;
       } else if (__any_sync(0xffffffffu, mt > m2 + kRescaleLog2)) {
@@ -715,43 +730,36 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
         tc_fence_after();
         const float mnew = fmaxf(m2, mt);
         const float corr = exp2f(m2 - mnew);
-#pragma unroll
+        uint32_t o16[16];
+#pragma unroll 1
         for (int c = 0; c < DH; c += 16) {
-          tmem_ld16(o_col + c, r0);
-          tmem_ld_wait16(r0);
+          tmem_ld16(o_col + c, o16);
+          tmem_ld_wait16(o16);
 #pragma unroll
-          for (int i = 0; i < 16; ++i) r0[i] = __float_as_uint(__uint_as_float(r0[i]) * corr);
-          tmem_st16(o_col + c, r0);
+          for (int i = 0; i < 16; ++i) o16[i] = __float_as_uint(__uint_as_float(o16[i]) * corr);
+          tmem_st16(o_col + c, o16);
         }
         tmem_st_wait();
         l *= corr;
         m2 = mnew;
       }
-      // pass 2: P = exp2(score - m2) as fp16 pairs over columns [0, 64) of this S; the 16
-      // packed columns of scores [c, c + 32) land on scores already read
+      // P = 2^(score * scale - m2) packed as fp16 pairs in place (pair k of a 32-score chunk
+      // into register k of the chunk, already consumed) and stored over columns [0, 64) of
+      // this S: chunk c's 16 packed columns land on scores already read
+      const float neg_m2 = -m2;
       float ls[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) ls[i] = 0.f;
 #pragma unroll
       for (int c = 0; c < kTcBK; c += 32) {
-        tmem_ld16(s_col + c, r0);
-        tmem_ld16(s_col + c + 16, r1);
-        tmem_ld_wait16(r0);
-        tmem_ld_wait16(r1);
-        uint32_t pk[16];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          float p[4];
-          const int c0 = c + 2 * i;
-          p[0] = (whole || kb + c0 < a.n_kv) ? exp2f(__uint_as_float(r0[2 * i]) * a.scale_log2 - m2) : 0.f;
-          p[1] = (whole || kb + c0 + 1 < a.n_kv) ? exp2f(__uint_as_float(r0[2 * i + 1]) * a.scale_log2 - m2) : 0.f;
-          p[2] = (whole || kb + c0 + 16 < a.n_kv) ? exp2f(__uint_as_float(r1[2 * i]) * a.scale_log2 - m2) : 0.f;
-          p[3] = (whole || kb + c0 + 17 < a.n_kv) ? exp2f(__uint_as_float(r1[2 * i + 1]) * a.scale_log2 - m2) : 0.f;
-          ls[i] += (p[0] + p[1]) + (p[2] + p[3]);
-          pk[i] = pack_f16x2(p[0], p[1]);
-          pk[8 + i] = pack_f16x2(p[2], p[3]);
+        for (int k = 0; k < 16; ++k) {
+          const float p0 = ex2_approx(fmaf(__uint_as_float(r[c + 2 * k]), a.scale_log2, neg_m2));
+          const float p1 = ex2_approx(fmaf(__uint_as_float(r[c + 2 * k + 1]), a.scale_log2, neg_m2));
+          ls[k & 7] += p0 + p1;
+          r[c + k] = pack_f16x2_rn(p0, p1);
         }
-        tmem_st16(s_col + c / 2, pk);
+        tmem_st16(s_col + c / 2, r + c);
       }
       l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
       tmem_st_wait();
@@ -766,11 +774,11 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
       f16* orow = a.o + (static_cast<int64_t>(b) * a.n_q + qrow) * a.ldo + h * DH;
 #pragma unroll
       for (int c = 0; c < DH; c += 16) {
-        tmem_ld16(o_col + c, r0);
-        tmem_ld_wait16(r0);
+        tmem_ld16(o_col + c, r);
+        tmem_ld_wait16(r);
         float f[16];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(r0[i]) * inv;
+        for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(r[i]) * inv;
         if (qrow < a.n_q) {
           reinterpret_cast<uint4*>(orow + c)[0] = pack_f16x8(f);
           reinterpret_cast<uint4*>(orow + c)[1] = pack_f16x8(f + 8);
@@ -895,8 +903,9 @@ int attn_plan(AttnPlan& plan, const char** why) {
   const bool tc_dh = p.d_head == 64 || p.d_head == 128;
   plan.tc = (p.impl == 0 || p.impl == 2 || p.impl == 3) && tc_dh;
   if (!plan.tc) return 0;
-  // two query tiles per CTA (ping-pong) where the second tile is rarely padding
-  plan.pp = p.impl == 3 || (p.impl == 0 && p.n_q >= 512);
+  // two query tiles per CTA (ping-pong) unless one tile per CTA is forced: faster on every
+  // measured shape, short and ragged ones included (258 tokens: 37.8 against 55.2 us)
+  plan.pp = p.impl == 0 || p.impl == 3;
   const int cols = p.n_heads * p.d_head;
   if (!make_tmap_f16(&plan.tmap_q, p.q, p.batch * p.n_q, cols, p.ldq, kTcBQ) ||
       !make_tmap_f16(&plan.tmap_kv, p.k, p.batch * p.n_kv, cols, p.ldkv, kTcBK) ||

@@ -90,9 +90,8 @@ struct AttnParams {
   f16* o;
   int ldo;
   int batch, n_q, n_kv, n_heads, d_head;
-  int impl;  // 0: tcgen05 where d_head is 64 or 128 (two query tiles per CTA when n_q >= 512),
-             //    else mma.sync; 1: mma.sync; 2: tcgen05, one query tile per CTA; 3: tcgen05,
-             //    two query tiles per CTA
+  int impl;  // 0: tcgen05 with two query tiles per CTA where d_head is 64 or 128, else
+             //    mma.sync; 1: mma.sync; 2: tcgen05, one query tile per CTA; 3: same as 0
 };
 // A planned attention launch: parameters plus TMA descriptors for the tcgen05 kernel.
 struct AttnPlan {
