@@ -231,7 +231,7 @@ __device__ __forceinline__ void store_partial(float* slot, int r, uint32_t tbase
 // Epilogue of one 128 x BN accumulator: this thread owns tile row `row` and handles
 // accumulator columns [cb, ce) (gated: output columns [cb, ce) of the BN / 2 the tile
 // produces), reading the accumulator through `src`.
-template <int BN, class Src>
+template <int BN, bool kFastRope, class Src>
 __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int row, int n_blk,
                                               const Src& src, int cb, int ce) {
   constexpr int kBN = BN;
@@ -253,7 +253,61 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
     return;
   }
   const int n0 = n_blk * kBN;
-  if (e.kind == SGD_EPI_ROPE) {
+  if (e.kind == SGD_EPI_ROPE && kFastRope) {
+    // every head of the tile shares the row's position, so each 16-wide chunk of the cos /
+    // sin tables is read once for all of them and the next chunk is fetched ahead (the
+    // 4-epilogue-warp kernel, which has the registers for it)
+    const int dh = e.d_head, hd = dh >> 1;
+    const int pos = row_ok ? row % e.rope_tokens : 0;
+    const float4* cs4 = reinterpret_cast<const float4*>(e.rope_cos + static_cast<int64_t>(pos) * hd);
+    const float4* sn4 = reinterpret_cast<const float4*>(e.rope_sin + static_cast<int64_t>(pos) * hd);
+    const bool any_rot = row_ok && (n0 + cb) < e.rope_cols;
+    float4 cn[4], sn[4];
+    if (any_rot) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        cn[i] = cs4[i];
+        sn[i] = sn4[i];
+      }
+    }
+    for (int j = 0; j < hd; j += 16) {
+      float cc[16], ss[16];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        cc[4 * i] = cn[i].x; cc[4 * i + 1] = cn[i].y; cc[4 * i + 2] = cn[i].z; cc[4 * i + 3] = cn[i].w;
+        ss[4 * i] = sn[i].x; ss[4 * i + 1] = sn[i].y; ss[4 * i + 2] = sn[i].z; ss[4 * i + 3] = sn[i].w;
+      }
+      if (any_rot && j + 16 < hd) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          cn[i] = cs4[(j + 16) / 4 + i];
+          sn[i] = sn4[(j + 16) / 4 + i];
+        }
+      }
+      for (int hb = cb; hb < ce; hb += dh) {
+        if (n0 + hb >= a.N) break;
+        const bool rot = (n0 + hb) < e.rope_cols;
+        src.load2(hb + j, hb + hd + j, x, y);
+        if (rot && row_ok) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const float a1 = x[i], a2 = y[i];
+            x[i] = a1 * cc[i] - a2 * ss[i];
+            y[i] = a2 * cc[i] + a1 * ss[i];
+          }
+        }
+        if (row_ok) {
+          const int c1 = n0 + hb + j, c2 = c1 + hd;
+          epi_store8(e, out, row, c1, x);
+          epi_store8(e, out, row, c1 + 8, x + 8);
+          epi_store8(e, out, row, c2, y);
+          epi_store8(e, out, row, c2 + 8, y + 8);
+        }
+      }
+    }
+    return;
+  }
+  if (e.kind == SGD_EPI_ROPE && !kFastRope) {
     const int dh = e.d_head, hd = dh >> 1;
     const int pos = row_ok ? row % e.rope_tokens : 0;
     for (int hb = cb; hb < ce; hb += dh) {
@@ -278,6 +332,46 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
           epi_store8(e, out, row, c1 + 8, x + 8);
           epi_store8(e, out, row, c2, y);
           epi_store8(e, out, row, c2 + 8, y + 8);
+        }
+      }
+    }
+    return;
+  }
+  if (e.kind == SGD_EPI_DELTA) {
+    // residual update: the chunk's h (and gate) loads are issued together, ahead of the
+    // accumulator reads, instead of one dependent load per 8 columns
+    const float* grow =
+        e.gate ? e.gate + static_cast<int64_t>(row_ok ? row / e.rows_per_batch : 0) * e.ld_gate + n0 : nullptr;
+    float* hrow = e.h + static_cast<int64_t>(row) * e.ldh + n0;
+    for (int c = cb; c < ce; c += 32) {
+      if (n0 + c >= a.N) break;
+      // unconditional loads (a predicated load here makes the compiler spill): columns past
+      // N repeat the row's last four, which are read but never used
+      float4 hv[8], gv[8];
+      const int hr = row_ok ? 0 : -row;  // rows past M read row 0 instead
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int col = min(c + 4 * q, a.N - n0 - 4);
+        hv[q] = *reinterpret_cast<const float4*>(hrow + static_cast<int64_t>(hr) * e.ldh + col);
+        gv[q] = grow ? *reinterpret_cast<const float4*>(grow + col) : make_float4(1.f, 1.f, 1.f, 1.f);
+      }
+      src.load2(c, c + 16, x, y);
+      if (row_ok) {
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+          if (n0 + c + 8 * g >= a.N) continue;
+          float* v = g < 2 ? x + 8 * g : y + 8 * (g - 2);  // constant once unrolled
+          if (grow) {
+            v[0] *= gv[2 * g].x; v[1] *= gv[2 * g].y; v[2] *= gv[2 * g].z; v[3] *= gv[2 * g].w;
+            v[4] *= gv[2 * g + 1].x; v[5] *= gv[2 * g + 1].y; v[6] *= gv[2 * g + 1].z; v[7] *= gv[2 * g + 1].w;
+          }
+          float4 h0 = hv[2 * g], h1 = hv[2 * g + 1];
+          h0.x += v[0]; h0.y += v[1]; h0.z += v[2]; h0.w += v[3];
+          h1.x += v[4]; h1.y += v[5]; h1.z += v[6]; h1.w += v[7];
+          float4* hp = reinterpret_cast<float4*>(hrow + c + 8 * g);
+          hp[0] = h0;
+          hp[1] = h1;
+          if (e.cache) store8_f16(e.cache, e.ld_cache, row, n0 + c + 8 * g, v);
         }
       }
     }
@@ -549,7 +643,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
       if (u >= w.n_sk) {  // data-parallel tile
         if (!warp_wait(&tfull[acc], aph, abort_flag, a.status, 4)) break;
         tc_fence_after();
-        epilogue_tile<kBN>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce);
+        epilogue_tile<kBN, kEpiWarps == 4>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -561,7 +655,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
       if (k0 == 0 && k1 == a.num_k) {  // the whole K range of the tile lies in this CTA's share
         if (ok) {
           tc_fence_after();
-          epilogue_tile<kBN>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce);
+          epilogue_tile<kBN, kEpiWarps == 4>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce);
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -593,7 +687,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
       epi_bar(kEpiThreads);
       if (*last_flag != 0) {
         __threadfence();
-        epilogue_tile<kBN>(a, out, row, n_blk, WsSrc<kBN>{slot0, nseg, q * 32 + lane, a.epi.alpha}, cb, ce);
+        epilogue_tile<kBN, kEpiWarps == 4>(a, out, row, n_blk, WsSrc<kBN>{slot0, nseg, q * 32 + lane, a.epi.alpha}, cb, ce);
         if (threadIdx.x == 64) a.sk_cnt[tile] = 0;
       }
     }
