@@ -75,7 +75,8 @@ typedef struct {
  * load of their B tile; 3 and 4 the forms of 0 and 2 with 32-element K-blocks (64-byte
  * swizzle); 5, 6, 7 force 128 x 256 tiles with 4 epilogue warps, 128 x 256 with 8, and
  * 128 x 128 with 8 and no stream-K (128 x 128 applies to plain, GELU and DELTA epilogues
- * only); 8 is 0 without stream-K, 9 is 0 with stream-K whenever the last wave is partial.
+ * only); 8 is 0 without stream-K, 9 is 0 with stream-K whenever the last wave is partial;
+ * 10 forces 128 x 224 tiles (5 pipeline stages, no stream-K; plain, GELU and DELTA only).
  * The stream-K workspace is owned by the library, one per (device, stream), allocated
  * or grown by the first call that needs it (after synchronising that stream).
  */

@@ -1475,7 +1475,7 @@ int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N
   p.M = M;
   p.N = N;
   p.K = K;
-  if (use_simt < 0 || use_simt > 9) return fail(SGD_ERR_ARG, "gemm: variant must be in 0..9");
+  if (use_simt < 0 || use_simt > 10) return fail(SGD_ERR_ARG, "gemm: variant must be in 0..10");
   p.simt = use_simt == 1;
   p.cluster = (use_simt == 2 || use_simt == 4) ? 2 : 1;
   p.bk = (use_simt == 3 || use_simt == 4) ? 32 : 64;
@@ -1484,6 +1484,7 @@ int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N
   if (use_simt == 7) { p.bn = 128; p.epiw = 8; p.sk = 0; }
   if (use_simt == 8) p.sk = 0;
   if (use_simt == 9) p.sk = 1;
+  if (use_simt == 10) { p.bn = 224; p.epiw = 8; }
   EpiParams& e = p.epi;
   e = EpiParams{};
   e.kind = ea->kind;
@@ -1527,7 +1528,7 @@ int sgd_kernel_gemm_static_ws(const void* A, int lda, const void* B, int ldb, in
                               const sgd_epilogue_args* ea, int variant, void* stream) {
   if (!ea) return fail(SGD_ERR_ARG, "null epilogue");
   if (ea->kind < 0 || ea->kind > SGD_EPI_ROPE) return fail(SGD_ERR_ARG, "bad epilogue kind");
-  if (variant < 0 || variant > 9) return fail(SGD_ERR_ARG, "gemm: variant must be in 0..9");
+  if (variant < 0 || variant > 10) return fail(SGD_ERR_ARG, "gemm: variant must be in 0..10");
   GemmPlan p;
   p.A = H16(A);
   p.lda = lda;
@@ -1544,6 +1545,7 @@ int sgd_kernel_gemm_static_ws(const void* A, int lda, const void* B, int ldb, in
   if (variant == 7) { p.bn = 128; p.epiw = 8; p.sk = 0; }
   if (variant == 8) p.sk = 0;
   if (variant == 9) p.sk = 1;
+  if (variant == 10) { p.bn = 224; p.epiw = 8; }
   EpiParams& e = p.epi;
   e = EpiParams{};
   e.kind = ea->kind;

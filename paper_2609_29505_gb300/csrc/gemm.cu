@@ -36,20 +36,22 @@ constexpr int kBM = 128;
 // K-block geometry.  BK = 64: 128-byte rows, 128-byte swizzle, 4 stages of 48 KB.
 // BK = 32: 64-byte rows, 64-byte swizzle, 9 stages of 24 KB — the same MMA work per
 // byte but a third more bytes in flight, to cover more of the TMA refill latency.
-// BN = 256 or 128 accumulator columns per tile (two accumulators in TMEM); EPIW = 4 or 8
-// epilogue warps (8: warps w and w + 4 split the tile's columns).
+// BN = 256, 224 or 128 accumulator columns per tile (two accumulators in TMEM); EPIW = 4 or
+// 8 epilogue warps (8: warps w and w + 4 split the tile's columns).  BN = 224 tiles N = 4096
+// into 19 columns of tiles (608 tiles = 4 full waves of 152 at M = 4096) and its 44 KB stages
+// fit 5 deep.
 template <int BK, int BN = 256, int EPIW = 8>
 struct TileCfg {
   static constexpr int kBK = BK;
   static constexpr int kBN = BN;
   static constexpr int kEpiWarps = EPIW;
   static constexpr int kThreads = 64 + 32 * EPIW;
-  static constexpr int kTmemCols = 2 * BN;
+  static constexpr int kTmemCols = BN == 224 ? 512 : 2 * BN;  // allocations are powers of 2
   static constexpr int kTileA = kBM * BK * 2;
   static constexpr int kTileBHalf = 128 * BK * 2;
   static constexpr int kTileB = BN * BK * 2;
   static constexpr int kStageBytes = kTileA + kTileB;
-  static constexpr int kStages = (192 * 1024) / kStageBytes;
+  static constexpr int kStages = BN == 224 ? 5 : (192 * 1024) / kStageBytes;
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
   static_assert(kSmemBytes <= 232448, "shared memory");
   static_assert((2 * kStages + 5) * 8 + 3 * 4 <= 256, "barrier block");
@@ -623,13 +625,16 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
     const int q = warp & 3;
     constexpr int kEpiThreads = 32 * kEpiWarps;
     // column range of this warp: all of the tile (4 epilogue warps) or one half (8)
+    // (8 warps: the first half rounded up to a multiple of 32 columns, e.g. 128 + 96 at BN 224)
+    constexpr int kSplit = ((kBN / 2 + 31) / 32) * 32, kSplitGated = ((kBN / 4 + 31) / 32) * 32;
     const int span = a.gated ? kBN / 2 : kBN;
     const int part = kEpiWarps == 8 ? ((warp - 2) >> 2) : 0;
-    const int cb = kEpiWarps == 8 ? part * (span / 2) : 0;
-    const int ce = kEpiWarps == 8 ? cb + span / 2 : span;
+    const int split = a.gated ? kSplitGated : kSplit;
+    const int cb = kEpiWarps == 8 ? part * split : 0;
+    const int ce = kEpiWarps == 8 ? (part ? span : split) : span;
     // accumulator columns this warp stores for a stream-K partial
-    const int pb = kEpiWarps == 8 ? part * (kBN / 2) : 0;
-    const int pe = kEpiWarps == 8 ? pb + kBN / 2 : kBN;
+    const int pb = kEpiWarps == 8 ? part * kSplit : 0;
+    const int pe = kEpiWarps == 8 ? (part ? kBN : kSplit) : kBN;
     const int total = a.sk_tiles * a.num_k;
     void* out = a.epi.out_slot ? *a.epi.out_slot : a.epi.out;
     for (int u = 0; u < w.n_units; ++u) {
@@ -984,11 +989,6 @@ int gemm_plan(GemmPlan& p, const char** why) {
   if (p.simt) return 0;
   const int b_rows = gated ? 2 * p.N : p.N;
   if (p.bk != 64 && p.bk != 32) p.bk = 64;
-  if (!make_tmap_f16(&p.tmap_a, p.A, p.M, p.K, p.lda, 128, p.bk) ||
-      !make_tmap_f16(&p.tmap_b, p.B, b_rows, p.K, p.ldb, 128, p.bk)) {
-    *why = "gemm: cuTensorMapEncodeTiled failed (driver entry point unavailable or bad layout)";
-    return -5;
-  }
   const int num_m = (p.M + kBM - 1) / kBM;
   const int sms = num_sms();
   const int num_k = (p.K + p.bk - 1) / p.bk;
@@ -999,6 +999,13 @@ int gemm_plan(GemmPlan& p, const char** why) {
   // the last wave; they need a plain epilogue and one-CTA launches.  4 epilogue warps for
   // RoPE and gated epilogues.
   const bool small_ok = !gated && e.kind != SGD_EPI_ROPE && p.bk == 64 && p.cluster == 1;
+  // 128 x 224 tiles where they fill whole waves exactly, K is long and the last column of
+  // tiles wastes under a tenth of N (e.g. M = N = 4096 at K >= 3072: 608 tiles = 4 waves;
+  // measured 1266 against 1233 TFLOP/s for 128 x 256 with stream-K)
+  const int n224 = (p.N + 223) / 224;
+  if (p.bn == 0 && p.sk != 1 && small_ok && p.K >= 3072 && (num_m * n224) % sms == 0 &&
+      10 * (n224 * 224 - p.N) < p.N)
+    p.bn = 224;
   if (p.bn == 0) {
     const int t256 = num_m * (gated ? (p.N + 127) / 128 : (p.N + 255) / 256);
     const int w256 = (t256 + sms - 1) / sms;
@@ -1007,9 +1014,15 @@ int gemm_plan(GemmPlan& p, const char** why) {
     const bool sk_on = p.cluster == 1 && p.sk != 0 && sk256.tiles > 0;
     p.bn = (small_ok && !sk_on && 2 * w128 < 3 * w256) ? 128 : 256;
   }
-  if (p.bn != 128 || !small_ok) p.bn = 256;
+  if ((p.bn != 128 && p.bn != 224) || !small_ok) p.bn = 256;
+  if (p.bn == 224) p.sk = 0;
   if (p.epiw == 0) p.epiw = (e.kind == SGD_EPI_ROPE || gated) ? 4 : 8;
-  if (p.bn == 128 || p.cluster == 2 || p.bk == 32) p.epiw = 8;
+  if (p.bn == 128 || p.bn == 224 || p.cluster == 2 || p.bk == 32) p.epiw = 8;
+  if (!make_tmap_f16(&p.tmap_a, p.A, p.M, p.K, p.lda, 128, p.bk) ||
+      !make_tmap_f16(&p.tmap_b, p.B, b_rows, p.K, p.ldb, p.bn == 224 ? 224 : 128, p.bk)) {
+    *why = "gemm: cuTensorMapEncodeTiled failed (driver entry point unavailable or bad layout)";
+    return -5;
+  }
   const int num_n = gated ? (p.N + 127) / 128 : (p.N + p.bn - 1) / p.bn;
   if (p.cluster == 2 && num_m < 2) p.cluster = 1;  // nothing to share
   int max_units = sms;
@@ -1102,6 +1115,7 @@ cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s) {
     return p.cluster == 2 ? launch_tc<2, 32, 256, 8>(p, a, s) : launch_tc<1, 32, 256, 8>(p, a, s);
   if (p.cluster == 2) return launch_tc<2, 64, 256, 8>(p, a, s);
   if (p.bn == 128) return launch_tc<1, 64, 128, 8>(p, a, s);
+  if (p.bn == 224) return launch_tc<1, 64, 224, 8>(p, a, s);
   return p.epiw == 4 ? launch_tc<1, 64, 256, 4>(p, a, s) : launch_tc<1, 64, 256, 8>(p, a, s);
 }
 

@@ -59,8 +59,8 @@ def _run(entry, A, W, h0, M, N, K, epi, variant, stream=None):
 
 @pytest.mark.gpu
 @pytest.mark.parametrize("M,N,K,epi,variant", [
-    (4096, 4096, 4096, "f16", 0),     # chooses stream-K by itself (attention-output shape)
-    (4096, 4096, 12288, "delta", 0),  # chooses stream-K by itself (MLP down-projection shape)
+    (4096, 4096, 4096, "f16", 9),     # stream-K forced (attention-output shape)
+    (4096, 4096, 12288, "delta", 9),  # stream-K forced (MLP down-projection shape)
     (2048, 1152, 1152, "delta", 9),   # stream-K forced, 128-column tiles
     (1000, 1376, 512, "gelu", 9),     # ragged M and N
     (2048, 2752, 1024, "gated", 9),   # 48 split tiles x 4 segments: 24 MiB of partials
@@ -134,4 +134,4 @@ def test_static_ws_validates_on_host():
     assert L.sgd_kernel_gemm_static_ws(None, 8, None, 8, 8, 8, 8, C.byref(epi), 0, None) == binding.SGD_ERR_ARG
     epi = binding.sgd_epilogue_args(kind=binding.EPI_F16, out=64, ldo=8)
     assert L.sgd_kernel_gemm_static_ws(64, 12, 64, 12, 8, 8, 12, C.byref(epi), 0, None) == binding.SGD_ERR_SHAPE
-    assert L.sgd_kernel_gemm_static_ws(64, 8, 64, 8, 8, 8, 8, C.byref(epi), 10, None) == binding.SGD_ERR_ARG
+    assert L.sgd_kernel_gemm_static_ws(64, 8, 64, 8, 8, 8, 8, C.byref(epi), 11, None) == binding.SGD_ERR_ARG
