@@ -42,6 +42,9 @@ def parse():
                     help="also time one trajectory at 100/50/33%% budgets (adds key 'budget_sweep')")
     ap.add_argument("--ablation", action="store_true",
                     help="also time the execution modes of Table tab:kernel (adds key 'ablation')")
+    ap.add_argument("--rankings", action="store_true",
+                    help="also time one trajectory per static ranking of Table tab:cross-ablation "
+                         "and for branch granularity, all at the same budget (adds key 'rankings')")
     ap.add_argument("--policies", action="store_true",
                     help="also time the static schedule against the activation-drift policy of "
                          "App. B.1 at the same budget (adds key 'policies')")
@@ -320,6 +323,11 @@ def run_native(args):
     if args.ablation:
         ablation = run_ablation(binding, model, cfg, T, weights, sched, xs, out, cls, ctx, stream)
 
+    rankings = None
+    if args.rankings:
+        rankings = run_rankings(binding, model, cfg, T, weights, args.budget, sched, xs, out, cls,
+                                ctx, stream)
+
     policies = None
     if args.policies:
         policies = run_policies(binding, model, cfg, T, xs, out, cls, ctx, stream)
@@ -346,7 +354,7 @@ def run_native(args):
                    "cache_gb": round(info["cache_bytes"] / 2 ** 30, 2), "setup": setup_t},
         "roofline": roofline, "step_roofline": step_roof, "kernels": kernels,
         "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(gpu_launches),
-        "ablation": ablation, "budget_sweep": sweep, "policies": policies,
+        "ablation": ablation, "budget_sweep": sweep, "policies": policies, "rankings": rankings,
         "clocks": clk.summary(),
     }
     if rank == 0:
@@ -427,6 +435,39 @@ def run_ablation(binding, model, cfg, T, weights, sched, xs, out, cls, ctx, stre
     base = rows[0]["trajectory_ms"]
     for r in rows:
         r["speedup_vs_eager_full"] = round(base / r["trajectory_ms"], 3)
+    return rows
+
+
+def run_rankings(binding, model, cfg, T, weights, budget, sched, xs, out, cls, ctx, stream):
+    """Latency of the alternative static rankings (Table tab:cross-ablation) and of branch
+    granularity at the same layer-step budget: the same kernels run; what changes is which
+    units are active at each step, hence the active patterns and graphs.  One trajectory
+    each after a warm-up trajectory, CUDA events on the stream."""
+    import torch
+    from paper_2609_29505_gb300 import schedule
+    from paper_2609_29505_gb300.synth import timestep
+    rows = []
+    variants = [(r, "block") for r in ("scr", "frobenius", "spectral", "stable_rank",
+                                       "frob_stable_rank", "raw_scr", "depth", "random")]
+    variants.append(("scr", "branch"))
+    for ranking, gran in variants:
+        sc = schedule.build_schedule(cfg, weights, T, budget=budget, ranking=ranking, granularity=gran)
+        model.set_schedule(T, sc["lifetimes"], sc["groups"])
+        for rep in range(2):
+            model.reset()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for s in range(1, T + 1):
+                model.step(xs[s - 1], out, timestep(cfg, s, T), s, class_ids=cls, ctx=ctx, stream=stream)
+            e1.record(stream)
+            torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        info = model.info()
+        rows.append({"ranking": ranking, "granularity": gran, "achieved_ratio": round(sc["ratio"], 4),
+                     "n_patterns": info["n_patterns"], "trajectory_ms": round(ms, 2),
+                     "steps_per_s": round(T / (ms / 1e3), 3)})
+    model.set_schedule(T, sched["lifetimes"], sched["groups"])
     return rows
 
 
