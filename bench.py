@@ -159,7 +159,8 @@ def setup_workload(args, device):
     t0 = time.time()
     weights = synth.make_weights(cfg, device)
     inp = synth.make_inputs(cfg, device)
-    torch.cuda.synchronize()
+    if str(device).startswith("cuda"):
+        torch.cuda.synchronize()
     t_w = time.time() - t0
     t0 = time.time()
     sched = schedule.build_schedule(cfg, weights, T, budget=args.budget)
