@@ -1461,75 +1461,13 @@ int kernel_ws(int dev, void* stream, size_t floats, int n_cnt, KernelWs** out) {
   return SGD_OK;
 }
 
-}  // namespace
-
-int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
-                    const sgd_epilogue_args* ea, int use_simt, void* stream) {
-  if (!ea) return fail(SGD_ERR_ARG, "null epilogue");
-  if (ea->kind < 0 || ea->kind > SGD_EPI_ROPE) return fail(SGD_ERR_ARG, "bad epilogue kind");
-  GemmPlan p;
-  p.A = H16(A);
-  p.lda = lda;
-  p.B = H16(B);
-  p.ldb = ldb;
-  p.M = M;
-  p.N = N;
-  p.K = K;
-  if (use_simt < 0 || use_simt > 10) return fail(SGD_ERR_ARG, "gemm: variant must be in 0..10");
-  p.simt = use_simt == 1;
-  p.cluster = (use_simt == 2 || use_simt == 4) ? 2 : 1;
-  p.bk = (use_simt == 3 || use_simt == 4) ? 32 : 64;
-  if (use_simt == 5) { p.bn = 256; p.epiw = 4; }
-  if (use_simt == 6) { p.bn = 256; p.epiw = 8; }
-  if (use_simt == 7) { p.bn = 128; p.epiw = 8; p.sk = 0; }
-  if (use_simt == 8) p.sk = 0;
-  if (use_simt == 9) p.sk = 1;
-  if (use_simt == 10) { p.bn = 224; p.epiw = 8; }
-  EpiParams& e = p.epi;
-  e = EpiParams{};
-  e.kind = ea->kind;
-  e.alpha = ea->alpha != 0.f ? ea->alpha : 1.f;
-  e.out = ea->out;
-  e.ldo = ea->ldo;
-  e.h = ea->h;
-  e.ldh = ea->ldh;
-  e.cache = static_cast<f16*>(ea->cache);
-  e.ld_cache = ea->ld_cache;
-  e.gate = ea->gate;
-  e.ld_gate = ea->ld_gate;
-  e.rows_per_batch = ea->rows_per_batch > 0 ? ea->rows_per_batch : 1;
-  e.act = ea->act;
-  e.rope_cos = ea->rope_cos;
-  e.rope_sin = ea->rope_sin;
-  e.rope_tokens = ea->rope_tokens;
-  e.d_head = ea->d_head;
-  e.rope_cols = ea->rope_cols;
-  e.M = M;
-  e.N = N;
-  const char* why = "";
-  const int rc = gemm_plan(p, &why);
-  if (rc) return fail(rc == -5 ? SGD_ERR_CUDA : (rc == -1 ? SGD_ERR_ARG : SGD_ERR_SHAPE), why);
-  if (p.sk_tiles > 0) {
-    int dev = 0;
-    CUDA_TRY(cudaGetDevice(&dev));
-    KernelWs* w = nullptr;
-    const int wrc = kernel_ws(dev, stream, gemm_ws_floats(p), p.sk_tiles, &w);
-    if (wrc) return wrc;
-    p.ws_ref = &w->ws;
-    p.cnt_ref = &w->cnt;
-    // a launch that stopped on an expired wait can leave counters behind; start from zero
-    CUDA_TRY(cudaMemsetAsync(w->cnt, 0, sizeof(int) * p.sk_tiles, static_cast<cudaStream_t>(stream)));
-  }
-  CUDA_TRY(gemm_launch(p, static_cast<cudaStream_t>(stream)));
-  return SGD_OK;
-}
-
-int sgd_kernel_gemm_static_ws(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
-                              const sgd_epilogue_args* ea, int variant, void* stream) {
+// The kernel-level GEMM arguments as a validated plan (variant codes: sgd_kernel_gemm);
+// returns an sgd_status.  Nothing touches the device before the checks pass.
+int kernel_gemm_plan(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
+                     const sgd_epilogue_args* ea, int variant, GemmPlan& p) {
   if (!ea) return fail(SGD_ERR_ARG, "null epilogue");
   if (ea->kind < 0 || ea->kind > SGD_EPI_ROPE) return fail(SGD_ERR_ARG, "bad epilogue kind");
   if (variant < 0 || variant > 10) return fail(SGD_ERR_ARG, "gemm: variant must be in 0..10");
-  GemmPlan p;
   p.A = H16(A);
   p.lda = lda;
   p.B = H16(B);
@@ -1570,6 +1508,37 @@ int sgd_kernel_gemm_static_ws(const void* A, int lda, const void* B, int ldb, in
   const char* why = "";
   const int rc = gemm_plan(p, &why);
   if (rc) return fail(rc == -5 ? SGD_ERR_CUDA : (rc == -1 ? SGD_ERR_ARG : SGD_ERR_SHAPE), why);
+  return SGD_OK;
+}
+
+}  // namespace
+
+int sgd_kernel_gemm(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
+                    const sgd_epilogue_args* ea, int use_simt, void* stream) {
+  GemmPlan p;
+  const int rc = kernel_gemm_plan(A, lda, B, ldb, M, N, K, ea, use_simt, p);
+  if (rc) return rc;
+  if (p.sk_tiles > 0) {
+    int dev = 0;
+    CUDA_TRY(cudaGetDevice(&dev));
+    KernelWs* w = nullptr;
+    const int wrc = kernel_ws(dev, stream, gemm_ws_floats(p), p.sk_tiles, &w);
+    if (wrc) return wrc;
+    p.ws_ref = &w->ws;
+    p.cnt_ref = &w->cnt;
+    // a launch that stopped on an expired wait can leave counters behind; start from zero
+    CUDA_TRY(cudaMemsetAsync(w->cnt, 0, sizeof(int) * p.sk_tiles, static_cast<cudaStream_t>(stream)));
+  }
+  CUDA_TRY(gemm_launch(p, static_cast<cudaStream_t>(stream)));
+  return SGD_OK;
+}
+
+int sgd_kernel_gemm_static_ws(const void* A, int lda, const void* B, int ldb, int M, int N, int K,
+                              const sgd_epilogue_args* ea, int variant, void* stream) {
+  GemmPlan p;
+  const int rc = kernel_gemm_plan(A, lda, B, ldb, M, N, K, ea, variant, p);
+  if (rc) return rc;
+  const char* why = "";
   float* ws = nullptr;
   int* tickets = nullptr;
   if (p.sk_tiles > 0) {
