@@ -220,8 +220,9 @@ SGD_API int sgd_step_host(sgd_ctx* ctx, const void* state_in_host, void* out_hos
  * step are queued on `stream`, the output copy on a library-owned copy stream, so the
  * copy of step s overlaps the compute of step s + 1 (the device output is
  * double-buffered).  in_host / out_host should be pinned; in_host must stay unchanged
- * until the step's input copy has run and out_host must not be read (or reused for
- * another step) until sgd_host_wait returns.
+ * until the step's input copy has run, and out_host must not be read until
+ * sgd_host_wait returns.  Output copies run in call order on the one copy stream, so a
+ * later step may name the same out_host: its copy lands after the earlier one.
  */
 SGD_API int sgd_step_host_async(sgd_ctx* ctx, const void* state_in_host, void* out_host,
                                 float timestep, const int32_t* class_ids_host, const void* ctx_host,
