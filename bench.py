@@ -118,14 +118,17 @@ class ClockSampler:
 
 
 def dist_setup(n_gpus):
+    """Rank, world size and local rank from the launcher's environment; for N > 1 one process
+    group over NCCL (gloo when no GPU is visible, as in the CPU tests of this path)."""
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if world > 1:
         import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl")
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
     elif torch.cuda.is_available():
         torch.cuda.set_device(0)
     return rank, world, local
@@ -138,11 +141,13 @@ def barrier(world):
 
 
 def max_over_ranks(x, world):
+    """The largest of every rank's x (the slowest rank's time sets the job's time)."""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
 
