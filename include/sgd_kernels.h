@@ -137,6 +137,16 @@ SGD_API int sgd_kernel_frozen_run(float* h, const void* const* caches_host, int 
 /* Device status word shared by all kernels (bounded-wait expiry); returns and clears it. */
 SGD_API int sgd_kernel_status(int* status_host);
 
+/*
+ * Failure-path self-test (no counterpart in the paper): launches on `stream` one kernel
+ * whose thread waits, with the same bounded wait every kernel uses, on an mbarrier that
+ * nothing completes.  After the wait limit (2 s) it records SGD_SELFTEST_TIMEOUT_CODE in
+ * the device status word (read and cleared by sgd_kernel_status) and returns, leaving the
+ * context usable.  Nothing faults, traps or hangs.
+ */
+#define SGD_SELFTEST_TIMEOUT_CODE 99
+SGD_API int sgd_selftest_wait_timeout(void* stream);
+
 #ifdef __cplusplus
 }
 #endif

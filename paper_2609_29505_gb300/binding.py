@@ -29,6 +29,7 @@ SGD_ERR_CUDA = -5
 SGD_ERR_DEVICE_TIMEOUT = -6
 SGD_ERR_OOM = -7
 SGD_ERR_STATE = -8
+SGD_SELFTEST_TIMEOUT_CODE = 99  # status code recorded by sgd_selftest_wait_timeout
 
 STEM = {"time_add": 0, "patch": 1, "patch_tokens": 2, "identity": 3, "embed": 4}
 BLOCK = {"prenorm": 0, "adaln": 1, "xattn": 2}
@@ -50,7 +51,7 @@ EXPORTED = [
     "sgd_compile_schedule", "sgd_step_profile", "sgd_sampler_update", "sgd_kernel_gemm",
     "sgd_kernel_attention", "sgd_kernel_norm", "sgd_kernel_frozen_run", "sgd_kernel_status",
     "sgd_set_exec_mode", "sgd_step_host_async", "sgd_host_wait", "sgd_kernel_gemm_static_ws",
-    "sgd_set_policy", "sgd_get_drift",
+    "sgd_set_policy", "sgd_get_drift", "sgd_selftest_wait_timeout",
 ]
 EXEC_JAGGED_GRAPH, EXEC_EAGER, EXEC_PADDED_GRAPH = 0, 1, 2
 POLICY_STATIC, POLICY_DRIFT = 0, 1
@@ -140,6 +141,7 @@ def lib() -> C.CDLL:
             "sgd_step_host_async": (i, [vp, vp, vp, f, vp, vp, i, vp]),
             "sgd_host_wait": (i, [vp]),
             "sgd_set_policy": (i, [vp, i]),
+            "sgd_selftest_wait_timeout": (i, [vp]),
             "sgd_get_drift": (i, [vp, i, vp, i]),
         }
         for name, (res, args) in sig.items():

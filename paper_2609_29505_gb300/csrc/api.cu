@@ -1601,6 +1601,13 @@ int sgd_kernel_frozen_run(float* h, const void* const* caches, int n_caches, int
   return SGD_OK;
 }
 
+int sgd_selftest_wait_timeout(void* stream) {
+  int* p = device_status_ptr();
+  if (!p) return fail(SGD_ERR_CUDA, "status word unavailable");
+  CUDA_TRY(wait_selftest_launch(p, SGD_SELFTEST_TIMEOUT_CODE, static_cast<cudaStream_t>(stream)));
+  return SGD_OK;
+}
+
 int sgd_kernel_status(int* status_host) {
   if (!status_host) return fail(SGD_ERR_ARG, "null argument");
   int* p = device_status_ptr();

@@ -237,6 +237,21 @@ __global__ void drift_reduce_kernel(const float* partials, double* sums) {
   }
 }
 
+// Failure-path self-test: thread 0 waits, with the kernels' bounded wait, on an mbarrier
+// whose phase nothing completes; after the wait limit it records `code` in the device
+// status word and returns.  Used to test the timeout path without faulting the GPU.
+__global__ void wait_selftest_kernel(int* status, int code) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) mbar_wait(&bar, 0, &abort_flag, status, code);
+}
+
 __global__ void __launch_bounds__(256) frozen_kernel(const __grid_constant__ FrozenParams p) {
   const int64_t n8 = p.n >> 3;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -497,6 +512,11 @@ cudaError_t norm_launch(const NormParams& p, cudaStream_t s) {
     norm_warp_kernel<<<(p.rows + 7) / 8, 256, 0, s>>>(p);
   else
     norm_kernel<<<p.rows, kNormThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t wait_selftest_launch(int* status, int code, cudaStream_t s) {
+  wait_selftest_kernel<<<1, 32, 0, s>>>(status, code);
   return cudaGetLastError();
 }
 

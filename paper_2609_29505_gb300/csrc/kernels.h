@@ -142,6 +142,8 @@ struct DriftParams {
   float* partial;  // [kDriftBlocks][2]
 };
 cudaError_t drift_launch(const DriftParams& p, cudaStream_t s);
+// One thread waits (bounded) on an mbarrier nothing completes and records `code`.
+cudaError_t wait_selftest_launch(int* status, int code, cudaStream_t s);
 cudaError_t drift_reduce_launch(const float* partials, int n_groups, double* sums, cudaStream_t s);
 
 // Per-step I/O slot (device memory) read by graph kernels.
