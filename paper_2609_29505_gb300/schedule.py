@@ -227,3 +227,82 @@ def build_schedule(cfg, weights, T: int, budget: Optional[float] = None,
     return dict(lifetimes=S_u.astype(np.int32), groups=groups.astype(np.int32),
                 group_lifetimes=S_g, tau=tau, lam=lam, branch_scores=np.asarray(branch_q),
                 ratio=float(S_g.sum()) / (len(S_g) * T), feasible=feasible, s_min=s_min, T=T)
+
+
+# ---------------------------------------------------------------------------
+# persistence: a schedule is the only state worth keeping across runs (caches are
+# per-trajectory scratch; a resumed run restarts at s = 1)
+# ---------------------------------------------------------------------------
+
+SCHEDULE_FORMAT = 1
+
+
+def weights_digest(weights) -> str:
+    """sha256 over every weight tensor's name, shape, dtype and two exact integer checksums of
+    its raw 16-bit words (a plain sum and a position-weighted sum), computed where the tensor
+    lives in chunks, so a digest of device-resident weights needs no host copy."""
+    import hashlib
+
+    import torch
+
+    h = hashlib.sha256()
+    for name in sorted(weights):
+        t = weights[name]
+        if not _is_torch(t):
+            t = torch.from_numpy(np.ascontiguousarray(t))
+        v = t.detach().contiguous().reshape(-1)
+        if v.element_size() == 2:
+            v = v.view(torch.int16)
+        elif v.element_size() == 4:
+            v = v.view(torch.int32)
+        s1 = s2 = 0
+        chunk = 1 << 24
+        for i in range(0, v.numel(), chunk):
+            x = v[i:i + chunk].to(torch.int64)
+            pos = torch.arange(i, i + x.numel(), device=x.device, dtype=torch.int64) % 65521 + 1
+            s1 += int(x.sum())
+            s2 += int(((x + 65537) * pos).sum())
+        h.update(f"{name}|{tuple(t.shape)}|{t.dtype}|{s1}|{s2};".encode())
+    return h.hexdigest()
+
+
+def save_schedule(path: str, sched: Dict, cfg, weights=None, eta: float = ETA,
+                  ranking: str = "scr", granularity: str = "block") -> None:
+    """Write a schedule from build_schedule (lifetimes, groups, tau, T, S_min, achieved
+    ratio) with the knobs that produced it, the model config's name and, when the weights
+    are given, their digest."""
+    import json
+    doc = {
+        "format": SCHEDULE_FORMAT, "config": cfg.name, "n_units": int(cfg.n_units),
+        "T": int(sched["T"]), "tau": float(sched["tau"]), "eta": float(eta),
+        "s_min": int(sched["s_min"]), "ratio": float(sched["ratio"]),
+        "feasible": bool(sched["feasible"]), "ranking": ranking, "granularity": granularity,
+        "lifetimes": [int(x) for x in sched["lifetimes"]],
+        "groups": [int(x) for x in sched["groups"]],
+        "weights_digest": weights_digest(weights) if weights is not None else None,
+    }
+    with open(path, "w") as f:
+        json.dump(doc, f, indent=1)
+
+
+def load_schedule(path: str, cfg=None, weights=None) -> Dict:
+    """Read a saved schedule; with `cfg` it must match the model's name and unit count, with
+    `weights` their digest (ValueError otherwise).  Returns the fields as build_schedule
+    names them (lifetimes and groups as int32 arrays)."""
+    import json
+    with open(path) as f:
+        doc = json.load(f)
+    if doc.get("format") != SCHEDULE_FORMAT:
+        raise ValueError(f"unknown schedule format {doc.get('format')}")
+    if cfg is not None and (doc["config"] != cfg.name or doc["n_units"] != cfg.n_units):
+        raise ValueError(f"schedule for {doc['config']} ({doc['n_units']} units), "
+                         f"model is {cfg.name} ({cfg.n_units} units)")
+    if weights is not None:
+        if doc["weights_digest"] is None:
+            raise ValueError("schedule was saved without a weights digest")
+        if weights_digest(weights) != doc["weights_digest"]:
+            raise ValueError("weights differ from the ones the schedule was computed from")
+    out = dict(doc)
+    out["lifetimes"] = np.asarray(doc["lifetimes"], dtype=np.int32)
+    out["groups"] = np.asarray(doc["groups"], dtype=np.int32)
+    return out
