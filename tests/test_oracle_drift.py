@@ -168,3 +168,34 @@ def test_forced_routing_reproduces_the_policy():
     for x, y in zip(a["outputs"], b["outputs"]):
         np.testing.assert_array_equal(x, y)
     assert a["drift"][2:] == b["drift"][2:]
+
+
+def test_deep_block_input_is_taken_after_the_skip_combine():
+    """Reading of App. B.1 for U-ViT: a deep block's drift input is the stream after its long
+    skip is combined, W_skip [h ; skip], recomputed here from the traced stream before the
+    combine and the pushed shallow-block output."""
+    cfg = synth.get_config("uvit_small").with_(n_blocks=3, n_skips=1, d=32, n_heads=2, d_head=16,
+                                                d_ff=64, batch=1, n_tokens=6, T=4, n_classes=4)
+    w = dn.to_numpy_weights(synth.make_weights(cfg, "cpu"))
+    inp = synth.make_inputs(cfg, "cpu")
+    S = [4] * cfg.n_units
+    groups = list(np.repeat(np.arange(cfg.n_blocks), len(cfg.branches)))
+    res = dr.run(cfg, w, S, groups, cfg.T, z0=inp.z0.numpy(), class_ids=inp.class_ids.numpy())
+    nb = len(cfg.branches)
+    cache, ins = {}, []
+    for s in range(1, cfg.T + 1):
+        tr = dn.Trace()
+        dn.denoise(cfg, w, res["states"][s - 1], tj.timestep(cfg.T, s), s, S, cache,
+                   inp.class_ids.numpy(), trace=tr)
+        ins.append(tr.units)
+    for s in range(3, cfg.T + 1):
+        d = []
+        for step in (s - 1, s - 2):
+            units = ins[step - 1]
+            skip = units[nb * 1 - 1][3]          # shallow block 0's output (pushed)
+            before = units[nb * 2 - 1][3]        # stream after the middle block
+            d.append(dn.skip_combine(w, 0, before, skip))
+            np.testing.assert_allclose(units[nb * 2][2], d[-1], rtol=0, atol=0)
+        a, b = d[0].astype(np.float64), d[1].astype(np.float64)
+        want = np.linalg.norm(a - b) / (np.linalg.norm(a) + 1e-8)
+        assert res["drift"][s - 1][2] == pytest.approx(want, rel=1e-12)
