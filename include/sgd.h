@@ -97,8 +97,7 @@ typedef enum {
 #define SGD_FLAG_SIMT_GEMM 1
 /* Run every attention on the mma.sync kernel instead of tcgen05 (d_head 64 / 128). */
 #define SGD_FLAG_MMA_SYNC_ATTENTION 2
-/* Run the tcgen05 GEMMs as 2-CTA clusters that multicast the shared B tile. */
-#define SGD_FLAG_GEMM_CLUSTER2 4
+/* (Flag bit 4 is not defined; sgd_create rejects it.) */
 /* Use 64-element K-blocks (4 stages, 128-byte swizzle) in the tcgen05 GEMMs. */
 #define SGD_FLAG_GEMM_BK64 8
 

@@ -70,10 +70,9 @@ typedef struct {
  * TMEM) with 64-element K-blocks, choosing by itself 128 x 256 or 128 x 128 tiles, 4 or 8
  * epilogue warps, and whether the tiles left over after the last full wave of CTAs are
  * split along K over all SMs ("stream-K": fp32 partial tiles in a workspace, summed in a
- * fixed order by the CTA that finishes a tile last, so results are deterministic); 2 the
- * same kernel as 2-CTA clusters in which vertically adjacent tiles share one multicast
- * load of their B tile; 3 and 4 the forms of 0 and 2 with 32-element K-blocks (64-byte
- * swizzle); 5, 6, 7 force 128 x 256 tiles with 4 epilogue warps, 128 x 256 with 8, and
+ * fixed order by the CTA that finishes a tile last, so results are deterministic); 3 the
+ * form of 0 with 32-element K-blocks (64-byte swizzle); 2 and 4 are not defined and are
+ * rejected with SGD_ERR_ARG; 5, 6, 7 force 128 x 256 tiles with 4 epilogue warps, 128 x 256 with 8, and
  * 128 x 128 with 8 and no stream-K (128 x 128 applies to plain, GELU and DELTA epilogues
  * only); 8 is 0 without stream-K, 9 is 0 with stream-K whenever the last wave is partial;
  * 10 forces 128 x 224 tiles (5 pipeline stages, no stream-K; plain, GELU and DELTA only).

@@ -38,7 +38,6 @@ MLP = {"swiglu": 0, "gelu_tanh": 1, "gelu_erf": 2, "geglu": 3}
 HEAD = {"linear": 0, "adaln_linear": 1, "identity": 2, "logits": 3}
 FLAG_SIMT_GEMM = 1
 FLAG_MMA_SYNC_ATTENTION = 2
-FLAG_GEMM_CLUSTER2 = 4
 FLAG_GEMM_BK64 = 8
 
 EPI_F16, EPI_F32, EPI_DELTA, EPI_GATED, EPI_GELU, EPI_ROPE = range(6)

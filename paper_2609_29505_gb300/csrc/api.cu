@@ -259,7 +259,6 @@ int make_gemm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, cons
   plan->K = K;
   plan->epi = epi;
   plan->simt = (c->d.flags & SGD_FLAG_SIMT_GEMM) != 0;
-  plan->cluster = (c->d.flags & SGD_FLAG_GEMM_CLUSTER2) ? 2 : 1;
   plan->bk = (c->d.flags & SGD_FLAG_GEMM_BK64) ? 64 : c->gemm_bk;
   const char* why = "";
   if (gemm_plan(*plan, &why) != 0) return fail(SGD_ERR_SHAPE, std::string(name) + ": " + why);
@@ -922,6 +921,8 @@ const char* sgd_last_error(void) { return g_err.c_str(); }
 int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out) {
   if (!desc || !w || !out) return fail(SGD_ERR_ARG, "null argument");
   *out = nullptr;
+  if (desc->flags & ~(SGD_FLAG_SIMT_GEMM | SGD_FLAG_MMA_SYNC_ATTENTION | SGD_FLAG_GEMM_BK64))
+    return fail(SGD_ERR_ARG, "unknown flag bits");
   int rc = check_shape(*desc, *w);
   if (rc) return rc;
   auto* c = new (std::nothrow) sgd_ctx();
@@ -1467,7 +1468,8 @@ int kernel_gemm_plan(const void* A, int lda, const void* B, int ldb, int M, int 
                      const sgd_epilogue_args* ea, int variant, GemmPlan& p) {
   if (!ea) return fail(SGD_ERR_ARG, "null epilogue");
   if (ea->kind < 0 || ea->kind > SGD_EPI_ROPE) return fail(SGD_ERR_ARG, "bad epilogue kind");
-  if (variant < 0 || variant > 10) return fail(SGD_ERR_ARG, "gemm: variant must be in 0..10");
+  if (variant < 0 || variant > 10 || variant == 2 || variant == 4)
+    return fail(SGD_ERR_ARG, "gemm: variant must be 0, 1, 3 or 5..10");
   p.A = H16(A);
   p.lda = lda;
   p.B = H16(B);
@@ -1476,8 +1478,7 @@ int kernel_gemm_plan(const void* A, int lda, const void* B, int ldb, int M, int 
   p.N = N;
   p.K = K;
   p.simt = variant == 1;
-  p.cluster = (variant == 2 || variant == 4) ? 2 : 1;
-  p.bk = (variant == 3 || variant == 4) ? 32 : 64;
+  p.bk = variant == 3 ? 32 : 64;
   if (variant == 5) { p.bn = 256; p.epiw = 4; }
   if (variant == 6) { p.bn = 256; p.epiw = 8; }
   if (variant == 7) { p.bn = 128; p.epiw = 8; p.sk = 0; }

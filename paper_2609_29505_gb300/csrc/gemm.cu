@@ -478,26 +478,20 @@ __device__ __forceinline__ void unit_at(const TcArgs& a, const CtaWork& w, int u
   }
 }
 
-// CLUSTER = 2: the two CTAs of a cluster compute vertically adjacent 128-row tiles of
-// the same 256 output columns; each loads its own A box and one of the two B halves,
-// multicast into both CTAs, so every B byte is read from L2 once per pair.  Each CTA's
-// MMA commits the release of a stage to both CTAs (empty barriers count 2 arrivals).
-//
-// Stream-K (CLUSTER = 1, sk_tiles > 0): the K iterations of the first sk_tiles tiles are
+// Stream-K (sk_tiles > 0): the K iterations of the first sk_tiles tiles are
 // spread evenly over sk_ctas CTAs (at most kMaxSeg per tile), so that the tiles left over
 // after the last full wave do not leave most SMs idle.  A CTA whose segment does not cover
 // a tile's whole K range stores its raw accumulator in its workspace slot, then draws a
 // ticket from the tile's counter; the CTA that draws the last ticket sums the slots in
 // order, runs the epilogue and puts the counter back to zero.  No CTA ever waits for
 // another.
-template <int CLUSTER, int BK, int BN, int EPIW>
+template <int BK, int BN, int EPIW>
 __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ TcArgs a) {
   using C = TileCfg<BK, BN, EPIW>;
   constexpr int kBK = C::kBK, kStages = C::kStages, kTileA = C::kTileA;
   constexpr int kTileBHalf = C::kTileBHalf, kStageBytes = C::kStageBytes;
   constexpr int kBN = C::kBN, kTmemCols = C::kTmemCols, kEpiWarps = C::kEpiWarps;
-  static_assert(CLUSTER == 1 || BN == 256, "multicast splits a 256-row B tile");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -514,12 +508,10 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
-  const uint32_t crank = CLUSTER > 1 ? cluster_ctarank() : 0;
-  const uint16_t cmask = static_cast<uint16_t>((1u << CLUSTER) - 1u);
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], CLUSTER);
+      mbar_init(&empty[s], 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull[i], 1);
@@ -538,12 +530,10 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (CLUSTER > 1) cluster_sync();  // the peer's barriers exist before any multicast lands
   const uint32_t tmem_base = *tmem_slot;
-  // work units: CLUSTER vertically adjacent tiles that share their B columns
-  const int num_mu = (a.num_m + CLUSTER - 1) / CLUSTER;
+  const int num_mu = a.num_m;
   const int num_tiles = num_mu * a.num_n;
-  const CtaWork w = cta_work(a, num_tiles, blockIdx.x / CLUSTER, gridDim.x / CLUSTER);
+  const CtaWork w = cta_work(a, num_tiles, blockIdx.x, gridDim.x);
 
   if (warp == 0) {
     if (lane == 0) {
@@ -551,7 +541,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
       for (int u = 0; u < w.n_units; ++u) {
         int tile, k0, k1;
         unit_at(a, w, u, tile, k0, k1);
-        const int m_blk = (tile % num_mu) * CLUSTER + crank, n_blk = tile / num_mu;
+        const int m_blk = tile % num_mu, n_blk = tile / num_mu;
         const int rb0 = a.gated ? n_blk * 128 : n_blk * kBN;
         const int rb1 = a.gated ? a.N + n_blk * 128 : rb0 + 128;  // BN = 256 only
         bool ok = true;
@@ -565,13 +555,8 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
           uint8_t* st = tiles + s * kStageBytes;
           mbar_arrive_expect_tx(&full[s], kStageBytes);
           tma_load_2d(st, &a.tmap_a, &full[s], kb * kBK, m_blk * kBM);
-          if (CLUSTER == 1) {
-            tma_load_2d(st + kTileA, &a.tmap_b, &full[s], kb * kBK, rb0);
-            if (kBN == 256) tma_load_2d(st + kTileA + kTileBHalf, &a.tmap_b, &full[s], kb * kBK, rb1);
-          } else {
-            tma_load_2d_mc(st + kTileA + crank * kTileBHalf, &a.tmap_b, &full[s], kb * kBK,
-                           crank ? rb1 : rb0, cmask);
-          }
+          tma_load_2d(st + kTileA, &a.tmap_b, &full[s], kb * kBK, rb0);
+          if (kBN == 256) tma_load_2d(st + kTileA + kTileBHalf, &a.tmap_b, &full[s], kb * kBK, rb1);
         }
         if (!ok) break;
       }
@@ -609,10 +594,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
             umma_f16(d_tmem, operand_desc<BK>(a_addr + 32 * k), operand_desc<BK>(b_addr + 32 * k),
                       idesc, (kb != k0 || k != 0) ? 1u : 0u);
           }
-          if (CLUSTER == 1)
-            umma_commit(&empty[s]);
-          else
-            umma_commit_mc(&empty[s], cmask);
+          umma_commit(&empty[s]);
         }
         if (!ok) break;
         umma_commit(&tfull[acc]);
@@ -640,7 +622,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
     for (int u = 0; u < w.n_units; ++u) {
       int tile, k0, k1;
       unit_at(a, w, u, tile, k0, k1);
-      const int m_blk = (tile % num_mu) * CLUSTER + crank, n_blk = tile / num_mu;
+      const int m_blk = tile % num_mu, n_blk = tile / num_mu;
       const int acc = u & 1;
       const uint32_t aph = (u >> 1) & 1;
       const int row = m_blk * kBM + q * 32 + lane;
@@ -700,8 +682,6 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
-  // no CTA leaves while its peer may still arrive on its barriers or write its tiles
-  if (CLUSTER > 1) cluster_sync();
   tc_fence_after();
   if (warp == 1) {
     __syncwarp();
@@ -886,40 +866,6 @@ int* device_status_ptr() {
   return ptr[dev];
 }
 
-// Clusters of two that can be resident at once (pairs must share a GPC), cached per device.
-template <int BK>
-int max_active_pairs() {
-  constexpr int kSmemBytes = TileCfg<BK>::kSmemBytes;
-  constexpr int kThreads = TileCfg<BK>::kThreads;
-  static int cached[64] = {0};
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev < 0 || dev >= 64) return 0;
-  if (!cached[dev]) {
-    if (cudaFuncSetAttribute(gemm_tc_kernel<2, BK, 256, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kSmemBytes) != cudaSuccess)
-      return 0;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(2);
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = kSmemBytes;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 2;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<2, BK, 256, 8>, &cfg) != cudaSuccess || n < 1) {
-      cudaGetLastError();
-      n = -1;
-    }
-    cached[dev] = n;
-  }
-  return cached[dev] > 0 ? cached[dev] : 0;
-}
-
 // Stream-K split of the tiles left after the last full wave of `sms` CTAs: their
 // tiles * num_k K iterations go to up to `sms` CTAs, at least a third of a tile's K range
 // each, so that no tile is shared by more than kMaxSeg = 4 CTAs.  Measured on GB300 under
@@ -992,13 +938,12 @@ int gemm_plan(GemmPlan& p, const char** why) {
   const int num_m = (p.M + kBM - 1) / kBM;
   const int sms = num_sms();
   const int num_k = (p.K + p.bk - 1) / p.bk;
-  if (p.cluster != 1 && p.cluster != 2) p.cluster = 1;
   // tile shape: 128-column tiles when they need clearly fewer tile-times than 256-column
   // tiles (a 128-column tile takes half the time of a 256-column one, at about 3/4 of its
   // efficiency, so: 2 * waves_128 < 3 * waves_256) and stream-K does not already even out
   // the last wave; they need a plain epilogue and one-CTA launches.  4 epilogue warps for
   // RoPE and gated epilogues.
-  const bool small_ok = !gated && e.kind != SGD_EPI_ROPE && p.bk == 64 && p.cluster == 1;
+  const bool small_ok = !gated && e.kind != SGD_EPI_ROPE && p.bk == 64;
   // 128 x 224 tiles where they fill whole waves exactly, K is long and the last column of
   // tiles wastes under a tenth of N (e.g. M = N = 4096 at K >= 3072: 608 tiles = 4 waves;
   // measured 1266 against 1233 TFLOP/s for 128 x 256 with stream-K)
@@ -1011,32 +956,23 @@ int gemm_plan(GemmPlan& p, const char** why) {
     const int w256 = (t256 + sms - 1) / sms;
     const int w128 = (num_m * ((p.N + 127) / 128) + sms - 1) / sms;
     SkSplit sk256 = sk_split(t256, num_k, sms);
-    const bool sk_on = p.cluster == 1 && p.sk != 0 && sk256.tiles > 0;
+    const bool sk_on = p.sk != 0 && sk256.tiles > 0;
     p.bn = (small_ok && !sk_on && 2 * w128 < 3 * w256) ? 128 : 256;
   }
   if ((p.bn != 128 && p.bn != 224) || !small_ok) p.bn = 256;
   if (p.bn == 224) p.sk = 0;
   if (p.epiw == 0) p.epiw = (e.kind == SGD_EPI_ROPE || gated) ? 4 : 8;
-  if (p.bn == 128 || p.bn == 224 || p.cluster == 2 || p.bk == 32) p.epiw = 8;
+  if (p.bn == 128 || p.bn == 224 || p.bk == 32) p.epiw = 8;
   if (!make_tmap_f16(&p.tmap_a, p.A, p.M, p.K, p.lda, 128, p.bk) ||
       !make_tmap_f16(&p.tmap_b, p.B, b_rows, p.K, p.ldb, p.bn == 224 ? 224 : 128, p.bk)) {
     *why = "gemm: cuTensorMapEncodeTiled failed (driver entry point unavailable or bad layout)";
     return -5;
   }
   const int num_n = gated ? (p.N + 127) / 128 : (p.N + p.bn - 1) / p.bn;
-  if (p.cluster == 2 && num_m < 2) p.cluster = 1;  // nothing to share
-  int max_units = sms;
-  if (p.cluster == 2) {
-    max_units = p.bk == 32 ? max_active_pairs<32>() : max_active_pairs<64>();
-    if (max_units < 1) {
-      p.cluster = 1;
-      max_units = sms;
-    }
-  }
-  const int units = ((num_m + p.cluster - 1) / p.cluster) * num_n;
-  p.grid = (units < max_units ? units : max_units) * p.cluster;
+  const int units = num_m * num_n;
+  p.grid = units < sms ? units : sms;
   p.sk_tiles = p.sk_ctas = p.max_seg = 0;
-  if (p.cluster == 1 && p.sk != 0) {
+  if (p.sk != 0) {
     const SkSplit k = sk_split(units, num_k, sms, p.sk == 1);
     if (k.tiles > 0) {
       p.sk_tiles = k.tiles;
@@ -1052,7 +988,7 @@ size_t gemm_ws_floats(const GemmPlan& p) {
   return p.sk_tiles > 0 ? static_cast<size_t>(p.sk_tiles) * p.max_seg * kBM * p.bn : 0;
 }
 
-template <int CLUSTER, int BK, int BN, int EPIW>
+template <int BK, int BN, int EPIW>
 cudaError_t launch_tc(const GemmPlan& p, const TcArgs& a, cudaStream_t s) {
   constexpr int kSmemBytes = TileCfg<BK, BN, EPIW>::kSmemBytes;
   constexpr int kThreads = TileCfg<BK, BN, EPIW>::kThreads;
@@ -1060,27 +996,12 @@ cudaError_t launch_tc(const GemmPlan& p, const TcArgs& a, cudaStream_t s) {
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<CLUSTER, BK, BN, EPIW>,
+    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<BK, BN, EPIW>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (err != cudaSuccess) return err;
     attr_done[dev] = true;
   }
-  if (CLUSTER == 2) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(p.grid);
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = kSmemBytes;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 2;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<CLUSTER, BK, BN, EPIW>, a);
-  }
-  gemm_tc_kernel<CLUSTER, BK, BN, EPIW><<<p.grid, kThreads, kSmemBytes, s>>>(a);
+  gemm_tc_kernel<BK, BN, EPIW><<<p.grid, kThreads, kSmemBytes, s>>>(a);
   return cudaGetLastError();
 }
 
@@ -1110,13 +1031,12 @@ cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s) {
   a.max_seg = p.max_seg;
   a.ws = p.ws_ref ? *p.ws_ref : nullptr;
   a.sk_cnt = p.cnt_ref ? *p.cnt_ref : nullptr;
-  if (p.sk_tiles > 0 && (!a.ws || !a.sk_cnt || p.cluster != 1)) return cudaErrorInvalidValue;
+  if (p.sk_tiles > 0 && (!a.ws || !a.sk_cnt)) return cudaErrorInvalidValue;
   if (p.bk == 32)
-    return p.cluster == 2 ? launch_tc<2, 32, 256, 8>(p, a, s) : launch_tc<1, 32, 256, 8>(p, a, s);
-  if (p.cluster == 2) return launch_tc<2, 64, 256, 8>(p, a, s);
-  if (p.bn == 128) return launch_tc<1, 64, 128, 8>(p, a, s);
-  if (p.bn == 224) return launch_tc<1, 64, 224, 8>(p, a, s);
-  return p.epiw == 4 ? launch_tc<1, 64, 256, 4>(p, a, s) : launch_tc<1, 64, 256, 8>(p, a, s);
+    return launch_tc<32, 256, 8>(p, a, s);
+  if (p.bn == 128) return launch_tc<64, 128, 8>(p, a, s);
+  if (p.bn == 224) return launch_tc<64, 224, 8>(p, a, s);
+  return p.epiw == 4 ? launch_tc<64, 256, 4>(p, a, s) : launch_tc<64, 256, 8>(p, a, s);
 }
 
 }  // namespace sgd

@@ -49,7 +49,6 @@ struct GemmPlan {
   int M = 0, N = 0, K = 0;   // N = output columns
   EpiParams epi{};
   bool simt = false;
-  int cluster = 1;           // 2: pairs of CTAs share (multicast) the B tile
   int bk = 64;               // K elements per stage: 64 (128-byte swizzle) or 32 (64-byte)
   int bn = 0;                // output columns per tile: 256, 128, or 0 = choose by tile count
   int epiw = 0;              // epilogue warps: 4, 8, or 0 = choose by epilogue kind

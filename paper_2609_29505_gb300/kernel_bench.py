@@ -108,9 +108,9 @@ def main():
     ap.add_argument("--epi", default="f16", choices=list(EPI))
     ap.add_argument("--store-cache", action="store_true")
     ap.add_argument("--simt", type=int, default=0,
-                    help="sgd_kernel_gemm variant: 0 tcgen05 (auto), 1 SIMT, 2 2-CTA multicast, 3 BK 32, "
-                         "4 BK 32 2-CTA, 5 4 epilogue warps, 6 8 warps, 7 128-column tiles, 8 no stream-K, "
-                         "9 stream-K forced")
+                    help="sgd_kernel_gemm variant: 0 tcgen05 (auto), 1 SIMT, 3 BK 32, "
+                         "5 4 epilogue warps, 6 8 warps, 7 128-column tiles, 8 no stream-K, "
+                         "9 stream-K forced, 10 128 x 224 tiles")
     ap.add_argument("--tokens", type=int, default=1024)
     ap.add_argument("--batch", type=int, default=4)
     ap.add_argument("--heads", type=int, default=32)
