@@ -4,8 +4,11 @@ Default workload: the LLaDA-8B-shaped masked-diffusion transformer (32 blocks,
 d 4096, 32 heads x 128, SwiGLU 12288, RMSNorm, RoPE, 126464-token head), batch 4 x
 1024 tokens, horizon T = 64, 50% layer-step budget from the SCR/Frobenius
 schedule.  A bench "step" is one denoiser evaluation (one sgd_step: stem, every
-active unit, frozen runs, head) at trajectory position s; timed steps run whole
-trajectories from s = 1, cycling every T steps.
+active unit, frozen runs, head) at trajectory position s.  The K timed steps are
+K // T whole trajectories plus, when K is not a multiple of T, K % T positions
+spread evenly over 1..T (the midpoints of K % T equal slices); every trajectory
+runs in order from s = 1 (the untimed steps in between fill the caches), and
+each run of consecutive timed steps sits between its own pair of CUDA events.
 
 Prints ONE JSON line (rank 0).  --impl reference times the CPU oracle instead.
 """
@@ -156,6 +159,27 @@ def max_over_ranks(x, world):
 # workload
 # ---------------------------------------------------------------------------
 
+def timed_plan(K, T):
+    """Trajectories of the timed region and, for each, its timed positions (1-based, in
+    order): K // T whole trajectories, then the midpoints of K % T equal slices of 1..T,
+    so that the timed steps sample the whole horizon and its active-set profile."""
+    full, rem = divmod(K, T)
+    plan = [list(range(1, T + 1)) for _ in range(full)]
+    if rem:
+        plan.append([int((i + 0.5) * T / rem) + 1 for i in range(rem)])
+    return plan
+
+
+def golden_module():
+    """tests/golden/full_size_schedules.py: the oracle's stored full-size schedules."""
+    import importlib.util
+    path = os.path.join(ROOT, "tests", "golden", "full_size_schedules.py")
+    spec = importlib.util.spec_from_file_location("sgd_full_size_schedules", path)
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    return mod
+
+
 def setup_workload(args, device):
     import torch
     from paper_2609_29505_gb300 import schedule, synth
@@ -232,21 +256,41 @@ def run_native(args):
     run_steps(W)
     torch.cuda.synchronize()
     model.check_device(stream)
-    # timed region: exactly K steps from s = 1
-    model.reset()
+    # timed region: exactly K steps (timed_plan), CUDA events around each run of
+    # consecutive timed steps; untimed steps between them only fill the caches
+    plan = timed_plan(K, T)
+    timed_pos = [s for traj in plan for s in traj]
     barrier(world)
     torch.cuda.synchronize()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    pairs = []
+    w0, w1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(dev.index if dev.index is not None else 0) as clk:
-        ev0.record(stream)
-        run_steps(K, start_fresh=False)
-        ev1.record(stream)
+        w0.record(stream)
+        for traj in plan:
+            model.reset()
+            tset = set(traj)
+            for s in range(1, max(traj) + 1):
+                if s in tset and s - 1 not in tset:
+                    e0 = torch.cuda.Event(enable_timing=True)
+                    e0.record(stream)
+                model.step(xs[s - 1], out, timestep(cfg, s, T), s, class_ids=cls, ctx=ctx, stream=stream)
+                if s in tset and s + 1 not in tset:
+                    e1 = torch.cuda.Event(enable_timing=True)
+                    e1.record(stream)
+                    pairs.append((e0, e1))
+        w1.record(stream)
         torch.cuda.synchronize()
     barrier(world)
-    ms = ev0.elapsed_time(ev1)
+    ms = sum(a.elapsed_time(b) for a, b in pairs)
     ms = max_over_ranks(ms, world)
+    region_ms = w0.elapsed_time(w1)
     model.check_device(stream)
     value = K * world / (ms / 1000.0)
+    n_groups = len(set(sched["groups"]))
+    group_S = {}
+    for g, S_u in zip(sched["groups"], sched["lifetimes"]):
+        group_S[int(g)] = int(S_u)
+    timed_ratio = sum(sum(1 for S_g in group_S.values() if S_g >= s) for s in timed_pos) / (K * n_groups)
 
     # per-op timing of one trajectory (same kernels, launched op by op with events)
     recs_by_step = []
@@ -255,12 +299,18 @@ def run_native(args):
         recs_by_step.append(model.profile_step(xs[s - 1], out, timestep(cfg, s, T), s,
                                                class_ids=cls, ctx=ctx, stream=stream))
     launches_per_pos = [len(r) + 1 for r in recs_by_step]  # + the per-step I/O-slot kernel
-    gpu_launches = sum(launches_per_pos[i % T] for i in range(K))
+    gpu_launches = sum(launches_per_pos[s - 1] for s in timed_pos)
     if cfg.block == "xattn":
-        gpu_launches += cfg.n_blocks * ((K + T - 1) // T)  # context K/V at each s = 1
+        gpu_launches += cfg.n_blocks * timed_pos.count(1)  # context K/V at each timed s = 1
+    # per-kernel sums over exactly the timed positions (with their multiplicity)
     by_kernel = {}
     tot_flops = tot_bytes = tot_ms = 0.0
-    for recs in recs_by_step:
+    t_roof_timed = 0.0
+    for s in timed_pos:
+        recs = recs_by_step[s - 1]
+        fl_s = sum(r["flops"] for r in recs)
+        by_s = sum(r["bytes"] for r in recs)
+        t_roof_timed += max(fl_s / (peaks["bf16_sus"] * 1e12), by_s / (peaks["hbm"] * 1e9))
         for r in recs:
             k = by_kernel.setdefault(r["kernel"], dict(ms=0.0, flops=0.0, bytes=0.0, launches=0))
             k["ms"] += r["ms"]
@@ -280,16 +330,25 @@ def run_native(args):
                 "traffic_unit": "DRAM bytes per launch (ncu launch list in profiles/, averaged over "
                                 "the step's GEMM launches)",
                 "algorithmic_bytes_per_launch": round(gemm["bytes"] / gemm["launches"]),
-                "launches_per_trajectory": gemm["launches"],
+                "launches_in_timed_steps": gemm["launches"],
+                "measured_over": "the timed positions, one eager op-by-op launch per op with "
+                                 "CUDA events (same kernels and launch configurations as the graphs)",
                 "share_of_step": round(gemm["ms"] / tot_ms, 3)}
     fz = by_kernel.get("frozen_run")
-    # whole-step roofline: max(FLOPs / bf16 peak, bytes / HBM peak) per step vs measured
-    t_roof = max(tot_flops / (peaks["bf16_sus"] * 1e12), tot_bytes / (peaks["hbm"] * 1e9)) / T
-    step_roof = {"t_roofline_ms": round(t_roof * 1e3, 3), "t_measured_ms": round(ms / K, 3),
-                 "frac": round(t_roof * 1e3 / (ms / K), 4),
-                 "flops_per_step": tot_flops / T, "bytes_per_step": tot_bytes / T,
-                 "roofline_steps_per_s": round(1.0 / t_roof, 2)}
-    kernels = {k: {"launches": v["launches"], "ms_per_traj": round(v["ms"], 3),
+    # step roofline over exactly the timed steps: sum over them of max(FLOPs / bf16 peak,
+    # bytes / HBM peak), against their measured time
+    traj_fl = sum(r["flops"] for recs in recs_by_step for r in recs)
+    traj_by = sum(r["bytes"] for recs in recs_by_step for r in recs)
+    t_roof_traj = sum(max(sum(r["flops"] for r in recs) / (peaks["bf16_sus"] * 1e12),
+                          sum(r["bytes"] for r in recs) / (peaks["hbm"] * 1e9)) for recs in recs_by_step)
+    step_roof = {"t_roofline_ms": round(t_roof_timed * 1e3 / K, 3), "t_measured_ms": round(ms / K, 3),
+                 "frac": round(t_roof_timed * 1e3 / ms, 4),
+                 "flops_per_step": tot_flops / K, "bytes_per_step": tot_bytes / K,
+                 "roofline_steps_per_s": round(K / t_roof_timed, 2),
+                 "over": "the K timed steps",
+                 "trajectory": {"flops_per_step": traj_fl / T, "bytes_per_step": traj_by / T,
+                                "roofline_steps_per_s": round(T / t_roof_traj, 2)}}
+    kernels = {k: {"launches": v["launches"], "ms_in_timed_steps": round(v["ms"], 3),
                    "share": round(v["ms"] / tot_ms, 4),
                    "tflops": round(v["flops"] / max(v["ms"], 1e-9) / 1e9, 1),
                    "gbs": round(v["bytes"] / max(v["ms"], 1e-9) / 1e6, 1)} for k, v in by_kernel.items()}
@@ -305,20 +364,23 @@ def run_native(args):
         outs_h = [out_buffer(cfg, "cpu", pinned=True) for _ in range(2)]
         cls_h = None if inp.class_ids is None else inp.class_ids.cpu().pin_memory()
         ctx_h = None if inp.ctx is None else inp.ctx.cpu().pin_memory()
-        model.reset()
+        n_e2e = len(plan) * T  # whole trajectories: every step of each, in order
         barrier(world)
         _t.cuda.synchronize()
         t0 = time.perf_counter()
-        for i in range(K):
+        for i in range(n_e2e):
             s = i % T + 1
+            if s == 1:
+                model.reset()
             model.step_host_async(xs_h[s - 1], outs_h[i % 2], timestep(cfg, s, T), s,
                                   class_ids_host=cls_h, ctx_host=ctx_h, stream=stream)
         model.host_wait()
         _t.cuda.synchronize()
         e2e_s = max_over_ranks(time.perf_counter() - t0, world)
         h2d = xs_h[0].numel() * xs_h[0].element_size() + (0 if cls_h is None else cls_h.numel() * 4)
-        e2e = {"value": round(K * world / e2e_s, 3), "unit": "steps/s", "h2d_bytes_per_step": int(h2d),
+        e2e = {"value": round(n_e2e * world / e2e_s, 3), "unit": "steps/s", "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(outs_h[0].numel() * outs_h[0].element_size()),
+               "steps": n_e2e, "over": f"{len(plan)} whole trajectory(ies) of T={T} steps",
                "api": "sgd_step_host_async + sgd_host_wait (output copy overlaps the next step)"}
 
     sweep = None
@@ -340,13 +402,16 @@ def run_native(args):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(cfg, T, weights, inp, sched, n_steps=8)
+        cpu = cpu_baseline(cfg, T, weights, inp, args.budget, n_steps=8)
 
     model.close()
     res = {
         "metric": METRIC if args.budget == 0.5 else METRIC.replace("50%", f"{args.budget:.0%}"),
         "value": round(value, 3), "unit": "steps/s", "n_gpus": world, "steps": K, "warmup": W,
         "ms_per_step": round(ms / K, 3), "higher_is_better": True, "scaling": "weak",
+        "timed_positions": timed_pos if len(timed_pos) <= 256 else None,
+        "timed_layer_step_ratio": round(timed_ratio, 4),
+        "timed_region_ms": round(region_ms, 2),
         "vs_baseline": None, "dtype": "f16", "data": "synthetic",
         "precision": "fp16 operands (bf16 weights converted exactly, power-of-two scaled), "
                      "fp32 accumulation and fp32 residual stream",
@@ -545,27 +610,41 @@ def workload_name(cfg, T, budget):
 TOKEN_SAMPLE = 128
 
 
-def oracle_sample(cfg, T, weights, inp, sched):
+def token_model_flops(cfg, n_active_blocks, batch, n_tokens):
+    """Dense FLOPs of one step of a token (pre-norm, gated-MLP) model with n_active_blocks
+    active blocks: per active block QKV, attention output, up and down projections
+    (2 n params) and non-causal attention (4 n^2 d); the vocabulary head at every step."""
+    d, f = cfg.d, cfg.d_ff
+    per_block = 2 * n_tokens * (4 * d * d + 3 * d * f) + 4 * n_tokens * n_tokens * d
+    return batch * (n_active_blocks * per_block + 2 * n_tokens * d * cfg.d_out)
+
+
+def oracle_sample(cfg, T, weights, inp):
     """Bounded sample of the workload for the CPU oracle: batch row 0 and, for token
     models, its first TOKEN_SAMPLE positions (full depth, width and head).  Returns the
-    oracle model config, fp32 weights, a state function and the scale factor from
-    sample steps/s to workload steps/s."""
-    import numpy as np
-    from oracle import denoiser as odn
+    oracle model config, fp32 weights, a state function, a function giving the workload's
+    FLOPs over the sample's FLOPs for a list of (position, active blocks), the class ids,
+    the context and a description."""
     from paper_2609_29505_gb300 import synth
     W = {k: v.detach().float().cpu().numpy() for k, v in weights.items()}
     if cfg.stem == "embed":
         n = min(TOKEN_SAMPLE, cfg.n_tokens)
         ocfg = cfg.with_(batch=1, n_tokens=n)
         state = lambda s: synth.token_ids_at(cfg, inp, s, T)[:1, :n].cpu().numpy()
-        scale = (n / cfg.n_tokens) / cfg.batch
-        desc = f"batch row 0 of {cfg.batch}, first {n} of {cfg.n_tokens} tokens, all layers"
+
+        def scale(active):
+            full = sum(token_model_flops(cfg, a, cfg.batch, cfg.n_tokens) for a in active)
+            samp = sum(token_model_flops(cfg, a, 1, n) for a in active)
+            return full / samp
+        desc = (f"batch row 0 of {cfg.batch}, first {n} of {cfg.n_tokens} tokens, all layers and "
+                f"the full head; scaled to the workload by its dense FLOPs (attention quadratic in "
+                f"tokens)")
     else:
         ocfg = cfg.with_(batch=1)
         z0 = inp.z0[:1].cpu().numpy()
         state = lambda s: z0
-        scale = 1.0 / cfg.batch
-        desc = f"batch row 0 of {cfg.batch}, all tokens and layers"
+        scale = lambda active: float(cfg.batch)  # samples are independent: exact
+        desc = f"batch row 0 of {cfg.batch}, all tokens and layers; scaled by the batch"
     cls = None if inp.class_ids is None else inp.class_ids[:1].cpu().numpy()
     ctx = None if inp.ctx is None else inp.ctx[:1].float().cpu().numpy()
     return ocfg, W, state, scale, cls, ctx, desc
@@ -580,54 +659,86 @@ def cpu_threads():
         return os.cpu_count()
 
 
-def cpu_baseline(cfg, T, weights, inp, sched, n_steps=4, oracle_ctx=None):
-    """Oracle steps/s on the host cores for a bounded sample (about 10-30 s of work)."""
+def oracle_schedule(cfg, weights, T, budget):
+    """Per-unit lifetimes from oracle.spectral (stored for the full-size models, checked
+    against the weights' checksum, else computed here) and the active blocks per step."""
+    from paper_2609_29505_gb300 import synth
+    S, source = golden_module().oracle_lifetimes(cfg, weights, T, budget)
+    groups = synth.block_groups(cfg)
+    G = max(groups) + 1
+    Sg = [0] * G
+    for g, x in zip(groups, S):
+        Sg[g] = int(x)
+    active = lambda s: sum(1 for x in Sg if x >= s)
+    return [int(x) for x in S], active, source
+
+
+def time_oracle(cfg, T, weights, inp, budget, positions, warm_positions=(), octx=None):
+    """Wall time of the oracle's scheduled forward on the sample at the given positions."""
     from oracle import trajectory as otj
-    ocfg, W, state, scale, cls, ctx, desc = oracle_ctx or oracle_sample(cfg, T, weights, inp, sched)
-    S = sched["lifetimes"]
-    # trajectory positions spread evenly over the horizon
-    steps = sorted({max(1, round((i + 0.5) * T / n_steps)) for i in range(n_steps)})
-    times = otj.time_steps(ocfg, W, S, T, steps, state, cls, ctx)
-    per_step = sum(times) / len(times)
-    return {"value": round(scale / per_step, 5), "unit": "steps/s", "cores": cpu_threads(),
-            "kind": "oracle",
-            "sample": f"{desc}; steps {steps} of T={T}, mean {per_step:.2f} s/step, "
-                      f"scaled by {1 / scale:g}x to the full batch"}
+    ocfg, W, state, scale, cls, ctx, desc = octx or oracle_sample(cfg, T, weights, inp)
+    S, active, source = oracle_schedule(cfg, weights, T, budget)
+    if warm_positions:
+        otj.time_steps(ocfg, W, S, T, list(warm_positions), state, cls, ctx)
+    t0 = time.perf_counter()
+    otj.time_steps(ocfg, W, S, T, list(positions), state, cls, ctx)
+    el = time.perf_counter() - t0
+    f = scale([active(s) for s in positions])
+    return el, f, desc, source
+
+
+def cpu_baseline(cfg, T, weights, inp, budget, n_steps=8):
+    """Oracle steps/s on the host cores for a bounded sample (about 10-30 s of work), at
+    n_steps positions spread over the horizon."""
+    positions = timed_plan(min(n_steps, T), T)[0]
+    el, f, desc, source = time_oracle(cfg, T, weights, inp, budget, positions)
+    per_step = el / len(positions)
+    return {"value": round(1.0 / (per_step * f), 6), "unit": "steps/s", "cores": cpu_threads(),
+            "kind": "oracle", "sample_s_per_step": round(per_step, 3), "scale": round(f, 4),
+            "lifetimes": f"oracle.spectral ({source})",
+            "sample": f"{desc}; positions {positions} of T={T}; value = 1 / (sample s/step x scale)"}
 
 
 def run_reference(args):
-    """--impl reference: the CPU oracle timed on the host cores (rank 0 only)."""
+    """--impl reference: the CPU oracle timed on the host cores (rank 0 only), at the
+    positions the native arm times, with the oracle's own lifetimes.  The synthetic weights
+    come from the same seeded generator on the same device as the native arm's (the same
+    bytes); nothing of the method runs on the GPU."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
     import torch
     from paper_2609_29505_gb300 import synth
-    from oracle import trajectory as otj
     cfg = synth.get_config(args.config)
     T = args.T or cfg.T
     dev = "cuda" if torch.cuda.is_available() else "cpu"
-    cfg0, T, weights, inp, sched, _ = setup_workload(args, dev)
+    weights = synth.make_weights(cfg, dev)
+    inp = synth.make_inputs(cfg, dev)
     K = args.steps if args.steps is not None else T
-    W = args.warmup if args.warmup is not None else 1
-    octx = oracle_sample(cfg0, T, weights, inp, sched)
-    ocfg, Wn, state, scale, cls, ctx, desc = octx
-    del weights
-    S = sched["lifetimes"]
-    otj.time_steps(ocfg, Wn, S, T, [i % T + 1 for i in range(W)], state, cls, ctx)
+    Wm = args.warmup if args.warmup is not None else 1
+    positions = [s for traj in timed_plan(K, T) for s in traj]
+    warm = [i % T + 1 for i in range(Wm)]
     t0 = time.perf_counter()
-    otj.time_steps(ocfg, Wn, S, T, [i % T + 1 for i in range(K)], state, cls, ctx)
-    el = time.perf_counter() - t0
-    value = scale * K / el
+    octx = oracle_sample(cfg, T, weights, inp)
+    el, f, desc, source = time_oracle(cfg, T, weights, inp, args.budget, positions, warm, octx)
+    setup_s = time.perf_counter() - t0 - el
+    per_step = el / K
+    value = 1.0 / (per_step * f)
     res = {"impl": "reference", "metric": METRIC if args.budget == 0.5 else
-           METRIC.replace("50%", f"{args.budget:.0%}"), "value": round(value, 5), "unit": "steps/s",
-           "n_gpus": 1, "steps": K, "warmup": W, "ms_per_step": round(1000.0 / value, 3),
-           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-           "data": "synthetic",
-           "config": {"workload": workload_name(cfg0, T, args.budget), "batch": cfg0.batch,
-                      "seq_len": cfg0.n_tokens, "T": T, "budget": args.budget},
-           "cpu_baseline": {"value": round(value, 5), "unit": "steps/s", "cores": cpu_threads(),
-                            "kind": "oracle", "sample": desc + f"; scaled by {1 / scale:g}x"},
-           "e2e": {"value": round(value, 5), "unit": "steps/s", "h2d_bytes_per_step": 0,
+           METRIC.replace("50%", f"{args.budget:.0%}"), "value": round(value, 6), "unit": "steps/s",
+           "n_gpus": 1, "steps": K, "warmup": Wm,
+           "ms_per_step": round(per_step * 1e3, 3),
+           "ms_per_step_is": "measured wall time of one sample step (value = 1 / (that x scale))",
+           "scale": round(f, 4), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+           "dtype": "f32", "data": "synthetic", "timed_positions": positions if K <= 256 else None,
+           "config": {"workload": workload_name(cfg, T, args.budget), "batch": cfg.batch,
+                      "seq_len": cfg.n_tokens, "T": T, "budget": args.budget},
+           "setup_s": round(setup_s, 1),
+           "cpu_baseline": {"value": round(value, 6), "unit": "steps/s", "cores": cpu_threads(),
+                            "kind": "oracle", "sample_s_per_step": round(per_step, 3),
+                            "scale": round(f, 4), "lifetimes": f"oracle.spectral ({source})",
+                            "sample": desc},
+           "e2e": {"value": round(value, 6), "unit": "steps/s", "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}
     print(json.dumps(res), flush=True)
 

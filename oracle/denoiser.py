@@ -258,7 +258,7 @@ class Trace:
 
 def denoise(cfg, weights, state, t: float, s: int, S_units: Sequence[int], cache: Dict,
             class_ids=None, ctx=None, trace: Optional[Trace] = None,
-            active_units: Optional[Sequence[bool]] = None) -> np.ndarray:
+            active_units: Optional[Sequence[bool]] = None, with_head: bool = True):
     """One denoiser evaluation at step s (1-based) under lifetimes S_units.
 
     ``cache`` maps unit index -> stored Delta and is updated in place: an active unit
@@ -267,6 +267,8 @@ def denoise(cfg, weights, state, t: float, s: int, S_units: Sequence[int], cache
     ``active_units``, when given, replaces the lifetime rule (unit u is active iff
     active_units[u]):
     the input-aware policy of App. B.1 chooses the active set per step.
+    With ``with_head`` False it returns (h_L, c) instead of the head's output, for callers
+    that apply the head to a subset of tokens.
     """
     h = stem(cfg, weights, state, t, class_ids)
     c = conditioning(cfg, weights, t, class_ids)
@@ -293,6 +295,8 @@ def denoise(cfg, weights, state, t: float, s: int, S_units: Sequence[int], cache
             u += 1
         if cfg.n_skips and b < cfg.n_skips:
             skips.append(h)
+    if not with_head:
+        return h, c
     return head(cfg, weights, h, c)
 
 

@@ -202,9 +202,11 @@ def active_sets(S_units: Sequence[int], T: int) -> np.ndarray:
 
 
 def schedule(cfg, weights: Dict[str, np.ndarray], T: int, budget: float,
-             group_of_unit: Sequence[int], eta: float = ETA) -> Dict:
-    """Algorithm 1 end to end: scores -> normalised scores -> tau -> per-unit lifetimes."""
-    bq = branch_scores(cfg, weights, eta)
+             group_of_unit: Sequence[int], eta: float = ETA, branch_q=None) -> Dict:
+    """Algorithm 1 end to end: scores -> normalised scores -> tau -> per-unit lifetimes.
+    ``branch_q``: the branch scores of these weights, when already computed by
+    ``branch_scores`` (the weights are then not read)."""
+    bq = branch_scores(cfg, weights, eta) if branch_q is None else [float(x) for x in branch_q]
     q = unit_scores(bq, group_of_unit)
     lam = normalise(q)
     s_min = min_lifetime(T)

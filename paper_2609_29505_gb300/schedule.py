@@ -238,32 +238,10 @@ SCHEDULE_FORMAT = 1
 
 
 def weights_digest(weights) -> str:
-    """sha256 over every weight tensor's name, shape, dtype and two exact integer checksums of
-    its raw 16-bit words (a plain sum and a position-weighted sum), computed where the tensor
-    lives in chunks, so a digest of device-resident weights needs no host copy."""
-    import hashlib
-
-    import torch
-
-    h = hashlib.sha256()
-    for name in sorted(weights):
-        t = weights[name]
-        if not _is_torch(t):
-            t = torch.from_numpy(np.ascontiguousarray(t))
-        v = t.detach().contiguous().reshape(-1)
-        if v.element_size() == 2:
-            v = v.view(torch.int16)
-        elif v.element_size() == 4:
-            v = v.view(torch.int32)
-        s1 = s2 = 0
-        chunk = 1 << 24
-        for i in range(0, v.numel(), chunk):
-            x = v[i:i + chunk].to(torch.int64)
-            pos = torch.arange(i, i + x.numel(), device=x.device, dtype=torch.int64) % 65521 + 1
-            s1 += int(x.sum())
-            s2 += int(((x + 65537) * pos).sum())
-        h.update(f"{name}|{tuple(t.shape)}|{t.dtype}|{s1}|{s2};".encode())
-    return h.hexdigest()
+    """Digest of the weights a schedule was computed from (synth.weights_checksum: exact
+    integer checksums of every tensor's raw words, computed where the tensor lives)."""
+    from .synth import weights_checksum
+    return weights_checksum(weights)
 
 
 def save_schedule(path: str, sched: Dict, cfg, weights=None, eta: float = ETA,

@@ -342,6 +342,36 @@ def token_ids_at(cfg: ModelConfig, inp: Inputs, s: int, T: Optional[int] = None)
     return ids
 
 
+def weights_checksum(weights) -> str:
+    """sha256 over every weight tensor's name, shape, dtype and two exact integer checksums of
+    its raw 16- or 32-bit words (a plain sum and a position-weighted sum), computed where the
+    tensor lives in chunks, so that device-resident weights need no host copy.  It identifies
+    one generated model (a stored schedule or stored scores belong to these exact bytes)."""
+    import hashlib
+
+    import numpy as np
+
+    h = hashlib.sha256()
+    for name in sorted(weights):
+        t = weights[name]
+        if not isinstance(t, torch.Tensor):
+            t = torch.from_numpy(np.ascontiguousarray(t))
+        v = t.detach().contiguous().reshape(-1)
+        if v.element_size() == 2:
+            v = v.view(torch.int16)
+        elif v.element_size() == 4:
+            v = v.view(torch.int32)
+        s1 = s2 = 0
+        chunk = 1 << 24
+        for i in range(0, v.numel(), chunk):
+            x = v[i:i + chunk].to(torch.int64)
+            pos = torch.arange(i, i + x.numel(), device=x.device, dtype=torch.int64) % 65521 + 1
+            s1 += int(x.sum())
+            s2 += int(((x + 65537) * pos).sum())
+        h.update(f"{name}|{tuple(t.shape)}|{t.dtype}|{s1}|{s2};".encode())
+    return h.hexdigest()
+
+
 def unit_names(cfg: ModelConfig) -> List[str]:
     """Residual units (branches) in graph order: 'b{block}.{branch}'."""
     return [f"b{b}.{br}" for b in range(cfg.n_blocks) for br in cfg.branches]

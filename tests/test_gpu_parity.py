@@ -44,14 +44,27 @@ def rel(a, b):
     return float(np.linalg.norm(a - b) / np.linalg.norm(b))
 
 
+def oracle_schedule(cfg, w_cpu, T, budget, granularity="block"):
+    """Algorithm 1 by the oracle (float64 spectra of the same bf16 weights)."""
+    W64 = {k: v.double().numpy() for k, v in w_cpu.items()}
+    groups = synth.block_groups(cfg) if granularity == "block" else synth.branch_groups(cfg)
+    return osp.schedule(cfg, W64, T, budget, groups)
+
+
 class Case:
-    def __init__(self, name, budget, flags=0):
+    """One small model at one budget: the product's schedule must equal the oracle's
+    (integer lifetimes); the oracle trajectory runs on the oracle's own lifetimes."""
+
+    def __init__(self, name, budget, flags=0, granularity="block"):
         self.cfg = cfg = synth.get_config(name)
         self.T = cfg.T
         self.w_cpu = synth.make_weights(cfg, "cpu")
         self.inp = synth.make_inputs(cfg, "cpu")
         self.W = odn.to_numpy_weights(self.w_cpu)
-        self.sched = schedule.build_schedule(cfg, self.w_cpu, self.T, budget=budget)
+        self.sched = schedule.build_schedule(cfg, self.w_cpu, self.T, budget=budget,
+                                             granularity=granularity)
+        self.osched = oracle_schedule(cfg, self.w_cpu, self.T, budget, granularity)
+        np.testing.assert_array_equal(self.sched["lifetimes"], self.osched["lifetimes"])
         self.w_dev = {k: v.cuda() for k, v in self.w_cpu.items()}
         self.cls = None if self.inp.class_ids is None else self.inp.class_ids.cuda()
         self.ctx = None if self.inp.ctx is None else self.inp.ctx.cuda()
@@ -62,7 +75,7 @@ class Case:
 
     def oracle(self):
         cfg = self.cfg
-        return otj.run(cfg, self.W, self.sched["lifetimes"], self.T,
+        return otj.run(cfg, self.W, self.osched["lifetimes"], self.T,
                        z0=None if self.inp.z0 is None else self.inp.z0.numpy(),
                        class_ids=None if self.inp.class_ids is None else self.inp.class_ids.numpy(),
                        ctx=None if self.inp.ctx is None else self.inp.ctx.float().numpy(),
@@ -85,10 +98,10 @@ class Case:
 _cases = {}
 
 
-def case(name, budget):
-    key = (name, budget)
+def case(name, budget, granularity="block"):
+    key = (name, budget, granularity)
     if key not in _cases:
-        c = Case(name, budget, FLAGS)
+        c = Case(name, budget, FLAGS, granularity)
         c.ref = c.oracle()
         _cases[key] = c
     return _cases[key]
@@ -99,7 +112,7 @@ def case(name, budget):
 def test_active_sets_and_teacher_forced_steps(B, name, budget):
     c = case(name, budget)
     m = c.model(B)
-    want_masks = osp.active_sets(c.sched["lifetimes"], c.T)
+    want_masks = osp.active_sets(c.osched["lifetimes"], c.T)
     out = c.out_buffer()
     errs = []
     for s in range(1, c.T + 1):
@@ -200,27 +213,56 @@ def test_step_order_and_state_errors(B):
     m.close()
 
 
-@pytest.mark.parametrize("name", ["llada_small", "uvit_small", "sdxl_small"])
-def test_execution_modes_are_bit_identical(B, name):
-    """Jagged graphs, eager op-by-op launches (host skipping) and padded graphs (frozen
-    branches evaluated and discarded) give the same outputs bit for bit."""
+@pytest.mark.parametrize("name", ["llada_small", "uvit_small", "sdxl_small", "dit_small"])
+def test_execution_modes_against_oracle(B, name):
+    """Every execution mode of Table tab:kernel -- jagged graphs, eager op-by-op launches
+    (host-side skipping) and padded graphs (frozen branches evaluated and discarded) --
+    matches the oracle teacher forced (per-step relative L2 <= 5e-3), and the three give
+    the same outputs bit for bit."""
     c = case(name, 0.5)
     results = {}
     for mode in (B.EXEC_JAGGED_GRAPH, B.EXEC_EAGER, B.EXEC_PADDED_GRAPH):
         m = c.model(B)
         m.set_exec_mode(mode)
         out = c.out_buffer()
-        res = []
+        res, errs = [], []
         for s in range(1, c.T + 1):
             x = c.ids_at(s).cuda() if c.cfg.stem == "embed" else torch.from_numpy(c.ref["states"][s - 1]).cuda()
             m.step(x, out, otj.timestep(c.T, s), s, class_ids=c.cls, ctx=c.ctx)
             res.append(out.cpu().clone())
+            errs.append(rel(res[-1].float().numpy(), c.ref["outputs"][s - 1]))
         m.check_device()
         m.close()
         results[mode] = res
+        assert max(errs) <= STEP_TOL, f"mode {mode}: per-step rel L2 {['%.2e' % e for e in errs]}"
     for mode in (B.EXEC_EAGER, B.EXEC_PADDED_GRAPH):
         for a, b in zip(results[B.EXEC_JAGGED_GRAPH], results[mode]):
             assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("budget", [0.5, 0.33])
+@pytest.mark.parametrize("name", ["llada_small", "dit_small", "sdxl_small"])
+def test_branch_granularity_against_oracle(B, name, budget):
+    """Branch granularity (every branch its own atomic group, so an attention branch can be
+    frozen while its block's MLP still runs, App. G): lifetimes equal to the oracle's,
+    bit-exact active sets, per-step relative L2 <= 5e-3 teacher forced."""
+    c = case(name, budget, "branch")
+    S = np.asarray(c.osched["lifetimes"])
+    nb = len(c.cfg.branches)
+    assert any(len(set(S[b * nb:(b + 1) * nb])) > 1 for b in range(c.cfg.n_blocks)), \
+        "schedule has no block with branches of different lifetimes"
+    m = c.model(B)
+    want_masks = osp.active_sets(S, c.T)
+    out = c.out_buffer()
+    errs = []
+    for s in range(1, c.T + 1):
+        np.testing.assert_array_equal(m.active_mask(s), want_masks[s - 1])
+        x = c.ids_at(s).cuda() if c.cfg.stem == "embed" else torch.from_numpy(c.ref["states"][s - 1]).cuda()
+        m.step(x, out, otj.timestep(c.T, s), s, class_ids=c.cls, ctx=c.ctx)
+        errs.append(rel(out.float().cpu().numpy(), c.ref["outputs"][s - 1]))
+    m.check_device()
+    m.close()
+    assert max(errs) <= STEP_TOL, f"per-step rel L2 {['%.2e' % e for e in errs]}"
 
 
 @pytest.mark.parametrize("name", ["llada_small", "sdxl_small"])
@@ -267,11 +309,13 @@ def test_long_context_4096_tokens(B):
     inp = synth.make_inputs(cfg, "cpu")
     W = odn.to_numpy_weights(w_cpu)
     sched = schedule.build_schedule(cfg, w_cpu, cfg.T, budget=0.5)
-    ref = otj.run(cfg, W, sched["lifetimes"], cfg.T,
+    osched = oracle_schedule(cfg, w_cpu, cfg.T, 0.5)
+    np.testing.assert_array_equal(sched["lifetimes"], osched["lifetimes"])
+    ref = otj.run(cfg, W, osched["lifetimes"], cfg.T,
                   ids_at=lambda s: synth.token_ids_at(cfg, inp, s).numpy())
     m = B.Denoiser(cfg, {k: v.cuda() for k, v in w_cpu.items()})
     m.set_schedule(cfg.T, sched["lifetimes"], sched["groups"])
-    masks = osp.active_sets(sched["lifetimes"], cfg.T)
+    masks = osp.active_sets(osched["lifetimes"], cfg.T)
     out = torch.empty(1, cfg.n_tokens, cfg.d_out, dtype=torch.float16, device="cuda")
     for s in range(1, cfg.T + 1):
         np.testing.assert_array_equal(m.active_mask(s), masks[s - 1])
