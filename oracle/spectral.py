@@ -19,6 +19,12 @@ Every function follows one passage of the paper:
   ratio is the largest not above the budget.
 * ``active_sets``                       — Sec. 3.1 / Algorithm 2: unit l is evaluated
   at step s iff s <= S_l.
+* ``matrix_statistic`` / ``ranked_branch_scores`` — the alternative static rankings of
+  Table tab:cross-ablation (random, depth-only, Frobenius norm, spectral norm, stable
+  rank, Frobenius x stable rank, raw SCR).  Reading: each replaces g(W) in the branch
+  formulas of App. G by its own per-matrix statistic, larger scores giving longer
+  lifetimes; depth-only scores a branch by its distance from the output (earlier
+  branches live longer); random takes the draws it is given.
 """
 from __future__ import annotations
 
@@ -117,6 +123,61 @@ def branch_scores(cfg, weights: Dict[str, np.ndarray], eta: float = ETA) -> List
             out.append(xattn_score(weights[p + "wx_q"], wkv[:d], wkv[d:], weights[p + "wx_o"],
                                    cfg.d_head, eta))
         out.append(mlp_score(weights[p + "w_1"], weights[p + "w_2"], eta))
+    return out
+
+
+RANKINGS = ("scr", "frobenius", "spectral", "stable_rank", "frob_stable_rank", "raw_scr",
+            "depth", "random")
+
+
+def matrix_statistic(W, ranking: str, eta: float = ETA) -> float:
+    """Per-matrix score of one static ranking (Table tab:cross-ablation):
+    scr -> g(W); frobenius -> ||W||_F; spectral -> ||W||_2 = sigma_1;
+    stable_rank -> ||W||_F^2 / ||W||_2^2; frob_stable_rank -> ||W||_F times the stable
+    rank; raw_scr -> SCR_eta(W) (Eq. scr-reg)."""
+    if ranking == "scr":
+        return matrix_score(W, eta)
+    if ranking == "raw_scr":
+        return scr_eta(W, eta)
+    f2 = frobenius_sq(W)
+    if ranking == "frobenius":
+        return math.sqrt(f2)
+    top = float(singular_energies(W)[0])
+    if ranking == "spectral":
+        return math.sqrt(top)
+    if ranking == "stable_rank":
+        return f2 / top
+    if ranking == "frob_stable_rank":
+        return math.sqrt(f2) * (f2 / top)
+    raise ValueError(ranking)
+
+
+def ranked_branch_scores(cfg, weights, ranking: str, eta: float = ETA,
+                         draws: Sequence[float] = None) -> List[float]:
+    """Branch scores of one static ranking, in graph order.  Matrix rankings use the
+    branch formulas of App. G (Eqs. app-attn-score, app-xattn-score, app-mlp-score) with
+    matrix_statistic in place of g; depth-only gives branch u of U the score U - u;
+    random returns ``draws`` (one per branch, drawn by the caller)."""
+    n = cfg.n_units
+    if ranking == "depth":
+        return [float(n - u) for u in range(n)]
+    if ranking == "random":
+        if draws is None or len(draws) != n:
+            raise ValueError("the random ranking takes one draw per branch")
+        return [float(x) for x in draws]
+    st = lambda W: matrix_statistic(W, ranking, eta)
+    d = cfg.d
+    out: List[float] = []
+    for b in range(cfg.n_blocks):
+        p = f"blocks.{b}."
+        wqkv = weights[p + "w_qkv"]
+        gq, gk, gv, go = st(wqkv[:d]), st(wqkv[d:2 * d]), st(wqkv[2 * d:]), st(weights[p + "w_o"])
+        out.append(go * gv * (1.0 + gq * gk / math.sqrt(cfg.d_head)))
+        if cfg.block == "xattn":
+            wkv = weights[p + "wx_kv"]
+            gq, gk, gv, go = st(weights[p + "wx_q"]), st(wkv[:d]), st(wkv[d:]), st(weights[p + "wx_o"])
+            out.append(go * gv * (1.0 + gq * gk / math.sqrt(cfg.d_head)))
+        out.append(st(weights[p + "w_2"]) * st(weights[p + "w_1"]))
     return out
 
 

@@ -406,3 +406,127 @@ def test_scheduled_active_sets_keep_groups_atomic():
     for b in range(cfg.n_blocks):
         assert np.all(A[:, b * nb:(b + 1) * nb] == A[:, b * nb:b * nb + 1])
     assert res["ratio"] <= 0.5
+
+
+# ---------------------------------------------------------------------------
+# AdaLN conditioning pins (DiT family): hand-computed cases whose weights are scaled
+# identities / selections, so that each quantity has a closed form and a dropped "1 +",
+# a SiLU at the wrong stage, a class embedding added before W_t2 or a permuted chunk
+# order each change the result.
+# ---------------------------------------------------------------------------
+
+def _silu(v):
+    return v / (1.0 + math.exp(-v))
+
+
+def test_modulate_hand_case():
+    """x (1 + scale_b) + shift_b, the sample's shift and scale broadcast over its tokens."""
+    x = np.array([[[1.0, -2.0], [0.5, 4.0]], [[3.0, 1.0], [-1.0, 0.0]]], F32)   # [B=2, N=2, d=2]
+    shift = np.array([[10.0, 20.0], [-5.0, 7.0]], F32)
+    scale = np.array([[0.5, -1.0], [2.0, 0.25]], F32)
+    got = dn.modulate(x, shift, scale)
+    for b in range(2):
+        for n in range(2):
+            for j in range(2):
+                want = float(x[b, n, j]) * (1.0 + float(scale[b, j])) + float(shift[b, j])
+                assert got[b, n, j] == pytest.approx(want, rel=1e-6, abs=1e-6)
+
+
+def _dit_micro_weights(cfg, rng):
+    """W_t1 = 3 x (selection of the first t_freq of d rows), W_t2 = 2 I, one-hot-ish class
+    rows, W_mod chunks = (j + 1) I, W_modf = [I; 2 I] (the rest random)."""
+    W = _weights(cfg)
+    d, tf = cfg.d, cfg.t_freq
+    W["w_t1"] = np.zeros((d, tf), F32)
+    for i in range(min(d, tf)):
+        W["w_t1"][i, i] = 3.0
+    W["w_t2"] = 2.0 * np.eye(d, dtype=F32)
+    W["class_emb"] = np.zeros((cfg.n_classes, d), F32)
+    for y in range(cfg.n_classes):
+        W["class_emb"][y, y % d] = 5.0 + y
+    for b in range(cfg.n_blocks):
+        W[f"blocks.{b}.w_mod"] = np.concatenate([(j + 1.0) * np.eye(d, dtype=F32) for j in range(6)])
+    W["w_modf"] = np.concatenate([np.eye(d, dtype=F32), 2.0 * np.eye(d, dtype=F32)])
+    return W
+
+
+def _hand_conditioning(cfg, t, y):
+    """c = W_t2 silu(W_t1 sinusoid(t)) + class_emb[y] for the weights above, by hand."""
+    d, tf = cfg.d, cfg.t_freq
+    half = tf // 2
+    emb = [math.cos(t * 10000.0 ** (-i / half)) for i in range(half)]
+    emb += [math.sin(t * 10000.0 ** (-i / half)) for i in range(half)]
+    c = []
+    for i in range(d):
+        hidden = _silu(3.0 * emb[i]) if i < tf else _silu(0.0)
+        c.append(2.0 * hidden + (5.0 + y if i == y % d else 0.0))
+    return np.array(c)
+
+
+def test_conditioning_hand_case():
+    cfg = _micro("adaln")
+    W = _dit_micro_weights(cfg, np.random.default_rng(5))
+    for t, y in ((0.0, 0), (137.25, 3), (999.0, 4)):
+        got = dn.conditioning(cfg, W, t, np.array([y]))
+        np.testing.assert_allclose(got[0], _hand_conditioning(cfg, t, y), rtol=1e-5, atol=1e-5)
+
+
+def test_block_modulation_chunk_order():
+    """shift1, scale1, gate1, shift2, scale2, gate2 = chunks 0..5 of W_mod silu(c)."""
+    cfg = _micro("adaln")
+    W = _dit_micro_weights(cfg, np.random.default_rng(6))
+    c = np.array([[0.3, -1.2] + [0.1 * i for i in range(cfg.d - 2)]], F32)
+    mods = dn.block_modulation(W, 0, c)
+    assert len(mods) == 6
+    for j, m in enumerate(mods):
+        want = [(j + 1.0) * _silu(float(v)) for v in c[0]]
+        np.testing.assert_allclose(m[0], want, rtol=1e-5, atol=1e-6)
+
+
+def test_adaln_branches_use_their_own_chunks():
+    """attn: LN(h)(1 + scale1) + shift1 -> attention -> gate1 * (o W_O^T); mlp: LN(h)(1 +
+    scale2) + shift2 -> GELU-tanh MLP -> gate2 * (.), with the chunks of the case above."""
+    cfg = _micro("adaln")
+    W = _dit_micro_weights(cfg, np.random.default_rng(7))
+    rng = np.random.default_rng(8)
+    h = rng.standard_normal((1, cfg.n_tokens, cfg.d)).astype(F32)
+    c = rng.standard_normal((1, cfg.d)).astype(F32)
+    sc = np.array([_silu(float(v)) for v in c[0]], np.float64)
+    chunk = [(j + 1.0) * sc for j in range(6)]
+    x = dn.layer_norm(h, None, None, cfg.eps).astype(np.float64)[0]
+    d = cfg.d
+    # attention branch
+    xm = x * (1.0 + chunk[1]) + chunk[0]
+    qkv = xm @ W["blocks.0.w_qkv"].T.astype(np.float64)
+    o = dn.attention(qkv[None, :, :d].astype(F32), qkv[None, :, d:2 * d].astype(F32),
+                     qkv[None, :, 2 * d:].astype(F32), cfg.n_heads)[0].astype(np.float64)
+    want = chunk[2] * (o @ W["blocks.0.w_o"].T.astype(np.float64))
+    np.testing.assert_allclose(dn.branch(cfg, W, 0, "attn", h, c)[0], want, rtol=2e-4, atol=2e-4)
+    # MLP branch
+    xm = x * (1.0 + chunk[4]) + chunk[3]
+    u = xm @ W["blocks.0.w_1"].T.astype(np.float64)
+    a = 0.5 * u * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (u + 0.044715 * u ** 3)))
+    want = chunk[5] * (a @ W["blocks.0.w_2"].T.astype(np.float64))
+    np.testing.assert_allclose(dn.branch(cfg, W, 0, "mlp", h, c)[0], want, rtol=2e-4, atol=2e-4)
+
+
+def test_adaln_linear_head_hand_case():
+    """shift, scale = chunks of W_modf silu(c) (here silu(c) and 2 silu(c)); out =
+    (LN(h)(1 + scale) + shift) W_head^T, first out_channels columns."""
+    cfg = _micro("adaln")
+    W = _dit_micro_weights(cfg, np.random.default_rng(9))
+    rng = np.random.default_rng(10)
+    h = rng.standard_normal((1, cfg.n_tokens, cfg.d)).astype(F32)
+    c = rng.standard_normal((1, cfg.d)).astype(F32)
+    got = dn.head(cfg, W, h, c)
+    assert got.shape == (1, cfg.n_tokens, cfg.out_channels)
+    sc = [_silu(float(v)) for v in c[0]]
+    for n in range(cfg.n_tokens):
+        row = [float(v) for v in h[0, n]]
+        mu = sum(row) / cfg.d
+        var = sum((v - mu) ** 2 for v in row) / cfg.d
+        xn = [(v - mu) / math.sqrt(var + cfg.eps) for v in row]
+        xm = [xn[i] * (1.0 + 2.0 * sc[i]) + sc[i] for i in range(cfg.d)]
+        for o in range(cfg.out_channels):
+            want = sum(xm[i] * float(W["w_head"][o, i]) for i in range(cfg.d))
+            assert got[0, n, o] == pytest.approx(want, rel=1e-4, abs=1e-4)

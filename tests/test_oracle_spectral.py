@@ -259,3 +259,77 @@ def test_active_sets_nested_and_group_closed():
     # row sums equal the number of units with S >= s
     for s in range(1, 5):
         assert A[s - 1].sum() == sum(1 for x in S_units if x >= s)
+
+
+# ---------------------------------------------------------------------------
+# alternative static rankings (Table tab:cross-ablation)
+# ---------------------------------------------------------------------------
+
+def test_matrix_statistics_on_known_spectra():
+    """diag(s) and U diag(s) V^T with known s: ||W||_F^2 = sum s^2, ||W||_2 = max s, stable
+    rank = sum s^2 / max s^2, the product, raw SCR = Eq. scr-reg from s."""
+    rng = np.random.default_rng(11)
+    s = np.array([5.0, 3.0, 2.0, 1.0, 0.5, 0.25, 0.1, 0.1, 0.05, 0.01, 0.01, 0.003])
+    U, _ = np.linalg.qr(rng.standard_normal((20, 12)))
+    V, _ = np.linalg.qr(rng.standard_normal((12, 12)))
+    for W in (np.diag(s), (U * s) @ V.T, ((U * s) @ V.T).T):
+        f2 = float(np.sum(s ** 2))
+        assert sp.matrix_statistic(W, "frobenius") == pytest.approx(math.sqrt(f2), rel=1e-12)
+        assert sp.matrix_statistic(W, "spectral") == pytest.approx(5.0, rel=1e-10)
+        assert sp.matrix_statistic(W, "stable_rank") == pytest.approx(f2 / 25.0, rel=1e-10)
+        assert sp.matrix_statistic(W, "frob_stable_rank") == pytest.approx(math.sqrt(f2) * f2 / 25.0,
+                                                                          rel=1e-10)
+        eta = 1e-6
+        want = math.log((25.0 + eta * f2) / (f2 - 25.0 + eta * f2))  # k = 1 for d = 12
+        assert sp.matrix_statistic(W, "raw_scr") == pytest.approx(want, rel=1e-10)
+        assert sp.matrix_statistic(W, "scr") == sp.matrix_score(W)
+
+
+def _scaled_identity_model():
+    """Two-block pre-norm model whose projections are diagonal with known entries, so that
+    every statistic has a closed form: W_Q, W_K, W_V, W_O = diag(a_j), j = 1..4, per block;
+    W_1 = [diag(p); diag(p)] (gated), W_2 = diag(w)."""
+    from paper_2609_29505_gb300 import synth
+    cfg = synth.ModelConfig(name="ranks", stem="time_add", block="prenorm", norm="rms",
+                            mlp="swiglu", head="linear", n_blocks=2, d=4, n_heads=1, d_head=4,
+                            d_ff=4, batch=1, n_tokens=2, d_in=4, d_out=4, out_channels=4, T=4)
+    base = np.array([1.0, 0.5, 0.25, 0.125])
+    W = {}
+    for b in range(2):
+        a = [(b + 1) * j * base for j in (1, 2, 3, 4)]
+        W[f"blocks.{b}.w_qkv"] = np.vstack([np.diag(a[0]), np.diag(a[1]), np.diag(a[2])])
+        W[f"blocks.{b}.w_o"] = np.diag(a[3])
+        W[f"blocks.{b}.w_1"] = np.vstack([np.diag(1.5 * base), np.diag(1.5 * base)])
+        W[f"blocks.{b}.w_2"] = np.diag((b + 2) * base)
+    return cfg, W, base
+
+
+@pytest.mark.parametrize("ranking", ["frobenius", "spectral", "stable_rank", "frob_stable_rank"])
+def test_ranked_branch_scores_hand_model(ranking):
+    """Branch formulas of App. G with the ranking's statistic, derived by hand: for
+    c diag(base), ||.||_F = c n2, ||.||_2 = c, stable rank = n2^2 (n2 = ||base||); the
+    stacked [diag(p); diag(p)] doubles the squared Frobenius norm."""
+    cfg, W, base = _scaled_identity_model()
+    n2 = math.sqrt(float(np.sum(base ** 2)))
+    stat = {"frobenius": lambda c, k=1: c * n2 * math.sqrt(k),
+            "spectral": lambda c, k=1: c * math.sqrt(k),
+            "stable_rank": lambda c, k=1: n2 ** 2,
+            "frob_stable_rank": lambda c, k=1: c * n2 * math.sqrt(k) * n2 ** 2}[ranking]
+    want = []
+    for b in range(2):
+        gq, gk, gv, go = (stat((b + 1) * j) for j in (1, 2, 3, 4))
+        want.append(go * gv * (1.0 + gq * gk / 2.0))
+        want.append(stat(b + 2) * stat(1.5, 2))
+    got = sp.ranked_branch_scores(cfg, W, ranking)
+    np.testing.assert_allclose(got, want, rtol=1e-10)
+
+
+def test_ranked_branch_scores_depth_random_and_scr():
+    cfg, W, _ = _scaled_identity_model()
+    assert sp.ranked_branch_scores(cfg, W, "depth") == [4.0, 3.0, 2.0, 1.0]
+    draws = [0.3, 0.9, 0.1, 0.5]
+    assert sp.ranked_branch_scores(cfg, W, "random", draws=draws) == draws
+    with pytest.raises(ValueError):
+        sp.ranked_branch_scores(cfg, W, "random")
+    np.testing.assert_allclose(sp.ranked_branch_scores(cfg, W, "scr"), sp.branch_scores(cfg, W),
+                               rtol=1e-15)

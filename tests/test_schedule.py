@@ -76,3 +76,22 @@ def test_alternative_rankings_meet_budget(ranking, weights):
     S = res["group_lifetimes"]
     order = np.argsort(lam, kind="stable")
     assert np.all(np.diff(S[order]) >= 0)
+
+
+@pytest.mark.parametrize("ranking", ["frobenius", "spectral", "stable_rank", "frob_stable_rank",
+                                     "raw_scr", "depth", "random"])
+@pytest.mark.parametrize("name", ["dit_small", "sdxl_small", "llada_small"])
+def test_alternative_rankings_match_oracle(ranking, name, weights):
+    """Every alternative ranking of Table tab:cross-ablation: the product's branch scores
+    equal the oracle's restatement (the random ranking's draws, seeded uniform numbers in
+    graph order, are handed to the oracle), and the lifetimes at 50% agree bit for bit."""
+    cfg = synth.get_config(name)
+    W = odn.to_numpy_weights(weights[name])
+    draws = np.random.default_rng(0).uniform(size=cfg.n_units) if ranking == "random" else None
+    want = np.array(osp.ranked_branch_scores(cfg, W, ranking, draws=draws))
+    got = schedule.branch_scores(cfg, weights[name], ranking=ranking)
+    np.testing.assert_allclose(got, want, rtol=1e-9)
+    groups = synth.block_groups(cfg)
+    S_want = osp.schedule(cfg, None, cfg.T, 0.5, groups, branch_q=want)["lifetimes"]
+    S_got = schedule.build_schedule(cfg, weights[name], cfg.T, budget=0.5, ranking=ranking)["lifetimes"]
+    np.testing.assert_array_equal(S_got, S_want)
