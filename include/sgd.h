@@ -54,7 +54,8 @@ typedef enum {
   SGD_ERR_CUDA = -5,           /* a CUDA runtime call failed                       */
   SGD_ERR_DEVICE_TIMEOUT = -6, /* a kernel's bounded wait expired (device status)  */
   SGD_ERR_OOM = -7,            /* device allocation failed                         */
-  SGD_ERR_STATE = -8           /* call order violated (e.g. step before schedule)  */
+  SGD_ERR_STATE = -8,          /* call order violated (e.g. step before schedule)  */
+  SGD_ERR_RANGE = -9           /* an fp16 value was clamped to +-65504 (or NaN)    */
 } sgd_status;
 
 /* Input stage of the denoiser. */
@@ -171,7 +172,11 @@ typedef struct sgd_ctx sgd_ctx;
 
 /*
  * sgd_create — validate the model shape, borrow the weights, make the fp16 projection
- * copies, allocate caches and workspaces on the current device.
+ * copies, allocate caches and workspaces on the current device.  The model is the
+ * pretrained network of the problem statement (Sec. 3.1: a stack of residual units
+ * h_{l,s} = h_{l-1,s} + F_l(h_{l-1,s}; c_s) evaluated once per sampler step); the context
+ * holds what the executor of Sec. 4.2 keeps across steps (per-unit update caches,
+ * captured graphs).
  * desc, w: host structs (copied).  Weight pointers: device, 16-byte aligned; norm
  * gains, embeddings, stem, conditioning and small-head weights are read in place and
  * must stay valid and unchanged for the context's lifetime.
@@ -230,8 +235,11 @@ SGD_API int sgd_step_host_async(sgd_ctx* ctx, const void* state_in_host, void* o
 /* sgd_host_wait — wait until every output copy queued by sgd_step_host_async is done. */
 SGD_API int sgd_host_wait(sgd_ctx* ctx);
 
-/* sgd_get_active_mask — mask_host[u] = 1 iff unit u is evaluated at `step` (1..T).  Under
- * the drift policy: the mask step `step` ran with (steps run since the last reset). */
+/* sgd_get_active_mask — the active set A_s of Sec. 3.1 / Algorithm 2 (unit u is evaluated
+ * at step s iff s <= S_u): mask_host[u] = 1 iff unit u is evaluated at `step` (1..T).
+ * Under the drift policy (App. B.1): the mask step `step` ran with (steps run since the
+ * last reset).  mask_host: uint8 [n_units], n_units must equal the model's.
+ * Errors: SGD_ERR_ARG, SGD_ERR_STATE (no schedule or step not yet run under drift). */
 SGD_API int sgd_get_active_mask(const sgd_ctx* ctx, int step, uint8_t* mask_host, int n_units);
 
 /* sgd_get_info — sizes and schedule statistics. */
@@ -281,17 +289,23 @@ SGD_API int sgd_set_policy(sgd_ctx* ctx, int policy);
  */
 SGD_API int sgd_get_drift(const sgd_ctx* ctx, int step, double* drift_host, int n_groups);
 
-/* sgd_reset — start a new trajectory: the next step must be 1 (caches invalidated). */
+/* sgd_reset — start a new trajectory (Algorithm 2 starts at s = 1 with no stored updates):
+ * the next step must be 1, and every cache counts as unwritten until its unit runs. */
 SGD_API int sgd_reset(sgd_ctx* ctx);
 
 /* sgd_check_device — synchronise `stream` and report a device-side status word set by
- * a kernel whose bounded wait expired (SGD_ERR_DEVICE_TIMEOUT); clears it. */
+ * a kernel whose bounded wait expired (SGD_ERR_DEVICE_TIMEOUT), else the fp16 clamp flag
+ * (SGD_ERR_RANGE: some fp16 activation, attention output or cached update left fp16's
+ * finite range, or was NaN, and was stored clamped to +-65504 since the last check, so the
+ * results are not to be trusted); clears what it reports. */
 SGD_API int sgd_check_device(sgd_ctx* ctx, void* stream);
 
-/* sgd_destroy — free everything the context owns (graphs, caches, workspaces). */
+/* sgd_destroy — free everything the context owns (graphs, caches, workspaces; the state
+ * the executor of Sec. 4.2 keeps across steps).  The borrowed weights are not touched. */
 SGD_API void sgd_destroy(sgd_ctx* ctx);
 
-/* sgd_last_error — message of the last failing call on this thread ("" if none). */
+/* sgd_last_error — message of the last failing call on this thread ("" if none).  ABI
+ * plumbing with no counterpart in the paper: errors cross the boundary as status codes. */
 SGD_API const char* sgd_last_error(void);
 
 /*

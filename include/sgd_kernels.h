@@ -136,6 +136,11 @@ SGD_API int sgd_kernel_frozen_run(float* h, const void* const* caches_host, int 
 /* Device status word shared by all kernels (bounded-wait expiry); returns and clears it. */
 SGD_API int sgd_kernel_status(int* status_host);
 
+/* *clamped_host = 1 if any kernel stored an fp16 value that it had to clamp to +-65504
+ * (the value was out of fp16's range, or NaN) since the last call, else 0; clears the
+ * flags.  A reading aid for fp16 operands, which the paper (bf16) does not use. */
+SGD_API int sgd_kernel_f16_clamped(int* clamped_host);
+
 /*
  * Failure-path self-test (no counterpart in the paper): launches on `stream` one kernel
  * whose thread waits, with the same bounded wait every kernel uses, on an mbarrier that

@@ -29,6 +29,7 @@ SGD_ERR_CUDA = -5
 SGD_ERR_DEVICE_TIMEOUT = -6
 SGD_ERR_OOM = -7
 SGD_ERR_STATE = -8
+SGD_ERR_RANGE = -9
 SGD_SELFTEST_TIMEOUT_CODE = 99  # status code recorded by sgd_selftest_wait_timeout
 
 STEM = {"time_add": 0, "patch": 1, "patch_tokens": 2, "identity": 3, "embed": 4}
@@ -50,7 +51,7 @@ EXPORTED = [
     "sgd_compile_schedule", "sgd_step_profile", "sgd_sampler_update", "sgd_kernel_gemm",
     "sgd_kernel_attention", "sgd_kernel_norm", "sgd_kernel_frozen_run", "sgd_kernel_status",
     "sgd_set_exec_mode", "sgd_step_host_async", "sgd_host_wait", "sgd_kernel_gemm_static_ws",
-    "sgd_set_policy", "sgd_get_drift", "sgd_selftest_wait_timeout",
+    "sgd_set_policy", "sgd_get_drift", "sgd_selftest_wait_timeout", "sgd_kernel_f16_clamped",
 ]
 EXEC_JAGGED_GRAPH, EXEC_EAGER, EXEC_PADDED_GRAPH = 0, 1, 2
 POLICY_STATIC, POLICY_DRIFT = 0, 1
@@ -136,6 +137,7 @@ def lib() -> C.CDLL:
             "sgd_kernel_norm": (i, [vp, vp, i, i, i, vp, vp, vp, vp, i, i, f, vp]),
             "sgd_kernel_frozen_run": (i, [vp, C.POINTER(vp), i, i64, vp]),
             "sgd_kernel_status": (i, [C.POINTER(C.c_int)]),
+            "sgd_kernel_f16_clamped": (i, [C.POINTER(C.c_int)]),
             "sgd_set_exec_mode": (i, [vp, i]),
             "sgd_step_host_async": (i, [vp, vp, vp, f, vp, vp, i, vp]),
             "sgd_host_wait": (i, [vp]),
@@ -229,6 +231,12 @@ def sgd_kernel_frozen_run(h, caches, stream=None):
 def sgd_kernel_status() -> int:
     st = C.c_int(0)
     check(lib().sgd_kernel_status(C.byref(st)), "sgd_kernel_status")
+    return int(st.value)
+
+
+def sgd_kernel_f16_clamped() -> int:
+    st = C.c_int(0)
+    check(lib().sgd_kernel_f16_clamped(C.byref(st)), "sgd_kernel_f16_clamped")
     return int(st.value)
 
 

@@ -1408,6 +1408,11 @@ int sgd_check_device(sgd_ctx* c, void* stream) {
   int rc = sgd_kernel_status(&st);
   if (rc) return rc;
   if (st) return fail(SGD_ERR_DEVICE_TIMEOUT, "a kernel's bounded wait expired (code " + std::to_string(st) + ")");
+  int clamped = 0;
+  if ((rc = sgd_kernel_f16_clamped(&clamped))) return rc;
+  if (clamped)
+    return fail(SGD_ERR_RANGE, "an fp16 activation or cache value was outside fp16's range "
+                               "(or NaN) and was clamped to +-65504");
   return SGD_OK;
 }
 
@@ -1606,6 +1611,23 @@ int sgd_selftest_wait_timeout(void* stream) {
   int* p = device_status_ptr();
   if (!p) return fail(SGD_ERR_CUDA, "status word unavailable");
   CUDA_TRY(wait_selftest_launch(p, SGD_SELFTEST_TIMEOUT_CODE, static_cast<cudaStream_t>(stream)));
+  return SGD_OK;
+}
+
+int sgd_kernel_f16_clamped(int* clamped_host) {
+  if (!clamped_host) return fail(SGD_ERR_ARG, "null argument");
+  *clamped_host = 0;
+  unsigned int* flags[3] = {f16_clamp_flag_gemm(), f16_clamp_flag_attention(),
+                            f16_clamp_flag_elementwise()};
+  for (unsigned int* p : flags) {
+    if (!p) return fail(SGD_ERR_CUDA, "fp16 clamp flag unavailable");
+    unsigned int v = 0;
+    CUDA_TRY(cudaMemcpy(&v, p, sizeof(v), cudaMemcpyDeviceToHost));
+    if (v) {
+      *clamped_host = 1;
+      CUDA_TRY(cudaMemset(p, 0, sizeof(v)));
+    }
+  }
   return SGD_OK;
 }
 

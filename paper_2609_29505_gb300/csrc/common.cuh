@@ -45,9 +45,18 @@ __device__ __forceinline__ uint4 pack_bf16x8(const float* f) {
   return u;
 }
 
+// Raised when an fp16 store had to clamp a value (|x| > 65504, or NaN) — one instance per
+// translation unit (internal linkage), read and cleared by the host through
+// f16_clamp_flag_here() of that unit.
+static __device__ unsigned int g_f16_clamped;
+
 // fp16 operands: values are clamped to the finite fp16 range before rounding so that
-// an out-of-range activation saturates instead of turning into inf / NaN downstream.
-__device__ __forceinline__ float sat_f16(float x) { return fminf(fmaxf(x, -65504.f), 65504.f); }
+// an out-of-range activation saturates instead of turning into inf / NaN downstream; the
+// clamp raises g_f16_clamped, which sgd_check_device reports.
+__device__ __forceinline__ float sat_f16(float x) {
+  if (!(fabsf(x) <= 65504.f)) g_f16_clamped = 1u;
+  return fminf(fmaxf(x, -65504.f), 65504.f);
+}
 
 __device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
   __half2 v = __floats2half2_rn(sat_f16(lo), sat_f16(hi));
@@ -331,6 +340,20 @@ __host__ __device__ constexpr uint32_t umma_idesc_f16(int M, int N) {
 // Same with B MN-major (transpose-B bit 16): B stored with its N index contiguous.
 __host__ __device__ constexpr uint32_t umma_idesc_f16_bmn(int M, int N) {
   return umma_idesc_f16(M, N) | (1u << 16);
+}
+
+// Device address of this translation unit's clamp flag on the current device (cached per
+// device; nullptr if it cannot be obtained).
+static inline unsigned int* f16_clamp_flag_here() {
+  static unsigned int* ptr[64] = {nullptr};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  if (!ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_f16_clamped) != cudaSuccess) return nullptr;
+    ptr[dev] = static_cast<unsigned int*>(p);
+  }
+  return ptr[dev];
 }
 
 }  // namespace sgd

@@ -1039,4 +1039,6 @@ cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s) {
   return p.epiw == 4 ? launch_tc<64, 256, 4>(p, a, s) : launch_tc<64, 256, 8>(p, a, s);
 }
 
+unsigned int* f16_clamp_flag_gemm() { return f16_clamp_flag_here(); }
+
 }  // namespace sgd

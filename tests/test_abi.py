@@ -25,7 +25,7 @@ def _declared():
         if f.endswith(".h"):
             src = open(os.path.join(ROOT, "include", f)).read()
             src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-            names |= set(re.findall(r"\b(sgd_[a-z_]+)\s*\(", src))
+            names |= set(re.findall(r"\b(sgd_[a-z0-9_]+)\s*\(", src))
     return names
 
 

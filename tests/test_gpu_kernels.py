@@ -13,6 +13,7 @@ import pytest
 import torch
 
 from oracle import denoiser as odn
+from paper_2609_29505_gb300 import synth
 
 pytestmark = pytest.mark.gpu
 
@@ -299,3 +300,52 @@ def test_gemm_streamk_repeatable(B, M, N, K, epi):
         _check_f16(first[rows], want, extra_abs=extra)
         a, b = _f(first), _f(dp)  # two fp16 roundings of nearly equal sums: 1 ulp apart at most
         assert np.all(np.abs(a - b) <= 2.0 ** -10 * np.abs(b) + extra)
+
+
+def test_f16_clamp_is_reported(B):
+    """An fp16 store that has to clamp (|x| > 65504) raises the clamp flag, which
+    sgd_kernel_f16_clamped reports once and clears; an in-range GEMM leaves it down."""
+    M = N = K = 64
+    A = torch.full((M, K), 300.0, dtype=torch.float16, device="cuda")
+    W = torch.full((N, K), 300.0, dtype=torch.float16, device="cuda")
+    out = torch.empty(M, N, dtype=torch.float16, device="cuda")
+    B.sgd_kernel_f16_clamped()
+    e = B.sgd_epilogue_args(kind=B.EPI_F16, out=out.data_ptr(), ldo=N)
+    B.sgd_kernel_gemm(A, W, M, N, K, e)
+    torch.cuda.synchronize()
+    assert torch.all(out == 65504.0)
+    assert B.sgd_kernel_f16_clamped() == 1
+    assert B.sgd_kernel_f16_clamped() == 0
+    A.fill_(0.5)
+    W.fill_(0.25)
+    B.sgd_kernel_gemm(A, W, M, N, K, e)
+    torch.cuda.synchronize()
+    assert torch.all(out == 8.0)
+    assert B.sgd_kernel_f16_clamped() == 0
+    assert B.sgd_kernel_status() == 0
+
+
+def test_check_device_reports_clamped_activations(B):
+    """A model whose projections overflow fp16 (tiny with W_QKV scaled by 2^17) still runs,
+    and sgd_check_device reports SGD_ERR_RANGE instead of returning silently clamped
+    results; the unscaled model reports nothing."""
+    cfg = synth.get_config("tiny")
+    w = {k: v.cuda() for k, v in synth.make_weights(cfg, "cpu").items()}
+    inp = synth.make_inputs(cfg, "cpu")
+    out = torch.empty(cfg.batch, cfg.n_out_tokens, cfg.out_channels, device="cuda")
+    S = [cfg.T] * cfg.n_units
+    for scale, want in ((1.0, None), (2.0 ** 17, B.SGD_ERR_RANGE)):
+        ws = dict(w)
+        ws["blocks.0.w_qkv"] = (w["blocks.0.w_qkv"].float() * scale).to(torch.bfloat16)
+        B.sgd_kernel_f16_clamped()
+        m = B.Denoiser(cfg, ws)
+        m.set_schedule(cfg.T, S, synth.block_groups(cfg))
+        m.step(inp.z0.cuda(), out, 1000.0, 1)
+        if want is None:
+            m.check_device()
+        else:
+            with pytest.raises(B.SgdError) as err:
+                m.check_device()
+            assert err.value.code == want
+            m.check_device()  # reported once
+        m.close()
