@@ -60,7 +60,37 @@ typedef struct {
   const float* rope_cos;         /* ROPE: fp32 [rope_tokens, d_head / 2] tables, row = token % rope_tokens */
   const float* rope_sin;
   int rope_tokens, d_head, rope_cols;
+  /* Pre-norm folded into the GEMM (Algorithm 2, an active branch's Norm before its first
+   * projection): A holds the un-normalised rows x (fp16), B = W diag(g) (the norm gain
+   * folded into the weight), and before its epilogue each accumulator value of row r, B
+   * row j becomes
+   *   SGD_FNORM_RMS (1): rstd_r acc,  rstd_r = rsqrt(sum_p sq[p][r] / K + norm_eps);
+   *   SGD_FNORM_LN  (2): rstd_r (acc - mean_r colsum[j]) + colbias[j], with mean_r =
+   *                      sum_p s[p][r] / K and rstd_r = rsqrt(sum_p sq[p][r] / K - mean_r^2 + eps),
+   * where sq[p][r] = rstat[p * stat_ld + r] and s[p][r] = rstat[(64 + p) * stat_ld + r] are
+   * the partial row sums of x^2 and x in stat_slots (1..64) slots, added in slot order.
+   * colsum[j] = alpha sum_k B[j, k] and colbias[j] = sum_k b_k W[j, k] (b the LayerNorm shift),
+   * fp32 with at least 512 entries of padding past the last B row.  Not with SGD_EPI_DELTA. */
+  int norm;
+  const float* rstat;
+  int stat_slots, stat_ld;
+  float norm_eps;
+  const float* colsum;
+  const float* colbias;
+  /* Writer of the residual stream (SGD_EPI_DELTA, or SGD_EPI_F32 writing h): with h16 set,
+   * also stores fp16(new h) in h16 (row stride ldh, or ldo for F32) and, per row, the partial
+   * sums of its new values' squares and values over the columns of each half of each output
+   * tile in slot 2 t + half of stat_out (same layout as rstat, stat_out_ld >= M): the
+   * statistics a following SGD_FNORM_* GEMM reads.  The slot count is 2 ceil(N / tile
+   * width); sgd_kernel_gemm_stat_slots returns it. */
+  void* h16;
+  float* stat_out;
+  int stat_out_ld;
 } sgd_epilogue_args;
+
+/* Partial-sum slots a residual writer with these arguments fills (see h16 above). */
+SGD_API int sgd_kernel_gemm_stat_slots(int M, int N, int K, const sgd_epilogue_args* epi,
+                                       int variant, int* slots);
 
 /*
  * C = alpha A B^T.  A fp16 [M, K] (row stride lda elements), B fp16 [N or 2N, K]

@@ -52,6 +52,7 @@ EXPORTED = [
     "sgd_kernel_attention", "sgd_kernel_norm", "sgd_kernel_frozen_run", "sgd_kernel_status",
     "sgd_set_exec_mode", "sgd_step_host_async", "sgd_host_wait", "sgd_kernel_gemm_static_ws",
     "sgd_set_policy", "sgd_get_drift", "sgd_selftest_wait_timeout", "sgd_kernel_f16_clamped",
+    "sgd_kernel_gemm_stat_slots",
 ]
 EXEC_JAGGED_GRAPH, EXEC_EAGER, EXEC_PADDED_GRAPH = 0, 1, 2
 POLICY_STATIC, POLICY_DRIFT = 0, 1
@@ -102,7 +103,11 @@ class sgd_epilogue_args(C.Structure):
                 ("ldh", C.c_int), ("cache", C.c_void_p), ("ld_cache", C.c_int),
                 ("gate", C.c_void_p), ("ld_gate", C.c_int), ("rows_per_batch", C.c_int),
                 ("act", C.c_int), ("rope_cos", C.c_void_p), ("rope_sin", C.c_void_p),
-                ("rope_tokens", C.c_int), ("d_head", C.c_int), ("rope_cols", C.c_int)]
+                ("rope_tokens", C.c_int), ("d_head", C.c_int), ("rope_cols", C.c_int),
+                ("norm", C.c_int), ("rstat", C.c_void_p), ("stat_slots", C.c_int),
+                ("stat_ld", C.c_int), ("norm_eps", C.c_float), ("colsum", C.c_void_p),
+                ("colbias", C.c_void_p), ("h16", C.c_void_p), ("stat_out", C.c_void_p),
+                ("stat_out_ld", C.c_int)]
 
 
 _lib = None
@@ -138,6 +143,7 @@ def lib() -> C.CDLL:
             "sgd_kernel_frozen_run": (i, [vp, C.POINTER(vp), i, i64, vp]),
             "sgd_kernel_status": (i, [C.POINTER(C.c_int)]),
             "sgd_kernel_f16_clamped": (i, [C.POINTER(C.c_int)]),
+            "sgd_kernel_gemm_stat_slots": (i, [i, i, i, C.POINTER(sgd_epilogue_args), i, C.POINTER(C.c_int)]),
             "sgd_set_exec_mode": (i, [vp, i]),
             "sgd_step_host_async": (i, [vp, vp, vp, f, vp, vp, i, vp]),
             "sgd_host_wait": (i, [vp]),
@@ -232,6 +238,13 @@ def sgd_kernel_status() -> int:
     st = C.c_int(0)
     check(lib().sgd_kernel_status(C.byref(st)), "sgd_kernel_status")
     return int(st.value)
+
+
+def sgd_kernel_gemm_stat_slots(M, N, K, epi: "sgd_epilogue_args", variant=0) -> int:
+    n = C.c_int(0)
+    check(lib().sgd_kernel_gemm_stat_slots(M, N, K, C.byref(epi), int(variant), C.byref(n)),
+          "sgd_kernel_gemm_stat_slots")
+    return int(n.value)
 
 
 def sgd_kernel_f16_clamped() -> int:

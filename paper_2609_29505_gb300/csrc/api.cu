@@ -108,6 +108,10 @@ void compile_patterns(int T, int n_units, const int32_t* S, std::vector<int>& pa
 struct PW {
   const f16* w = nullptr;
   float alpha = 1.f;
+  // pre-norm folded into this weight (its gain multiplied into the columns): LayerNorm
+  // column vectors alpha sum_k W'[j, k] and sum_k b_k W[j, k], padded past the last row
+  const float* colsum = nullptr;
+  const float* colbias = nullptr;
 };
 
 struct BlockPW {
@@ -130,6 +134,13 @@ struct sgd_ctx {
   int gemm_bk = 64;   // default K-block of the tcgen05 GEMM
   int exec_mode = SGD_EXEC_JAGGED_GRAPH;
   float* h_pad = nullptr;  // padded mode: residual that discarded branch updates land in
+  // pre-norms folded into the GEMMs (RMSNorm / LayerNorm models): every writer of h also
+  // writes h16 = fp16(h) and partial row sums into rstat; prog_slots = slots the current
+  // writer fills (tracked while a step program is built)
+  bool fold = false;
+  f16* h16 = nullptr;
+  float* rstat = nullptr;
+  int prog_slots = 0;
   // stream-K GEMM workspace, shared by every GEMM of this context (they run one after
   // another on one stream); grown when a new plan needs more, the old buffers stay
   // allocated for graphs captured with them
@@ -249,6 +260,10 @@ const f16* H16(const void* p) { return static_cast<const f16*>(p); }
 int make_gemm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, const f16* A,
                  int lda, const PW& B, int ldb, int M, int N, int K, EpiParams epi) {
   epi.alpha = B.alpha;
+  if (epi.norm == SGD_FNORM_LN) {
+    epi.colsum = B.colsum;
+    epi.colbias = B.colbias;
+  }
   auto plan = std::make_shared<GemmPlan>();
   plan->A = A;
   plan->lda = lda;
@@ -274,6 +289,12 @@ int make_gemm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, cons
     case SGD_EPI_DELTA: out_b = 8.0 * M * N + (epi.cache ? 2.0 * M * N : 0.0); break;
     default: out_b = 2.0 * M * N; break;
   }
+  if (epi.h16) {  // writer of h: its fp16 copy and row sums (slots of this plan's column tiles)
+    const int num_n = (N + plan->bn - 1) / plan->bn;
+    out_b += 2.0 * M * N + 16.0 * M * num_n;
+    c->prog_slots = 2 * num_n;
+  }
+  if (epi.norm != SGD_FNORM_NONE) out_b += 8.0 * M * epi.stat_slots * (epi.norm == SGD_FNORM_LN ? 2 : 1);
   Op op;
   op.name = name;
   op.kernel = plan->simt ? SGD_KERNEL_GEMM_SIMT : SGD_KERNEL_GEMM_TC;
@@ -290,6 +311,43 @@ EpiParams epi_base(int kind) {
   e.alpha = 1.f;
   e.rows_per_batch = 1;
   return e;
+}
+
+// The GEMM that follows a folded pre-norm: A is h16, the epilogue normalises each row with
+// the statistics of the current writer of h.
+void set_folded_norm(sgd_ctx* c, EpiParams& e, int norm_kind) {
+  e.norm = norm_kind == SGD_NORM_RMS ? SGD_FNORM_RMS : SGD_FNORM_LN;
+  e.rstat = c->rstat;
+  e.stat_slots = c->prog_slots;
+  e.stat_ld = c->M;
+  e.norm_eps = c->d.eps;
+  e.norm_inv_d = 1.0f / static_cast<float>(c->d.d);
+}
+
+// A GEMM epilogue that writes h also writes h16 and the row sums.
+void set_h_writer(sgd_ctx* c, EpiParams& e) {
+  e.h16 = c->h16;
+  e.stat_out = c->rstat;
+  e.stat_out_ld = c->M;
+}
+
+// h16 and row sums of h as it stands (after the stem): a frozen run of no units.
+void make_hstat_op(sgd_ctx* c, std::vector<Op>& ops) {
+  FrozenParams p{};
+  p.h = c->h;
+  p.n = static_cast<int64_t>(c->M) * c->d.d;
+  p.rows = c->M;
+  p.d = c->d.d;
+  p.h16 = c->h16;
+  p.stat = c->rstat;
+  Op op;
+  op.name = "h_stats";
+  op.kernel = SGD_KERNEL_FROZEN_RUN;
+  op.flops = 2.0 * p.n;
+  op.bytes = 6.0 * p.n;
+  op.run = [p](cudaStream_t s) { return frozen_launch(p, s); };
+  ops.push_back(std::move(op));
+  c->prog_slots = frozen_stat_slots(c->d.d);
 }
 
 void make_norm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, int kind,
@@ -349,12 +407,19 @@ void flush_run(sgd_ctx* c, std::vector<Op>& ops, std::vector<const f16*>& run, i
     p.h = c->h;
     p.n = static_cast<int64_t>(c->M) * c->d.d;
     p.n_caches = 0;
+    p.rows = c->M;
+    p.d = c->d.d;
+    if (c->fold) {
+      p.h16 = c->h16;
+      p.stat = c->rstat;
+      c->prog_slots = frozen_stat_slots(c->d.d);
+    }
     while (i < run.size() && p.n_caches < kMaxRun) p.caches[p.n_caches++] = run[i++];
     Op op;
     op.name = "frozen_run(u" + std::to_string(first_unit) + "+" + std::to_string(p.n_caches) + ")";
     op.kernel = SGD_KERNEL_FROZEN_RUN;
     op.flops = static_cast<double>(p.n) * p.n_caches;
-    op.bytes = static_cast<double>(p.n) * (8.0 + 2.0 * p.n_caches);
+    op.bytes = static_cast<double>(p.n) * (8.0 + 2.0 * p.n_caches + (c->fold ? 2.0 : 0.0));
     op.run = [p](cudaStream_t s) { return frozen_launch(p, s); };
     ops.push_back(std::move(op));
   }
@@ -376,11 +441,16 @@ int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_c
   delta.ldh = D;
   delta.cache = discard ? nullptr : cache;
   delta.ld_cache = D;
+  if (c->fold && !discard) set_h_writer(c, delta);
+  // the pre-norm's input: h16 with the norm folded into the GEMM, else the norm kernel's output
+  const f16* xin = c->fold ? c->h16 : c->xn;
   int rc;
   if (kind == 0) {  // self-attention
-    make_norm_op(c, ops, pre + "attn.norm", d.norm, W.norm1_w, W.norm1_b, adaln ? mod : nullptr,
-                 adaln ? mod + D : nullptr, 6 * D);
+    if (!c->fold)
+      make_norm_op(c, ops, pre + "attn.norm", d.norm, W.norm1_w, W.norm1_b, adaln ? mod : nullptr,
+                   adaln ? mod + D : nullptr, 6 * D);
     EpiParams e = epi_base(d.rope ? SGD_EPI_ROPE : SGD_EPI_F16);
+    if (c->fold) set_folded_norm(c, e, d.norm);
     e.out = c->qkv;
     e.ldo = 3 * D;
     if (d.rope) {
@@ -390,7 +460,7 @@ int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_c
       e.d_head = d.d_head;
       e.rope_cols = 2 * D;
     }
-    if ((rc = make_gemm_op(c, ops, pre + "attn.qkv", c->xn, D, P.qkv, D, M, 3 * D, D, e)))
+    if ((rc = make_gemm_op(c, ops, pre + "attn.qkv", xin, D, P.qkv, D, M, 3 * D, D, e)))
       return rc;
     AttnParams ap{c->qkv, 3 * D, c->qkv + D, c->qkv + 2 * D, 3 * D, c->attn, D,
                   d.batch, d.n_tokens, d.n_tokens, d.n_heads, d.d_head, c->attn_impl};
@@ -403,25 +473,29 @@ int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_c
     return make_gemm_op(c, ops, pre + "attn.out", c->attn, D, P.o, D, M, D, D, delta);
   }
   if (kind == 1) {  // cross-attention
-    make_norm_op(c, ops, pre + "xattn.norm", SGD_NORM_LN, W.normx_w, W.normx_b, nullptr, nullptr, 0);
+    if (!c->fold)
+      make_norm_op(c, ops, pre + "xattn.norm", SGD_NORM_LN, W.normx_w, W.normx_b, nullptr, nullptr, 0);
     EpiParams e = epi_base(SGD_EPI_F16);
+    if (c->fold) set_folded_norm(c, e, SGD_NORM_LN);
     e.out = c->qkv;
     e.ldo = D;
-    if ((rc = make_gemm_op(c, ops, pre + "xattn.q", c->xn, D, P.xq, D, M, D, D, e))) return rc;
+    if ((rc = make_gemm_op(c, ops, pre + "xattn.q", xin, D, P.xq, D, M, D, D, e))) return rc;
     AttnParams ap{c->qkv, D, c->ctxkv[b], c->ctxkv[b] + D, 2 * D, c->attn, D,
                   d.batch, d.n_tokens, d.ctx_len, d.n_heads, d.d_head, c->attn_impl};
     if ((rc = make_attn_op(c, ops, pre + "xattn.sdpa", ap))) return rc;
     return make_gemm_op(c, ops, pre + "xattn.out", c->attn, D, P.xo, D, M, D, D, delta);
   }
   // MLP
-  make_norm_op(c, ops, pre + "mlp.norm", d.norm, W.norm2_w, W.norm2_b, adaln ? mod + 3 * D : nullptr,
-               adaln ? mod + 4 * D : nullptr, 6 * D);
+  if (!c->fold)
+    make_norm_op(c, ops, pre + "mlp.norm", d.norm, W.norm2_w, W.norm2_b, adaln ? mod + 3 * D : nullptr,
+                 adaln ? mod + 4 * D : nullptr, 6 * D);
   const bool gated = d.mlp == SGD_MLP_SWIGLU || d.mlp == SGD_MLP_GEGLU;
   EpiParams e = epi_base(gated ? SGD_EPI_GATED : SGD_EPI_GELU);
+  if (c->fold) set_folded_norm(c, e, d.norm);
   e.out = c->act;
   e.ldo = F;
   e.act = (d.mlp == SGD_MLP_GEGLU || d.mlp == SGD_MLP_GELU_ERF) ? 1 : 0;
-  if ((rc = make_gemm_op(c, ops, pre + "mlp.up", c->xn, D, P.w1, D, M, F, D, e))) return rc;
+  if ((rc = make_gemm_op(c, ops, pre + "mlp.up", xin, D, P.w1, D, M, F, D, e))) return rc;
   if (adaln) {
     delta.gate = mod + 5 * D;
     delta.ld_gate = 6 * D;
@@ -460,6 +534,7 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
                (d.stem == SGD_STEM_EMBED ? 2.0 * M * D : 0.0);
     op.run = [p](cudaStream_t s) { return stem_launch(p, s); };
     ops.push_back(std::move(op));
+    if (c->fold) make_hstat_op(c, ops);
   }
   if (d.block == SGD_BLOCK_ADALN) {  // conditioning: c = W_t2 silu(W_t1 sin(t)) + class_emb[y]
     GemvParams g{};
@@ -525,6 +600,7 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
       EpiParams e = epi_base(SGD_EPI_F32);
       e.out = c->h;
       e.ldo = D;
+      if (c->fold) set_h_writer(c, e);
       if ((rc = make_gemm_op(c, ops, "b" + std::to_string(b) + ".skip_linear", cat, 2 * D,
                              c->pw_skip[j], 2 * D, M, D, 2 * D, e)))
         return rc;
@@ -600,6 +676,8 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
     ops.push_back(std::move(op));
     return SGD_OK;
   }
+  const float* shift = nullptr;
+  const float* scale = nullptr;
   if (d.head == SGD_HEAD_ADALN_LINEAR) {
     GemvParams g{};
     g.out = c->modf;
@@ -613,15 +691,22 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
     g.K = D;
     g.rows = d.batch;
     make_gemv_op(ops, "head.mod", g);
-    make_norm_op(c, ops, "head.norm", SGD_NORM_LN_PLAIN, nullptr, nullptr, c->modf, c->modf + D, 2 * D);
-  } else {
-    make_norm_op(c, ops, "head.norm", d.norm == SGD_NORM_RMS ? SGD_NORM_RMS : SGD_NORM_LN,
-                 c->w.normf_w, c->w.normf_b, nullptr, nullptr, 0);
+    shift = c->modf;
+    scale = c->modf + D;
   }
   if (d.d_out <= 64 && d.head != SGD_HEAD_LOGITS) {
+    // small heads normalise each fp32 row in the kernel that applies W_head
     HeadParams hp{};
-    hp.x = c->xn;
+    hp.h = c->h;
     hp.ldx = D;
+    hp.norm_kind = d.head == SGD_HEAD_ADALN_LINEAR ? SGD_NORM_LN_PLAIN
+                                                   : (d.norm == SGD_NORM_RMS ? SGD_NORM_RMS : SGD_NORM_LN);
+    hp.g = d.head == SGD_HEAD_ADALN_LINEAR ? nullptr : B16(c->w.normf_w);
+    hp.b = d.head == SGD_HEAD_ADALN_LINEAR || d.norm == SGD_NORM_RMS ? nullptr : B16(c->w.normf_b);
+    hp.shift = shift;
+    hp.scale = scale;
+    hp.ld_mod = 2 * D;
+    hp.eps = d.eps;
     hp.W = B16(c->w.w_head);
     hp.N = d.d_out;
     hp.K = D;
@@ -634,14 +719,20 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
     op.name = "head.linear";
     op.kernel = SGD_KERNEL_SMALL;
     op.flops = 2.0 * M * d.out_channels * D;
-    op.bytes = 2.0 * M * D + 4.0 * M * d.out_channels;
+    op.bytes = 4.0 * M * D + 4.0 * M * d.out_channels;
     op.run = [hp](cudaStream_t s) { return head_small_launch(hp, s); };
     ops.push_back(std::move(op));
     return SGD_OK;
   }
+  const int head_norm = d.norm == SGD_NORM_RMS ? SGD_NORM_RMS : SGD_NORM_LN;
   EpiParams e = epi_base(d.head == SGD_HEAD_LOGITS ? SGD_EPI_F16 : SGD_EPI_F32);
   e.out_slot = out_slot;
   e.ldo = d.head == SGD_HEAD_LOGITS ? d.d_out : d.out_channels;
+  if (c->fold) {
+    set_folded_norm(c, e, head_norm);
+    return make_gemm_op(c, ops, "head.linear", c->h16, D, c->pw_head, D, M, d.d_out, D, e);
+  }
+  make_norm_op(c, ops, "head.norm", head_norm, c->w.normf_w, c->w.normf_b, nullptr, nullptr, 0);
   return make_gemm_op(c, ops, "head.linear", c->xn, D, c->pw_head, D, M, d.d_out, D, e);
 }
 
@@ -756,6 +847,11 @@ int ensure_alloc(sgd_ctx* c) {
   if ((rc = c->alloc(&c->act, M * F, &c->ws_bytes))) return rc;
   if ((rc = c->alloc(&c->slot, 1, &c->ws_bytes))) return rc;
   CUDA_TRY(cudaMemset(c->slot, 0, sizeof(IoSlot)));
+  if (c->fold) {
+    if ((rc = c->alloc(&c->h16, M * D, &c->ws_bytes))) return rc;
+    if ((rc = c->alloc(&c->rstat, 2 * static_cast<size_t>(kStatSlots) * M, &c->ws_bytes))) return rc;
+    CUDA_TRY(cudaMemset(c->rstat, 0, 2 * sizeof(float) * kStatSlots * M));
+  }
   if (d.block == SGD_BLOCK_ADALN) {
     if ((rc = c->alloc(&c->t_hidden, D, &c->ws_bytes))) return rc;
     if ((rc = c->alloc(&c->cond_c, d.batch * D, &c->ws_bytes))) return rc;
@@ -813,6 +909,42 @@ int prep_weight(sgd_ctx* c, const void* src, int64_t n, PW& out) {
   return SGD_OK;
 }
 
+// The same for a weight that consumes a folded pre-norm: fp16(W diag(g) 2^shift) and, for
+// LayerNorm, the column vectors alpha sum_k W'[j, k] (from the fp16 copy, so that it matches
+// what the tensor cores multiply) and sum_k b_k W[j, k].
+int prep_weight_folded(sgd_ctx* c, const void* src, int64_t rows, int K, const void* g, const void* b,
+                       bool ln, PW& out) {
+  f16* dst = nullptr;
+  int rc = c->alloc(&dst, static_cast<size_t>(rows) * K, &c->weight_bytes);
+  if (rc) return rc;
+  CUDA_TRY(cudaMemset(c->absmax, 0, sizeof(float)));
+  CUDA_TRY(absmax_scaled_launch(B16(src), B16(g), rows, K, c->absmax, 0));
+  float m = 0.f;
+  CUDA_TRY(cudaMemcpy(&m, c->absmax, sizeof(float), cudaMemcpyDeviceToHost));
+  int shift = 0;
+  if (m > 0.f && std::isfinite(m)) {
+    shift = static_cast<int>(std::floor(std::log2(65504.0 / m)));
+    shift = std::max(-100, std::min(100, shift));
+  }
+  CUDA_TRY(convert_scaled_launch(B16(src), B16(g), dst, rows, K, shift, 0));
+  out.w = dst;
+  out.alpha = std::ldexp(1.0f, -shift);
+  if (ln) {
+    float* cs = nullptr;
+    float* cb = nullptr;
+    const size_t padded = static_cast<size_t>(rows) + 512;
+    if ((rc = c->alloc(&cs, padded, &c->weight_bytes)) || (rc = c->alloc(&cb, padded, &c->weight_bytes)))
+      return rc;
+    CUDA_TRY(cudaMemset(cs, 0, padded * sizeof(float)));
+    CUDA_TRY(cudaMemset(cb, 0, padded * sizeof(float)));
+    CUDA_TRY(rowsum_f16_launch(dst, rows, K, out.alpha, cs, 0));
+    CUDA_TRY(rowdot_bf16_launch(B16(src), B16(b), rows, K, cb, 0));
+    out.colsum = cs;
+    out.colbias = cb;
+  }
+  return SGD_OK;
+}
+
 int prep_weights(sgd_ctx* c) {
   const sgd_model_desc& d = c->d;
   const int64_t D = d.d, F = d.d_ff;
@@ -823,12 +955,23 @@ int prep_weights(sgd_ctx* c) {
   for (int b = 0; b < d.n_blocks; ++b) {
     const sgd_block_weights& W = c->blk[b];
     BlockPW& P = c->pw[b];
-    if ((rc = prep_weight(c, W.w_qkv, 3 * D * D, P.qkv))) return rc;
+    const bool ln = d.norm == SGD_NORM_LN;
+    if (c->fold) {
+      if ((rc = prep_weight_folded(c, W.w_qkv, 3 * D, D, W.norm1_w, W.norm1_b, ln, P.qkv)) ||
+          (rc = prep_weight_folded(c, W.w_1, (gated ? 2 : 1) * F, D, W.norm2_w, W.norm2_b, ln, P.w1)))
+        return rc;
+    } else if ((rc = prep_weight(c, W.w_qkv, 3 * D * D, P.qkv)) ||
+               (rc = prep_weight(c, W.w_1, (gated ? 2 : 1) * F * D, P.w1))) {
+      return rc;
+    }
     if ((rc = prep_weight(c, W.w_o, D * D, P.o))) return rc;
-    if ((rc = prep_weight(c, W.w_1, (gated ? 2 : 1) * F * D, P.w1))) return rc;
     if ((rc = prep_weight(c, W.w_2, D * F, P.w2))) return rc;
     if (d.block == SGD_BLOCK_XATTN) {
-      if ((rc = prep_weight(c, W.wx_q, D * D, P.xq))) return rc;
+      if (c->fold)
+        rc = prep_weight_folded(c, W.wx_q, D, D, W.normx_w, W.normx_b, true, P.xq);
+      else
+        rc = prep_weight(c, W.wx_q, D * D, P.xq);
+      if (rc) return rc;
       if ((rc = prep_weight(c, W.wx_kv, 2 * D * d.d_ctx, P.xkv))) return rc;
       if ((rc = prep_weight(c, W.wx_o, D * D, P.xo))) return rc;
     }
@@ -837,8 +980,14 @@ int prep_weights(sgd_ctx* c) {
   for (int j = 0; j < d.n_skips; ++j)
     if ((rc = prep_weight(c, c->skip_w[j], D * 2 * D, c->pw_skip[j]))) return rc;
   const bool tc_head = d.head == SGD_HEAD_LOGITS || (d.head == SGD_HEAD_LINEAR && d.d_out > 64);
-  if (tc_head && (rc = prep_weight(c, c->w.w_head, static_cast<int64_t>(d.d_out) * D, c->pw_head)))
-    return rc;
+  if (tc_head) {
+    if (c->fold)
+      rc = prep_weight_folded(c, c->w.w_head, d.d_out, static_cast<int>(D), c->w.normf_w, c->w.normf_b,
+                              d.norm == SGD_NORM_LN, c->pw_head);
+    else
+      rc = prep_weight(c, c->w.w_head, static_cast<int64_t>(d.d_out) * D, c->pw_head);
+    if (rc) return rc;
+  }
   CUDA_TRY(cudaDeviceSynchronize());
   return SGD_OK;
 }
@@ -939,6 +1088,10 @@ int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out) 
   }
   c->M = desc->batch * desc->n_tokens;
   c->attn_impl = (desc->flags & SGD_FLAG_MMA_SYNC_ATTENTION) ? 1 : 0;
+  // RMSNorm / LayerNorm pre-norms fold into the GEMMs that follow them; the AdaLN
+  // modulation (a per-sample scale of the weight's columns) and the SIMT debug GEMM do not
+  c->fold = (desc->norm == SGD_NORM_RMS || desc->norm == SGD_NORM_LN) &&
+            !(desc->flags & SGD_FLAG_SIMT_GEMM);
   c->nbr = desc->block == SGD_BLOCK_XATTN ? 3 : 2;
   c->U = desc->n_blocks * c->nbr;
   if ((rc = ensure_alloc(c)) || (rc = prep_weights(c))) {
@@ -1511,6 +1664,17 @@ int kernel_gemm_plan(const void* A, int lda, const void* B, int ldb, int M, int 
   e.rope_cols = ea->rope_cols;
   e.M = M;
   e.N = N;
+  e.norm = ea->norm;
+  e.rstat = ea->rstat;
+  e.stat_slots = ea->stat_slots;
+  e.stat_ld = ea->stat_ld;
+  e.norm_eps = ea->norm_eps;
+  e.norm_inv_d = 1.0f / static_cast<float>(K);
+  e.colsum = ea->colsum;
+  e.colbias = ea->colbias;
+  e.h16 = static_cast<f16*>(ea->h16);
+  e.stat_out = ea->stat_out;
+  e.stat_out_ld = ea->stat_out_ld;
   const char* why = "";
   const int rc = gemm_plan(p, &why);
   if (rc) return fail(rc == -5 ? SGD_ERR_CUDA : (rc == -1 ? SGD_ERR_ARG : SGD_ERR_SHAPE), why);
@@ -1611,6 +1775,19 @@ int sgd_selftest_wait_timeout(void* stream) {
   int* p = device_status_ptr();
   if (!p) return fail(SGD_ERR_CUDA, "status word unavailable");
   CUDA_TRY(wait_selftest_launch(p, SGD_SELFTEST_TIMEOUT_CODE, static_cast<cudaStream_t>(stream)));
+  return SGD_OK;
+}
+
+int sgd_kernel_gemm_stat_slots(int M, int N, int K, const sgd_epilogue_args* ea, int variant, int* slots) {
+  if (!slots || !ea) return fail(SGD_ERR_ARG, "null argument");
+  // the tile width is chosen on the host from the shape alone; plan with dummy aligned operands
+  static const uint4 dummy[1] = {};
+  sgd_epilogue_args e = *ea;
+  GemmPlan p;
+  p.encode = false;
+  int rc = kernel_gemm_plan(dummy, K, dummy, K, M, N, K, &e, variant, p);
+  if (rc) return rc;
+  *slots = p.simt ? 0 : 2 * ((N + p.bn - 1) / p.bn);
   return SGD_OK;
 }
 

@@ -2,8 +2,10 @@
 //   frozen_run   — Algorithm 2, frozen branch: h_{l,s} = h_{l-1,s} + Delta_{l, r_l(s)}
 //                  for a run of consecutive frozen units in one read-modify-write of h
 //                  (16-byte vectors: 8 fp32 of h, 8 fp16 of each cached update).
-//   norm         — pre-norm of an active branch (RMSNorm / LayerNorm / AdaLN modulate),
-//                  fp32 residual in, fp16 GEMM operand out.
+//   frozen_rows  — the same for models whose pre-norms are folded into the GEMMs, also
+//                  writing fp16(h) and the partial row sums the next GEMM normalises with.
+//   norm         — pre-norm of an active branch where it cannot be folded (the AdaLN
+//                  modulate of DiT-style blocks), fp32 residual in, fp16 GEMM operand out.
 //   stem, gemv, head_small, copy_out, pack_f16 — the always-on parts around the
 //                  scheduled units (input stage, conditioning, output head, U-ViT skip
 //                  operands), Sec. 4.2: conditioning and skip features stay current.
@@ -271,6 +273,53 @@ __global__ void __launch_bounds__(256) frozen_kernel(const __grid_constant__ Fro
   }
 }
 
+// Frozen run for models whose pre-norms are folded into the GEMMs: also the writer of h's
+// fp16 copy and row sums.  Warp w of the grid takes chunk (row, ch) of kStatChunk columns;
+// each lane handles 8 consecutive columns per 256-column step, adds the cached updates in
+// cache order (the same fp32 arithmetic as frozen_kernel), stores h and fp16(h), and the
+// warp reduces its sums with a fixed xor tree into stat slot ch.
+__global__ void __launch_bounds__(256) frozen_rows_kernel(const __grid_constant__ FrozenParams p) {
+  const int nch = (p.d + kStatChunk - 1) / kStatChunk;
+  const int64_t wid = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (wid >= static_cast<int64_t>(p.rows) * nch) return;
+  const int lane = threadIdx.x & 31;
+  const int row = static_cast<int>(wid / nch), ch = static_cast<int>(wid % nch);
+  const int c1 = min(p.d, (ch + 1) * kStatChunk);
+  float ss = 0.f, s1 = 0.f;
+  for (int c = ch * kStatChunk + lane * 8; c < c1; c += 256) {
+    const int64_t i = (static_cast<int64_t>(row) * p.d + c) >> 3;
+    float4* hp = reinterpret_cast<float4*>(p.h) + 2 * i;
+    const float4 a = hp[0], b = hp[1];
+    float acc[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+    for (int k = 0; k < p.n_caches; ++k) {
+      const uint4 u = __ldcs(reinterpret_cast<const uint4*>(p.caches[k]) + i);
+      float f[8];
+      unpack_f16x8(u, f);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) acc[q] += f[q];
+    }
+    if (p.n_caches) {
+      hp[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+      hp[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+    }
+    reinterpret_cast<uint4*>(p.h16)[i] = pack_f16x8(acc);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      ss = fmaf(acc[q], acc[q], ss);
+      s1 += acc[q];
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+  }
+  if (lane == 0) {
+    p.stat[static_cast<int64_t>(ch) * p.rows + row] = ss;
+    p.stat[static_cast<int64_t>(kStatSlots + ch) * p.rows + row] = s1;
+  }
+}
+
 __global__ void io_set_kernel(IoSlot* slot, const IoSlot v) { *slot = v; }
 
 // sinusoid(t, dim)[c] = cos(t w_i) for c < half, sin(t w_{c-half}) otherwise,
@@ -413,7 +462,15 @@ __global__ void __launch_bounds__(256) gemv_kernel(const GemvParams p) {
   }
 }
 
-// One warp per row; W rows re-read from L1.
+// One warp per row: the row's mean and rstd from the fp32 residual stream (two passes, as the
+// norm kernels), then every output channel's dot product with the normalised row formed on
+// the fly (fp32; W rows re-read from L1).
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
 __global__ void __launch_bounds__(256) head_small_kernel(const HeadParams p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t r = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + warp;
@@ -424,19 +481,46 @@ __global__ void __launch_bounds__(256) head_small_kernel(const HeadParams p) {
   float* out = reinterpret_cast<float*>(p.slot->out) +
                (static_cast<int64_t>(b) * (p.n_tokens - p.n_prefix) + (n - p.n_prefix)) *
                    p.out_channels;
-  const f16* x = p.x + r * p.ldx;
+  const float* x = p.h + r * p.ldx;
+  float mean = 0.f;
+  if (p.norm_kind != SGD_NORM_RMS) {
+    float s1 = 0.f;
+    for (int k = lane * 4; k < p.K; k += 128) {
+      const float4 v = *reinterpret_cast<const float4*>(x + k);
+      s1 += (v.x + v.y) + (v.z + v.w);
+    }
+    mean = warp_sum(s1) / p.K;
+  }
+  float sq = 0.f;
+  for (int k = lane * 4; k < p.K; k += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(x + k);
+    const float a0 = v.x - mean, a1 = v.y - mean, a2 = v.z - mean, a3 = v.w - mean;
+    sq += (a0 * a0 + a1 * a1) + (a2 * a2 + a3 * a3);
+  }
+  const float rstd = rsqrtf(warp_sum(sq) / p.K + p.eps);
+  const float* sh = p.shift ? p.shift + static_cast<int64_t>(b) * p.ld_mod : nullptr;
+  const float* sc = p.scale ? p.scale + static_cast<int64_t>(b) * p.ld_mod : nullptr;
   for (int j = 0; j < p.out_channels; ++j) {
     const bf16* w = p.W + static_cast<int64_t>(j) * p.K;
     float acc = 0.f;
     for (int k = lane * 8; k < p.K; k += 256) {
-      float fx[8], fw[8];
-      unpack_f16x8(*reinterpret_cast<const uint4*>(x + k), fx);
+      const float4 va = *reinterpret_cast<const float4*>(x + k);
+      const float4 vb = *reinterpret_cast<const float4*>(x + k + 4);
+      float fx[8] = {va.x, va.y, va.z, va.w, vb.x, vb.y, vb.z, vb.w}, fw[8];
       unpack_bf16x8(*reinterpret_cast<const uint4*>(w + k), fw);
+      float g[8], bb[8];
+      if (p.g) unpack_bf16x8(*reinterpret_cast<const uint4*>(p.g + k), g);
+      if (p.b) unpack_bf16x8(*reinterpret_cast<const uint4*>(p.b + k), bb);
 #pragma unroll
-      for (int q = 0; q < 8; ++q) acc = fmaf(fx[q], fw[q], acc);
+      for (int q = 0; q < 8; ++q) {
+        float y = (fx[q] - mean) * rstd;
+        if (p.g) y *= g[q];
+        if (p.b) y += bb[q];
+        if (sc) y = y * (1.f + sc[k + q]) + sh[k + q];
+        acc = fmaf(y, fw[q], acc);
+      }
     }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    acc = warp_sum(acc);
     if (lane == 0) out[j] = acc;
   }
 }
@@ -490,6 +574,48 @@ __global__ void convert_bf16_f16_kernel(const bf16* w, f16* dst, int64_t n, floa
     dst[i] = __float2half_rn(sat_f16(__bfloat162float(w[i]) * scale));
 }
 
+// max |W[j, k] g[k]| (non-negative floats compared as integers, as absmax_bf16_kernel).
+__global__ void absmax_scaled_kernel(const bf16* w, const bf16* g, int64_t n, int K, float* out) {
+  __shared__ float red[8];
+  float m = 0.f;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n; i += stride)
+    m = fmaxf(m, fabsf(__bfloat162float(w[i]) * __bfloat162float(g[i % K])));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = m;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int i = 1; i < (blockDim.x >> 5); ++i) m = fmaxf(m, red[i]);
+    atomicMax(reinterpret_cast<int*>(out), __float_as_int(m));
+  }
+}
+
+// dst = fp16(W[j, k] g[k] 2^shift): the product of two bf16 values is exact in fp32, and
+// is rounded once to fp16.
+__global__ void convert_scaled_kernel(const bf16* w, const bf16* g, f16* dst, int64_t n, int K,
+                                      float scale) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n; i += stride)
+    dst[i] = __float2half_rn(sat_f16(__bfloat162float(w[i]) * __bfloat162float(g[i % K]) * scale));
+}
+
+// One warp per row j: out[j] = scale sum_k W[j, k] (x[k] or 1), accumulated in double.
+template <typename TW>
+__global__ void rowdot_kernel(const TW* w, const bf16* x, int64_t rows, int K, float scale, float* out) {
+  const int64_t j = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (j >= rows) return;
+  double acc = 0.0;
+  for (int k = lane; k < K; k += 32) {
+    const double wv = static_cast<double>(static_cast<float>(w[j * K + k]));
+    acc += x ? wv * static_cast<double>(__bfloat162float(x[k])) : wv;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  if (lane == 0) out[j] = static_cast<float>(acc * scale);
+}
+
 __global__ void sampler_kernel(float* z, const float* eps, float alpha, float beta, int64_t n) {
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n; i += stride)
@@ -531,6 +657,12 @@ cudaError_t drift_reduce_launch(const float* partials, int n_groups, double* sum
 }
 
 cudaError_t frozen_launch(const FrozenParams& p, cudaStream_t s) {
+  if (p.h16) {
+    if (!p.stat || p.d % 8 || p.rows < 1 || frozen_stat_slots(p.d) > kStatSlots) return cudaErrorInvalidValue;
+    const int64_t warps = static_cast<int64_t>(p.rows) * frozen_stat_slots(p.d);
+    frozen_rows_kernel<<<static_cast<unsigned>((warps + 7) / 8), 256, 0, s>>>(p);
+    return cudaGetLastError();
+  }
   frozen_kernel<<<grid_for(p.n / 8, 256), 256, 0, s>>>(p);
   return cudaGetLastError();
 }
@@ -592,6 +724,29 @@ cudaError_t absmax_bf16_launch(const bf16* w, int64_t n, float* out, cudaStream_
 
 cudaError_t convert_bf16_f16_launch(const bf16* w, f16* dst, int64_t n, int shift, cudaStream_t s) {
   convert_bf16_f16_kernel<<<grid_for(n, 256), 256, 0, s>>>(w, dst, n, ldexpf(1.0f, shift));
+  return cudaGetLastError();
+}
+
+cudaError_t absmax_scaled_launch(const bf16* w, const bf16* g, int64_t rows, int K, float* out,
+                                 cudaStream_t s) {
+  absmax_scaled_kernel<<<grid_for(rows * K, 256), 256, 0, s>>>(w, g, rows * K, K, out);
+  return cudaGetLastError();
+}
+
+cudaError_t convert_scaled_launch(const bf16* w, const bf16* g, f16* dst, int64_t rows, int K, int shift,
+                                  cudaStream_t s) {
+  convert_scaled_kernel<<<grid_for(rows * K, 256), 256, 0, s>>>(w, g, dst, rows * K, K, ldexpf(1.0f, shift));
+  return cudaGetLastError();
+}
+
+cudaError_t rowsum_f16_launch(const f16* w, int64_t rows, int K, float scale, float* out, cudaStream_t s) {
+  rowdot_kernel<f16><<<static_cast<unsigned>((rows + 7) / 8), 256, 0, s>>>(w, nullptr, rows, K, scale, out);
+  return cudaGetLastError();
+}
+
+cudaError_t rowdot_bf16_launch(const bf16* w, const bf16* x, int64_t rows, int K, float* out,
+                               cudaStream_t s) {
+  rowdot_kernel<bf16><<<static_cast<unsigned>((rows + 7) / 8), 256, 0, s>>>(w, x, rows, K, 1.f, out);
   return cudaGetLastError();
 }
 

@@ -230,21 +230,87 @@ __device__ __forceinline__ void store_partial(float* slot, int r, uint32_t tbase
   }
 }
 
+// Folded pre-norm (EpiParams::norm): the row's rstd and mean from the partial sums the
+// last writer of h left, summed in slot order (the same order on every run).
+struct RowNorm {
+  float rstd, mean;
+};
+
+__device__ __forceinline__ RowNorm row_norm(const EpiParams& e, int row, bool row_ok) {
+  RowNorm n{1.f, 0.f};
+  if (e.norm == SGD_FNORM_NONE) return n;
+  const int r = row_ok ? row : 0;
+  float ss = 0.f, s1 = 0.f;
+  for (int p = 0; p < e.stat_slots; ++p) ss += e.rstat[static_cast<int64_t>(p) * e.stat_ld + r];
+  if (e.norm == SGD_FNORM_RMS) {
+    n.rstd = rsqrtf(ss * e.norm_inv_d + e.norm_eps);
+    return n;
+  }
+  for (int p = 0; p < e.stat_slots; ++p)
+    s1 += e.rstat[static_cast<int64_t>(kStatSlots + p) * e.stat_ld + r];
+  const double mean = static_cast<double>(s1) * e.norm_inv_d;
+  const double var = fmax(static_cast<double>(ss) * e.norm_inv_d - mean * mean, 0.0);
+  n.mean = static_cast<float>(mean);
+  n.rstd = rsqrtf(static_cast<float>(var) + e.norm_eps);
+  return n;
+}
+
+// Apply the folded norm to 16 accumulator values whose B rows are brow .. brow + 15
+// (colsum / colbias are padded past the last B row, so the loads need no guard).
+__device__ __forceinline__ void apply_norm16(const EpiParams& e, const RowNorm& n, int brow, float* v) {
+  if (e.norm == SGD_FNORM_RMS) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] *= n.rstd;
+  } else if (e.norm == SGD_FNORM_LN) {
+    const float4* cs = reinterpret_cast<const float4*>(e.colsum + brow);
+    const float4* cb = reinterpret_cast<const float4*>(e.colbias + brow);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4 u = cs[q], w = cb[q];
+      v[4 * q] = n.rstd * (v[4 * q] - n.mean * u.x) + w.x;
+      v[4 * q + 1] = n.rstd * (v[4 * q + 1] - n.mean * u.y) + w.y;
+      v[4 * q + 2] = n.rstd * (v[4 * q + 2] - n.mean * u.z) + w.z;
+      v[4 * q + 3] = n.rstd * (v[4 * q + 3] - n.mean * u.w) + w.w;
+    }
+  }
+}
+
+// Writer of h: the fp16 copy of 8 new values of h and their contribution to the row sums.
+__device__ __forceinline__ void emit_h8(const EpiParams& e, int ld, int row, int col, const float* hv,
+                                        float& ss, float& s1) {
+  store8_f16(e.h16, ld, row, col, hv);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    ss = fmaf(hv[i], hv[i], ss);
+    s1 += hv[i];
+  }
+}
+
+__device__ __forceinline__ void emit_stats(const EpiParams& e, int row, int slot, float ss, float s1) {
+  e.stat_out[static_cast<int64_t>(slot) * e.stat_out_ld + row] = ss;
+  e.stat_out[static_cast<int64_t>(kStatSlots + slot) * e.stat_out_ld + row] = s1;
+}
+
 // Epilogue of one 128 x BN accumulator: this thread owns tile row `row` and handles
 // accumulator columns [cb, ce) (gated: output columns [cb, ce) of the BN / 2 the tile
-// produces), reading the accumulator through `src`.
+// produces), reading the accumulator through `src`.  `part` (0 or 1) is the column half
+// the thread covers, `halves` the number of halves (1 with 4 epilogue warps): a writer of h
+// puts its row sums in stat slot 2 n_blk + part.
 template <int BN, bool kFastRope, class Src>
 __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int row, int n_blk,
-                                              const Src& src, int cb, int ce) {
+                                              const Src& src, int cb, int ce, int part, int halves) {
   constexpr int kBN = BN;
   const EpiParams& e = a.epi;
   const bool row_ok = row < a.M;
+  const RowNorm rn = row_norm(e, row, row_ok);
   float x[16], y[16];
   if (a.gated) {
     const int n0 = n_blk * (kBN / 2);
     for (int c = cb; c < ce; c += 16) {
       if (n0 + c >= a.N) break;
       src.load2(c, kBN / 2 + c, x, y);
+      apply_norm16(e, rn, n0 + c, x);
+      apply_norm16(e, rn, a.N + n0 + c, y);
 #pragma unroll
       for (int i = 0; i < 16; ++i) x[i] = e.act ? x[i] * gelu_erf_f(y[i]) : silu_f(x[i]) * y[i];
       if (row_ok) {
@@ -290,6 +356,8 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
         if (n0 + hb >= a.N) break;
         const bool rot = (n0 + hb) < e.rope_cols;
         src.load2(hb + j, hb + hd + j, x, y);
+        apply_norm16(e, rn, n0 + hb + j, x);
+        apply_norm16(e, rn, n0 + hb + hd + j, y);
         if (rot && row_ok) {
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
@@ -317,6 +385,8 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
       const bool rot = (n0 + hb) < e.rope_cols;
       for (int j = 0; j < hd; j += 16) {
         src.load2(hb + j, hb + hd + j, x, y);
+        apply_norm16(e, rn, n0 + hb + j, x);
+        apply_norm16(e, rn, n0 + hb + hd + j, y);
         if (rot && row_ok) {
           const float* cs = e.rope_cos + static_cast<int64_t>(pos) * hd + j;
           const float* sn = e.rope_sin + static_cast<int64_t>(pos) * hd + j;
@@ -345,6 +415,7 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
     const float* grow =
         e.gate ? e.gate + static_cast<int64_t>(row_ok ? row / e.rows_per_batch : 0) * e.ld_gate + n0 : nullptr;
     float* hrow = e.h + static_cast<int64_t>(row) * e.ldh + n0;
+    float st_ss = 0.f, st_s1 = 0.f;
     for (int c = cb; c < ce; c += 32) {
       if (n0 + c >= a.N) break;
       // unconditional loads (a predicated load here makes the compiler spill): columns past
@@ -374,21 +445,42 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
           hp[0] = h0;
           hp[1] = h1;
           if (e.cache) store8_f16(e.cache, e.ld_cache, row, n0 + c + 8 * g, v);
+          if (e.h16) {
+            const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+            emit_h8(e, e.ldh, row, n0 + c + 8 * g, hv, st_ss, st_s1);
+          }
         }
       }
     }
+    if (e.stat_out && row_ok) {
+      emit_stats(e, row, 2 * n_blk + part, st_ss, st_s1);
+      if (halves == 1) emit_stats(e, row, 2 * n_blk + 1, 0.f, 0.f);
+    }
     return;
   }
+  float st_ss = 0.f, st_s1 = 0.f;
   for (int c = cb; c < ce; c += 32) {
     if (n0 + c >= a.N) break;
     src.load2(c, c + 16, x, y);
+    apply_norm16(e, rn, n0 + c, x);
+    apply_norm16(e, rn, n0 + c + 16, y);
     if (row_ok) {
 #pragma unroll
       for (int q = 0; q < 2; ++q) {
-        if (n0 + c + 8 * q < a.N) epi_store8(e, out, row, n0 + c + 8 * q, x + 8 * q);
-        if (n0 + c + 16 + 8 * q < a.N) epi_store8(e, out, row, n0 + c + 16 + 8 * q, y + 8 * q);
+        if (n0 + c + 8 * q < a.N) {
+          epi_store8(e, out, row, n0 + c + 8 * q, x + 8 * q);
+          if (e.h16) emit_h8(e, e.ldo, row, n0 + c + 8 * q, x + 8 * q, st_ss, st_s1);
+        }
+        if (n0 + c + 16 + 8 * q < a.N) {
+          epi_store8(e, out, row, n0 + c + 16 + 8 * q, y + 8 * q);
+          if (e.h16) emit_h8(e, e.ldo, row, n0 + c + 16 + 8 * q, y + 8 * q, st_ss, st_s1);
+        }
       }
     }
+  }
+  if (e.stat_out && row_ok) {
+    emit_stats(e, row, 2 * n_blk + part, st_ss, st_s1);
+    if (halves == 1) emit_stats(e, row, 2 * n_blk + 1, 0.f, 0.f);
   }
 }
 
@@ -630,7 +722,8 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
       if (u >= w.n_sk) {  // data-parallel tile
         if (!warp_wait(&tfull[acc], aph, abort_flag, a.status, 4)) break;
         tc_fence_after();
-        epilogue_tile<kBN, kEpiWarps == 4>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce);
+        epilogue_tile<kBN, kEpiWarps == 4>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce, part,
+                                           kEpiWarps == 8 ? 2 : 1);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -642,7 +735,8 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
       if (k0 == 0 && k1 == a.num_k) {  // the whole K range of the tile lies in this CTA's share
         if (ok) {
           tc_fence_after();
-          epilogue_tile<kBN, kEpiWarps == 4>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce);
+          epilogue_tile<kBN, kEpiWarps == 4>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce, part,
+                                           kEpiWarps == 8 ? 2 : 1);
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -674,7 +768,8 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
       epi_bar(kEpiThreads);
       if (*last_flag != 0) {
         __threadfence();
-        epilogue_tile<kBN, kEpiWarps == 4>(a, out, row, n_blk, WsSrc<kBN>{slot0, nseg, q * 32 + lane, a.epi.alpha}, cb, ce);
+        epilogue_tile<kBN, kEpiWarps == 4>(a, out, row, n_blk, WsSrc<kBN>{slot0, nseg, q * 32 + lane, a.epi.alpha},
+                                           cb, ce, part, kEpiWarps == 8 ? 2 : 1);
         if (threadIdx.x == 64) a.sk_cnt[tile] = 0;
       }
     }
@@ -932,7 +1027,32 @@ int gemm_plan(GemmPlan& p, const char** why) {
     *why = "gemm: RoPE epilogue needs d_head 64 or 128 and cos/sin tables";
     return -2;
   }
-  if (p.simt) return 0;
+  if (e.norm != SGD_FNORM_NONE) {
+    if (e.norm != SGD_FNORM_RMS && e.norm != SGD_FNORM_LN) {
+      *why = "gemm: bad folded-norm kind";
+      return -1;
+    }
+    if (!e.rstat || e.stat_slots < 1 || e.stat_slots > kStatSlots || e.stat_ld < p.M ||
+        (e.norm == SGD_FNORM_LN && (!e.colsum || !e.colbias)) || e.kind == SGD_EPI_DELTA) {
+      *why = "gemm: folded norm needs row statistics (1..64 slots, stat_ld >= M), LN column "
+             "vectors, and a non-residual epilogue";
+      return -2;
+    }
+  }
+  if (e.h16) {
+    if ((e.kind != SGD_EPI_DELTA && e.kind != SGD_EPI_F32) || !e.stat_out || e.stat_out_ld < p.M ||
+        !aligned16(e.h16)) {
+      *why = "gemm: the fp16 copy of h needs a DELTA or F32 epilogue and a statistics buffer";
+      return -2;
+    }
+  }
+  if (p.simt) {
+    if (e.norm != SGD_FNORM_NONE || e.h16) {
+      *why = "gemm: the SIMT kernel has no folded norm";
+      return -2;
+    }
+    return 0;
+  }
   const int b_rows = gated ? 2 * p.N : p.N;
   if (p.bk != 64 && p.bk != 32) p.bk = 64;
   const int num_m = (p.M + kBM - 1) / kBM;
@@ -963,12 +1083,16 @@ int gemm_plan(GemmPlan& p, const char** why) {
   if (p.bn == 224) p.sk = 0;
   if (p.epiw == 0) p.epiw = (e.kind == SGD_EPI_ROPE || gated) ? 4 : 8;
   if (p.bn == 128 || p.bn == 224 || p.bk == 32) p.epiw = 8;
-  if (!make_tmap_f16(&p.tmap_a, p.A, p.M, p.K, p.lda, 128, p.bk) ||
-      !make_tmap_f16(&p.tmap_b, p.B, b_rows, p.K, p.ldb, p.bn == 224 ? 224 : 128, p.bk)) {
+  if (p.encode && (!make_tmap_f16(&p.tmap_a, p.A, p.M, p.K, p.lda, 128, p.bk) ||
+                   !make_tmap_f16(&p.tmap_b, p.B, b_rows, p.K, p.ldb, p.bn == 224 ? 224 : 128, p.bk))) {
     *why = "gemm: cuTensorMapEncodeTiled failed (driver entry point unavailable or bad layout)";
     return -5;
   }
   const int num_n = gated ? (p.N + 127) / 128 : (p.N + p.bn - 1) / p.bn;
+  if (e.h16 && 2 * num_n > kStatSlots) {
+    *why = "gemm: too many column tiles for the row-statistics slots";
+    return -2;
+  }
   const int units = num_m * num_n;
   p.grid = units < sms ? units : sms;
   p.sk_tiles = p.sk_ctas = p.max_seg = 0;

@@ -38,7 +38,30 @@ struct EpiParams {
   int rope_cols;
   int M;
   int N;  // output columns (gated: f)
+  // Pre-norm folded into the GEMM (A = fp16 copy of the residual stream h, the norm gain
+  // folded into B): per row, rstd (and for LayerNorm the mean) come from the partial row
+  // sums the last writer of h left in `rstat`; accumulator column j (B row j) becomes
+  // RMS: rstd * acc_j;  LN: rstd * (acc_j - mean * colsum_j) + colbias_j.
+  int norm;               // SGD_FNORM_NONE / _RMS / _LN
+  const float* rstat;     // partial sums: slot p of row r at rstat[p * stat_ld + r] (sum of
+                          // squares), rstat[(kStatSlots + p) * stat_ld + r] (sum)
+  int stat_slots;         // slots the writer of h filled
+  int stat_ld;            // rows between slots (M)
+  float norm_eps;
+  float norm_inv_d;       // 1 / K
+  const float* colsum;    // LN: alpha * sum_k B[j, k] per B row
+  const float* colbias;   // LN: sum_k b_k W[j, k] per B row (the shift through the weight)
+  // Writer of h (DELTA, and F32 with h16 set): also store fp16(h_new) in h16 (ld = ldh, or
+  // ldo for F32) and the row's partial sums over this thread's columns in slot
+  // 2 * n_blk + part of stat_out (part: which column half of the tile).
+  f16* h16;
+  float* stat_out;
+  int stat_out_ld;
 };
+
+// Row-statistics buffer: kStatSlots slots of sums of squares, then kStatSlots of sums.
+constexpr int kStatSlots = 64;
+enum { SGD_FNORM_NONE = 0, SGD_FNORM_RMS = 1, SGD_FNORM_LN = 2 };
 
 // A planned GEMM: operands, epilogue and prebuilt TMA descriptors.
 struct GemmPlan {
@@ -53,6 +76,7 @@ struct GemmPlan {
   int bn = 0;                // output columns per tile: 256, 128, or 0 = choose by tile count
   int epiw = 0;              // epilogue warps: 4, 8, or 0 = choose by epilogue kind
   int sk = -1;               // stream-K for the tiles after the last full wave: -1 choose, 0 off, 1 on
+  bool encode = true;        // false: choose the tiling only (no tensor maps; operands unused)
   CUtensorMap tmap_a;
   CUtensorMap tmap_b;
   int grid = 0;
@@ -123,15 +147,23 @@ struct NormParams {
 };
 cudaError_t norm_launch(const NormParams& p, cudaStream_t s);
 
-// Frozen run: h += sum caches.
+// Frozen run: h += sum caches (in cache order, fp32).  With h16 set, the rows are
+// processed in chunks of kStatChunk columns (one warp per chunk) and each chunk also
+// stores fp16(h) into h16 and its partial row sums into stat slot `chunk` (sum of squares,
+// and the sum at kStatSlots + chunk); n_caches may then be 0 (statistics of h only).
 constexpr int kMaxRun = 96;
+constexpr int kStatChunk = 1024;
 struct FrozenParams {
   float* h;
   const f16* caches[kMaxRun];
   int n_caches;
   int64_t n;
+  int rows, d;       // row structure (used with h16)
+  f16* h16;
+  float* stat;       // [2 kStatSlots][rows]
 };
 cudaError_t frozen_launch(const FrozenParams& p, cudaStream_t s);
+inline int frozen_stat_slots(int d) { return (d + kStatChunk - 1) / kStatChunk; }
 
 // Lagged-drift reduction of the input-aware policy (App. B.1) for one scheduled group:
 // partial[b] = (sum (h - snap)^2, sum h^2) over block b's elements (fp32, fixed order),
@@ -192,10 +224,19 @@ struct GemvParams {
 };
 cudaError_t gemv_launch(const GemvParams& p, cudaStream_t s);
 
-// Row-wise small-N linear for heads: out[r, j] = x[r] . W[j] for j < N (N <= 64).
+// Row-wise small-N linear for heads: out[r, j] = norm(h[r]) . W[j] for j < N (N <= 64); the
+// norm (RMSNorm, LayerNorm, or LayerNorm without affine then the AdaLN modulation
+// x (1 + scale_b) + shift_b) is computed from the fp32 row in the same kernel.
 struct HeadParams {
-  const f16* x;        // [rows_total, K] fp16 (normalised states)
+  const float* h;      // [rows_total, K] fp32 residual stream
   int ldx;
+  int norm_kind;       // sgd_norm_kind
+  const bf16* g;
+  const bf16* b;
+  const float* shift;  // AdaLN: [batch, ld_mod]
+  const float* scale;
+  int ld_mod;
+  float eps;
   const bf16* W;       // [N, K]
   int N, K;
   int batch, n_tokens, n_prefix;  // rows r = b * n_tokens + n, n >= n_prefix are output
@@ -215,6 +256,17 @@ cudaError_t pack_f16_launch(f16* dst, int ld_dst, int col0, const float* h, int 
 // conversion dst = fp16(w * 2^shift); also plain bf16 -> fp16 conversion (shift 0).
 cudaError_t absmax_bf16_launch(const bf16* w, int64_t n, float* out, cudaStream_t s);
 cudaError_t convert_bf16_f16_launch(const bf16* w, f16* dst, int64_t n, int shift, cudaStream_t s);
+// Folded pre-norm gain: W[j, k] g[k] for a bf16 [rows, K] weight and bf16 gain [K] — the
+// max |W g| (absmax, *out starting at 0) and the conversion dst = fp16(W g 2^shift).
+cudaError_t absmax_scaled_launch(const bf16* w, const bf16* g, int64_t rows, int K, float* out,
+                                 cudaStream_t s);
+cudaError_t convert_scaled_launch(const bf16* w, const bf16* g, f16* dst, int64_t rows, int K, int shift,
+                                  cudaStream_t s);
+// out[j] = scale * sum_k W[j, k] x[k] per row j of an fp16 (x = 1) or bf16 (x bf16 [K])
+// [rows, K] matrix, accumulated in double.
+cudaError_t rowsum_f16_launch(const f16* w, int64_t rows, int K, float scale, float* out, cudaStream_t s);
+cudaError_t rowdot_bf16_launch(const bf16* w, const bf16* x, int64_t rows, int K, float* out,
+                               cudaStream_t s);
 
 cudaError_t sampler_launch(float* z, const float* eps, float alpha, float beta, int64_t n,
                            cudaStream_t s);

@@ -349,3 +349,129 @@ def test_check_device_reports_clamped_activations(B):
             assert err.value.code == want
             m.check_device()  # reported once
         m.close()
+
+
+# ---------------------------------------------------------------------------
+# pre-norm folded into the GEMM (the north-star's fused norm + projection)
+# ---------------------------------------------------------------------------
+
+FOLD_VARIANTS = [0, 3, 5, 6, 7, 9]
+FOLD_IDS = ["tcgen05", "tcgen05_bk32", "tcgen05_epi4", "tcgen05_epi8", "tcgen05_bn128",
+            "tcgen05_streamk"]
+
+
+def _row_stats(x, slots):
+    """Partial row sums of x^2 and x over `slots` column blocks (test input: any partition
+    is valid), in the kernel layout [2 * 64, M]."""
+    M, K = x.shape
+    st = np.zeros((128, M), np.float32)
+    edges = np.linspace(0, K, slots + 1).astype(int)
+    for p in range(slots):
+        blk = x[:, edges[p]:edges[p + 1]].astype(np.float64)
+        st[p] = np.sum(blk * blk, axis=1)
+        st[64 + p] = np.sum(blk, axis=1)
+    return st
+
+
+@pytest.mark.parametrize("variant", FOLD_VARIANTS, ids=FOLD_IDS)
+@pytest.mark.parametrize("norm", ["rms", "ln"])
+@pytest.mark.parametrize("epi", ["f16", "rope", "gated", "gelu", "f32"])
+def test_gemm_folded_norm(B, norm, epi, variant):
+    """norm(x) W^T with the norm's gain folded into B and rstd (and the LayerNorm mean /
+    shift) applied in the epilogue, against the oracle's norm followed by its linear map
+    and epilogue function, on ragged shapes."""
+    rng = np.random.default_rng(31 + variant)
+    H, dh, n_tok, bsz = 3, 64, 70, 3
+    K = H * dh
+    M = bsz * n_tok
+    N = {"rope": 3 * K, "gated": 328, "gelu": 520, "f16": 264, "f32": 264}[epi]
+    b_rows = 2 * N if epi == "gated" else N
+    x = (rng.standard_normal((M, K)) * 2.0 + rng.standard_normal((M, 1)) * 0.7).astype(np.float32)
+    g = torch.from_numpy(1.0 + 0.1 * rng.standard_normal(K).astype(np.float32)).to(torch.bfloat16)
+    bsh = torch.from_numpy(0.1 * rng.standard_normal(K).astype(np.float32)).to(torch.bfloat16)
+    W = _rand(rng, (b_rows, K), 1 / math.sqrt(K), torch.bfloat16)
+    Wg = (W.float() * g.float()).half()                      # gain folded, one fp16 rounding
+    colsum = np.zeros(b_rows + 512, np.float32)
+    colsum[:b_rows] = Wg.double().sum(dim=1).numpy()
+    colbias = np.zeros(b_rows + 512, np.float32)
+    colbias[:b_rows] = (W.double() @ bsh.double()).numpy()
+    slots = 3
+    st = torch.from_numpy(_row_stats(x, slots)).cuda()
+    A = torch.from_numpy(x).half().cuda()
+    out = torch.empty(M, N, dtype=torch.float32 if epi == "f32" else torch.float16, device="cuda")
+    kind = {"f16": B.EPI_F16, "rope": B.EPI_ROPE, "gated": B.EPI_GATED, "gelu": B.EPI_GELU,
+            "f32": B.EPI_F32}[epi]
+    cs, cb = torch.from_numpy(colsum).cuda(), torch.from_numpy(colbias).cuda()
+    e = B.sgd_epilogue_args(kind=kind, out=out.data_ptr(), ldo=N, norm=1 if norm == "rms" else 2,
+                            rstat=st.data_ptr(), stat_slots=slots, stat_ld=M, norm_eps=1e-6,
+                            colsum=cs.data_ptr(), colbias=cb.data_ptr(), act=1 if epi == "gelu" else 0)
+    if epi == "rope":
+        half = dh // 2
+        pos = np.arange(n_tok, dtype=np.float64)[:, None]
+        freq = 10000.0 ** (-np.arange(half) * 2.0 / dh)
+        cos = torch.from_numpy(np.cos(pos * freq).astype(np.float32)).cuda()
+        sin = torch.from_numpy(np.sin(pos * freq).astype(np.float32)).cuda()
+        e.rope_cos, e.rope_sin = cos.data_ptr(), sin.data_ptr()
+        e.rope_tokens, e.d_head, e.rope_cols = n_tok, dh, 2 * K
+    B.sgd_kernel_gemm(A, Wg.cuda(), M, N, K, e, use_simt=variant)
+    torch.cuda.synchronize()
+    assert B.sgd_kernel_status() == 0
+    if norm == "rms":
+        xn = odn.rms_norm(x, g.float().numpy(), 1e-6)
+    else:
+        xn = odn.layer_norm(x, g.float().numpy(), bsh.float().numpy(), 1e-6)
+    u = odn.linear(xn, W.float().numpy())
+    if epi == "gated":
+        want = odn.silu(u[:, :N]) * u[:, N:]
+    elif epi == "gelu":
+        want = odn.gelu_erf(u)
+    elif epi == "rope":
+        qkv = u.reshape(bsz, n_tok, 3, H, dh)
+        want = qkv.copy()
+        for j in range(2):
+            t = qkv[:, :, j].transpose(0, 2, 1, 3)
+            want[:, :, j] = odn.rope(t, np.arange(n_tok), 10000.0).transpose(0, 2, 1, 3)
+        want = want.reshape(M, N)
+    else:
+        want = u
+    # fp16 rounding of x and of W g (2^-11 each) on top of the fp16 output rounding
+    _check_f16(out, want, extra_abs=3e-3 * float(np.sqrt(np.mean(want.astype(np.float64) ** 2))))
+
+
+@pytest.mark.parametrize("variant", [0, 5, 7, 9, 10], ids=["tcgen05", "epi4", "bn128", "streamk", "bn224"])
+@pytest.mark.parametrize("kind", ["delta", "f32"])
+def test_gemm_residual_writer_emits_h16_and_row_sums(B, kind, variant):
+    """A writer of the residual stream also stores fp16(h_new) (bit-exact against torch's
+    rounding of the same fp32 values) and, per row, partial sums of h_new^2 and h_new whose
+    slot sums equal the full row sums."""
+    rng = np.random.default_rng(41 + variant)
+    M, N, K = 300, 1032 if variant != 10 else 4096, 512
+    if variant == 9:
+        M, N, K = 4096, 4096, 4096
+    A = _rand(rng, (M, K)).cuda()
+    W = _rand(rng, (N, K), 1 / math.sqrt(K)).cuda()
+    h = torch.from_numpy(rng.standard_normal((M, N)).astype(np.float32)).cuda()
+    h16 = torch.empty(M, N, dtype=torch.float16, device="cuda")
+    st = torch.full((128, M), float("nan"), device="cuda")
+    if kind == "delta":
+        e = B.sgd_epilogue_args(kind=B.EPI_DELTA, h=h.data_ptr(), ldh=N, h16=h16.data_ptr(),
+                                stat_out=st.data_ptr(), stat_out_ld=M)
+    else:
+        e = B.sgd_epilogue_args(kind=B.EPI_F32, out=h.data_ptr(), ldo=N, h16=h16.data_ptr(),
+                                stat_out=st.data_ptr(), stat_out_ld=M)
+    slots = B.sgd_kernel_gemm_stat_slots(M, N, K, e, variant)
+    assert 2 <= slots <= 64 and slots % 2 == 0
+    h0 = h.clone()
+    B.sgd_kernel_gemm(A, W, M, N, K, e, use_simt=variant)
+    torch.cuda.synchronize()
+    assert B.sgd_kernel_status() == 0
+    rows = np.sort(rng.choice(M, 48, replace=False))
+    u = odn.linear(_f(A[rows]), _f(W))
+    want = (_f(h0[rows]) if kind == "delta" else 0.0) + u
+    np.testing.assert_allclose(_f(h[rows]), want, rtol=2e-5, atol=2e-5)
+    assert torch.equal(h16, h.half())
+    hv = h.double()
+    ss = st[:slots].double().sum(dim=0)
+    s1 = st[64:64 + slots].double().sum(dim=0)
+    torch.testing.assert_close(ss, (hv * hv).sum(dim=1), rtol=2e-5, atol=1e-3)
+    torch.testing.assert_close(s1, hv.sum(dim=1), rtol=2e-5, atol=1e-2)
