@@ -105,7 +105,10 @@ SGD_API int sgd_kernel_gemm_stat_slots(int M, int N, int K, const sgd_epilogue_a
  * rejected with SGD_ERR_ARG; 5, 6, 7 force 128 x 256 tiles with 4 epilogue warps, 128 x 256 with 8, and
  * 128 x 128 with 8 and no stream-K (128 x 128 applies to plain, GELU and DELTA epilogues
  * only); 8 is 0 without stream-K, 9 is 0 with stream-K whenever the last wave is partial;
- * 10 forces 128 x 224 tiles (5 pipeline stages, no stream-K; plain, GELU and DELTA only).
+ * 10 forces 128 x 224 tiles (5 pipeline stages, no stream-K; plain, GELU and DELTA only);
+ * 11 and 12 are 0 with the tiles visited M-fastest, and in groups of 16 row-blocks (each
+ * group column by column, every other group backwards), instead of the choice made by 0
+ * (groups where there are at least two groups and two waves).
  * The stream-K workspace is owned by the library, one per (device, stream), allocated
  * or grown by the first call that needs it (after synchronising that stream).
  */

@@ -1626,8 +1626,8 @@ int kernel_gemm_plan(const void* A, int lda, const void* B, int ldb, int M, int 
                      const sgd_epilogue_args* ea, int variant, GemmPlan& p) {
   if (!ea) return fail(SGD_ERR_ARG, "null epilogue");
   if (ea->kind < 0 || ea->kind > SGD_EPI_ROPE) return fail(SGD_ERR_ARG, "bad epilogue kind");
-  if (variant < 0 || variant > 10 || variant == 2 || variant == 4)
-    return fail(SGD_ERR_ARG, "gemm: variant must be 0, 1, 3 or 5..10");
+  if (variant < 0 || variant > 12 || variant == 2 || variant == 4)
+    return fail(SGD_ERR_ARG, "gemm: variant must be 0, 1, 3 or 5..12");
   p.A = H16(A);
   p.lda = lda;
   p.B = H16(B);
@@ -1643,6 +1643,8 @@ int kernel_gemm_plan(const void* A, int lda, const void* B, int ldb, int M, int 
   if (variant == 8) p.sk = 0;
   if (variant == 9) p.sk = 1;
   if (variant == 10) { p.bn = 224; p.epiw = 8; }
+  if (variant == 11) p.group_m = 0;
+  if (variant == 12) p.group_m = 16;
   EpiParams& e = p.epi;
   e = EpiParams{};
   e.kind = ea->kind;

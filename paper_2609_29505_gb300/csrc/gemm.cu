@@ -68,6 +68,7 @@ struct TcArgs {
   EpiParams epi;
   int M, N, K;  // N = output columns
   int num_m, num_n, num_k;
+  int group_m;  // tile order: 0 = M-fastest; G = groups of G row-blocks, see tile_coords
   int gated;    // B second half starts at row N (= f)
   int* status;
   // stream-K (0 tiles: data-parallel only)
@@ -520,6 +521,26 @@ __device__ __forceinline__ void epi_bar(int nthreads) {
   asm volatile("bar.sync 1, %0;" ::"r"(nthreads) : "memory");
 }
 
+// Output tile of linear tile index t.  group_m = 0: M-fastest (m = t % num_m).  group_m = G:
+// the row-blocks form groups of G; a group's tiles come one after another, column by column
+// (G row-blocks of one column, then the next column), and every other group walks its
+// columns backwards.  A wave of CTAs then covers about G row-blocks by (CTAs / G) columns,
+// so its A rows are shared by all of its columns, and consecutive groups start on the
+// columns the previous one ended on (still in L2).
+__device__ __forceinline__ void tile_coords(const TcArgs& a, int t, int& m_blk, int& n_blk) {
+  if (a.group_m <= 0) {
+    m_blk = t % a.num_m;
+    n_blk = t / a.num_m;
+    return;
+  }
+  const int per_group = a.group_m * a.num_n;
+  const int g = t / per_group, w = t - g * per_group;
+  const int gm = min(a.group_m, a.num_m - g * a.group_m);  // row-blocks in this (last) group
+  const int col = w / gm;
+  m_blk = g * a.group_m + (w - col * gm);
+  n_blk = (g & 1) ? a.num_n - 1 - col : col;
+}
+
 // Stream-K split of the K iterations of tiles [0, sk_tiles): CTA c < sk_ctas owns the
 // contiguous iterations [start(c), start(c + 1)) of the sk_tiles * num_k iteration space,
 // start(c) = floor(c * total / sk_ctas); every CTA owns at least one iteration (the host
@@ -633,7 +654,8 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
       for (int u = 0; u < w.n_units; ++u) {
         int tile, k0, k1;
         unit_at(a, w, u, tile, k0, k1);
-        const int m_blk = tile % num_mu, n_blk = tile / num_mu;
+        int m_blk, n_blk;
+        tile_coords(a, tile, m_blk, n_blk);
         const int rb0 = a.gated ? n_blk * 128 : n_blk * kBN;
         const int rb1 = a.gated ? a.N + n_blk * 128 : rb0 + 128;  // BN = 256 only
         bool ok = true;
@@ -714,7 +736,8 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
     for (int u = 0; u < w.n_units; ++u) {
       int tile, k0, k1;
       unit_at(a, w, u, tile, k0, k1);
-      const int m_blk = tile % num_mu, n_blk = tile / num_mu;
+      int m_blk, n_blk;
+      tile_coords(a, tile, m_blk, n_blk);
       const int acc = u & 1;
       const uint32_t aph = (u >> 1) & 1;
       const int row = m_blk * kBM + q * 32 + lane;
@@ -1095,6 +1118,10 @@ int gemm_plan(GemmPlan& p, const char** why) {
   }
   const int units = num_m * num_n;
   p.grid = units < sms ? units : sms;
+  // tile order: groups of 16 row-blocks where there are several groups and several waves
+  // (a 152-tile wave then spans ~16 x 9.5 tiles, about balanced between A and B bytes for
+  // 224- and 256-column tiles); M-fastest otherwise
+  if (p.group_m < 0) p.group_m = (num_m >= 32 && num_n >= 4 && units >= 2 * sms) ? 16 : 0;
   p.sk_tiles = p.sk_ctas = p.max_seg = 0;
   if (p.sk != 0) {
     const SkSplit k = sk_split(units, num_k, sms, p.sk == 1);
@@ -1149,6 +1176,7 @@ cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s) {
   a.num_m = (p.M + kBM - 1) / kBM;
   a.num_n = a.gated ? (p.N + 127) / 128 : (p.N + p.bn - 1) / p.bn;
   a.num_k = (p.K + p.bk - 1) / p.bk;
+  a.group_m = p.group_m;
   a.status = device_status_ptr();
   a.sk_tiles = p.sk_tiles;
   a.sk_ctas = p.sk_ctas;

@@ -77,6 +77,7 @@ struct GemmPlan {
   int epiw = 0;              // epilogue warps: 4, 8, or 0 = choose by epilogue kind
   int sk = -1;               // stream-K for the tiles after the last full wave: -1 choose, 0 off, 1 on
   bool encode = true;        // false: choose the tiling only (no tensor maps; operands unused)
+  int group_m = -1;          // tile order: -1 choose, 0 M-fastest, G > 0 groups of G row-blocks
   CUtensorMap tmap_a;
   CUtensorMap tmap_b;
   int grid = 0;

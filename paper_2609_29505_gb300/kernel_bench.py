@@ -110,7 +110,7 @@ def main():
     ap.add_argument("--simt", type=int, default=0,
                     help="sgd_kernel_gemm variant: 0 tcgen05 (auto), 1 SIMT, 3 BK 32, "
                          "5 4 epilogue warps, 6 8 warps, 7 128-column tiles, 8 no stream-K, "
-                         "9 stream-K forced, 10 128 x 224 tiles")
+                         "9 stream-K forced, 10 128 x 224 tiles, 11 M-fastest tile order, 12 grouped tile order")
     ap.add_argument("--tokens", type=int, default=1024)
     ap.add_argument("--batch", type=int, default=4)
     ap.add_argument("--heads", type=int, default=32)

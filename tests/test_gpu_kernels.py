@@ -48,9 +48,10 @@ def _check_f16(got, want, extra_abs=0.0):
 
 
 # sgd_kernel_gemm variant codes (include/sgd_kernels.h)
-VARIANTS = [0, 3, 5, 6, 7, 8, 9, 10, 1]
+VARIANTS = [0, 3, 5, 6, 7, 8, 9, 10, 11, 12, 1]
 VARIANT_IDS = ["tcgen05", "tcgen05_bk32", "tcgen05_epi4",
-               "tcgen05_epi8", "tcgen05_bn128", "tcgen05_dp", "tcgen05_streamk", "tcgen05_bn224", "simt"]
+               "tcgen05_epi8", "tcgen05_bn128", "tcgen05_dp", "tcgen05_streamk", "tcgen05_bn224",
+               "tcgen05_mfast", "tcgen05_grouped", "simt"]
 
 GEMM_SHAPES = [(64, 256, 256), (300, 520, 688), (129, 264, 72), (1000, 1376, 512), (4128, 1024, 2048)]
 
