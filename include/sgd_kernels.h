@@ -142,12 +142,26 @@ SGD_API int sgd_kernel_gemm_static_ws(const void* A, int lda, const void* B, int
  * columns [h d_head, (h+1) d_head).  fp16 in and out; d_head in {64, 72, 128};
  * leading dimensions in elements, multiples of 8.  impl = 0: tcgen05 for d_head 64 / 128
  * (S, P and O in TMEM; two 128-query tiles per CTA whose softmax warpgroups alternate with
- * each other's MMAs), the mma.sync kernel for 72; 1: the mma.sync kernel for every d_head;
+ * each other's MMAs), the mma.sync kernel for 72 (see sgd_kernel_attention_hs for 72 on
+ * tcgen05); 1: the mma.sync kernel for every d_head;
  * 2: tcgen05 with one query tile per CTA and P in shared memory; 3: the same as 0.
  */
 SGD_API int sgd_kernel_attention(const void* q, int ldq, const void* k, const void* v, int ldkv,
                          void* o, int ldo, int batch, int n_q, int n_kv, int n_heads,
                          int d_head, int impl, void* stream);
+
+/*
+ * sgd_kernel_attention with the input heads `head_stride` columns apart (head h of q, k, v
+ * at columns [h head_stride, h head_stride + d_head); head_stride >= d_head, a multiple of
+ * 8); o keeps d_head columns per head.  With d_head 72, impl 0 / 3 run the tcgen05 kernel
+ * when head_stride >= 80: each head is read as 80 columns (one 64-column and one
+ * 16-column block), so columns [72, 80) after every Q head must be zero and those after
+ * every K and V head finite (a layout whose gaps are zero, as sgd_step uses, satisfies
+ * both); with head_stride 72 they fall back to the mma.sync kernel.
+ */
+SGD_API int sgd_kernel_attention_hs(const void* q, int ldq, const void* k, const void* v, int ldkv,
+                                    int head_stride, void* o, int ldo, int batch, int n_q, int n_kv,
+                                    int n_heads, int d_head, int impl, void* stream);
 
 /*
  * out fp16 [rows, d] = norm(h fp32 [rows, d]); kind = sgd_norm_kind.  g, b: bf16 [d]

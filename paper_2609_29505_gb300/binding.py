@@ -52,7 +52,7 @@ EXPORTED = [
     "sgd_kernel_attention", "sgd_kernel_norm", "sgd_kernel_frozen_run", "sgd_kernel_status",
     "sgd_set_exec_mode", "sgd_step_host_async", "sgd_host_wait", "sgd_kernel_gemm_static_ws",
     "sgd_set_policy", "sgd_get_drift", "sgd_selftest_wait_timeout", "sgd_kernel_f16_clamped",
-    "sgd_kernel_gemm_stat_slots",
+    "sgd_kernel_gemm_stat_slots", "sgd_kernel_attention_hs",
 ]
 EXEC_JAGGED_GRAPH, EXEC_EAGER, EXEC_PADDED_GRAPH = 0, 1, 2
 POLICY_STATIC, POLICY_DRIFT = 0, 1
@@ -139,6 +139,7 @@ def lib() -> C.CDLL:
             "sgd_kernel_gemm": (i, [vp, i, vp, i, i, i, i, C.POINTER(sgd_epilogue_args), i, vp]),
             "sgd_kernel_gemm_static_ws": (i, [vp, i, vp, i, i, i, i, C.POINTER(sgd_epilogue_args), i, vp]),
             "sgd_kernel_attention": (i, [vp, i, vp, vp, i, vp, i, i, i, i, i, i, i, vp]),
+            "sgd_kernel_attention_hs": (i, [vp, i, vp, vp, i, i, vp, i, i, i, i, i, i, i, vp]),
             "sgd_kernel_norm": (i, [vp, vp, i, i, i, vp, vp, vp, vp, i, i, f, vp]),
             "sgd_kernel_frozen_run": (i, [vp, C.POINTER(vp), i, i64, vp]),
             "sgd_kernel_status": (i, [C.POINTER(C.c_int)]),
@@ -219,6 +220,13 @@ def sgd_kernel_attention(q, ldq, k, v, ldkv, o, ldo, batch, n_q, n_kv, n_heads, 
     return check(lib().sgd_kernel_attention(_ptr(q), ldq, _ptr(k), _ptr(v), ldkv, _ptr(o), ldo,
                                             batch, n_q, n_kv, n_heads, d_head, impl,
                                             _stream(stream)), "sgd_kernel_attention")
+
+
+def sgd_kernel_attention_hs(q, ldq, k, v, ldkv, head_stride, o, ldo, batch, n_q, n_kv, n_heads,
+                            d_head, impl=0, stream=None):
+    return check(lib().sgd_kernel_attention_hs(_ptr(q), ldq, _ptr(k), _ptr(v), ldkv, head_stride,
+                                               _ptr(o), ldo, batch, n_q, n_kv, n_heads, d_head,
+                                               impl, _stream(stream)), "sgd_kernel_attention_hs")
 
 
 def sgd_kernel_norm(h, out, rows, d, kind, g=None, b=None, shift=None, scale=None, ld_mod=0,

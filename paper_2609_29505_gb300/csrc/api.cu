@@ -131,6 +131,7 @@ struct sgd_ctx {
   int device = 0;
   int M = 0, U = 0, nbr = 0;
   int attn_impl = 0;  // 1: mma.sync attention everywhere (SGD_FLAG_MMA_SYNC_ATTENTION)
+  int head_stride = 0;  // columns per head in qkv: d_head, or 80 for d_head 72 on tcgen05
   int gemm_bk = 64;   // default K-block of the tcgen05 GEMM
   int exec_mode = SGD_EXEC_JAGGED_GRAPH;
   float* h_pad = nullptr;  // padded mode: residual that discarded branch updates land in
@@ -451,8 +452,13 @@ int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_c
                    adaln ? mod + D : nullptr, 6 * D);
     EpiParams e = epi_base(d.rope ? SGD_EPI_ROPE : SGD_EPI_F16);
     if (c->fold) set_folded_norm(c, e, d.norm);
+    const int HS = c->head_stride, QW = d.n_heads * HS;  // qkv: [M, 3 QW], head h of Q at h HS
     e.out = c->qkv;
-    e.ldo = 3 * D;
+    e.ldo = 3 * QW;
+    if (HS != d.d_head) {
+      e.pad_src = d.d_head;
+      e.pad_dst = HS;
+    }
     if (d.rope) {
       e.rope_cos = c->rope_cos;
       e.rope_sin = c->rope_sin;
@@ -462,8 +468,8 @@ int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_c
     }
     if ((rc = make_gemm_op(c, ops, pre + "attn.qkv", xin, D, P.qkv, D, M, 3 * D, D, e)))
       return rc;
-    AttnParams ap{c->qkv, 3 * D, c->qkv + D, c->qkv + 2 * D, 3 * D, c->attn, D,
-                  d.batch, d.n_tokens, d.n_tokens, d.n_heads, d.d_head, c->attn_impl};
+    AttnParams ap{c->qkv, 3 * QW, c->qkv + QW, c->qkv + 2 * QW, 3 * QW, c->attn, D,
+                  d.batch, d.n_tokens, d.n_tokens, d.n_heads, d.d_head, c->attn_impl, HS};
     if ((rc = make_attn_op(c, ops, pre + "attn.sdpa", ap))) return rc;
     if (adaln) {
       delta.gate = mod + 2 * D;
@@ -481,7 +487,7 @@ int build_branch(sgd_ctx* c, std::vector<Op>& ops, int b, int kind, bool write_c
     e.ldo = D;
     if ((rc = make_gemm_op(c, ops, pre + "xattn.q", xin, D, P.xq, D, M, D, D, e))) return rc;
     AttnParams ap{c->qkv, D, c->ctxkv[b], c->ctxkv[b] + D, 2 * D, c->attn, D,
-                  d.batch, d.n_tokens, d.ctx_len, d.n_heads, d.d_head, c->attn_impl};
+                  d.batch, d.n_tokens, d.ctx_len, d.n_heads, d.d_head, c->attn_impl, 0};
     if ((rc = make_attn_op(c, ops, pre + "xattn.sdpa", ap))) return rc;
     return make_gemm_op(c, ops, pre + "xattn.out", c->attn, D, P.xo, D, M, D, D, delta);
   }
@@ -842,7 +848,11 @@ int ensure_alloc(sgd_ctx* c) {
   int rc;
   if ((rc = c->alloc(&c->h, M * D, &c->ws_bytes))) return rc;
   if ((rc = c->alloc(&c->xn, M * D, &c->ws_bytes))) return rc;
-  if ((rc = c->alloc(&c->qkv, M * 3 * D, &c->ws_bytes))) return rc;
+  // d_head 72 on tcgen05: heads padded to 80 columns in qkv, the gaps zero (never written)
+  c->head_stride = (d.d_head == 72 && c->attn_impl == 0) ? 80 : d.d_head;
+  const size_t QW = static_cast<size_t>(d.n_heads) * c->head_stride;
+  if ((rc = c->alloc(&c->qkv, M * 3 * QW, &c->ws_bytes))) return rc;
+  CUDA_TRY(cudaMemset(c->qkv, 0, M * 3 * QW * sizeof(f16)));
   if ((rc = c->alloc(&c->attn, M * D, &c->ws_bytes))) return rc;
   if ((rc = c->alloc(&c->act, M * F, &c->ws_bytes))) return rc;
   if ((rc = c->alloc(&c->slot, 1, &c->ws_bytes))) return rc;
@@ -1734,10 +1744,17 @@ int sgd_kernel_gemm_static_ws(const void* A, int lda, const void* B, int ldb, in
 int sgd_kernel_attention(const void* q, int ldq, const void* k, const void* v, int ldkv, void* o,
                          int ldo, int batch, int n_q, int n_kv, int n_heads, int d_head, int impl,
                          void* stream) {
+  return sgd_kernel_attention_hs(q, ldq, k, v, ldkv, d_head, o, ldo, batch, n_q, n_kv, n_heads, d_head,
+                                 impl, stream);
+}
+
+int sgd_kernel_attention_hs(const void* q, int ldq, const void* k, const void* v, int ldkv, int head_stride,
+                            void* o, int ldo, int batch, int n_q, int n_kv, int n_heads, int d_head,
+                            int impl, void* stream) {
   if (impl < 0 || impl > 3) return fail(SGD_ERR_ARG, "attention: impl must be in 0..3");
   AttnPlan plan;
   plan.p = AttnParams{H16(q), ldq, H16(k), H16(v), ldkv, static_cast<f16*>(o), ldo,
-                      batch, n_q, n_kv, n_heads, d_head, impl};
+                      batch, n_q, n_kv, n_heads, d_head, impl, head_stride};
   const char* why = "";
   const int rc = attn_plan(plan, &why);
   if (rc) return fail(rc == -1 ? SGD_ERR_ARG : (rc == -5 ? SGD_ERR_CUDA : SGD_ERR_SHAPE), why);

@@ -82,9 +82,10 @@ __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnParams p) {
   const int q0 = blockIdx.x * kBQ;
   const int bh = blockIdx.y;
   const int b = bh / p.n_heads, h = bh % p.n_heads;
-  const f16* qbase = p.q + (static_cast<int64_t>(b) * p.n_q) * p.ldq + h * DH;
-  const f16* kbase = p.k + (static_cast<int64_t>(b) * p.n_kv) * p.ldkv + h * DH;
-  const f16* vbase = p.v + (static_cast<int64_t>(b) * p.n_kv) * p.ldkv + h * DH;
+  const int hs = p.head_stride > 0 ? p.head_stride : DH;  // input columns between heads
+  const f16* qbase = p.q + (static_cast<int64_t>(b) * p.n_q) * p.ldq + h * hs;
+  const f16* kbase = p.k + (static_cast<int64_t>(b) * p.n_kv) * p.ldkv + h * hs;
+  const f16* vbase = p.v + (static_cast<int64_t>(b) * p.n_kv) * p.ldkv + h * hs;
 
   // Q tile
   for (int i = tid; i < kBQ * kPadChunks; i += kWarps * 32) {
@@ -272,6 +273,11 @@ struct AttnTcArgs {
   CUtensorMap tmap_q;
   CUtensorMap tmap_k;
   CUtensorMap tmap_v;
+  // d_h = 72 (heads padded to 80 columns in the input): boxes of the last 16 columns
+  CUtensorMap tmap_q16;
+  CUtensorMap tmap_k16;
+  CUtensorMap tmap_v16;
+  int head_stride;  // input columns between heads
   f16* o;
   int ldo;
   int n_q, n_kv, n_heads;
@@ -360,7 +366,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const __grid_con
     if (lane == 0) {
       mbar_arrive_expect_tx(q_full, L::kAtoms * kAtom);
       for (int at = 0; at < L::kAtoms; ++at)
-        tma_load_2d(sm + L::kQ + at * kAtom, &a.tmap_q, q_full, h * DH + at * 64,
+        tma_load_2d(sm + L::kQ + at * kAtom, &a.tmap_q, q_full, h * a.head_stride + at * 64,
                     b * a.n_q + qt * kTcBQ);
       int j = 0;
       for (; j < nt; ++j) {
@@ -370,8 +376,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const __grid_con
         mbar_arrive_expect_tx(&kv_full[s], 2 * L::kAtoms * kAtom);
         const int row = b * a.n_kv + j * kTcBK;
         for (int at = 0; at < L::kAtoms; ++at) {
-          tma_load_2d(st + at * kAtom, &a.tmap_k, &kv_full[s], h * DH + at * 64, row);
-          tma_load_2d(st + (L::kAtoms + at) * kAtom, &a.tmap_v, &kv_full[s], h * DH + at * 64, row);
+          tma_load_2d(st + at * kAtom, &a.tmap_k, &kv_full[s], h * a.head_stride + at * 64, row);
+          tma_load_2d(st + (L::kAtoms + at) * kAtom, &a.tmap_v, &kv_full[s], h * a.head_stride + at * 64, row);
         }
       }
       if (*abort_flag) {
@@ -553,17 +559,29 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const __grid_con
 constexpr int kPpThreads = 320;
 constexpr int kPpBQ = 256;
 
+// d_h 64 / 128: every 128-row operand tile is d_h / 64 atoms of 64 columns (128-byte swizzle).
+// d_h 72: the input heads are padded to 80 columns (columns 72..79 of Q zero), and a tile is
+// one 64-column atom plus one 16-column atom (32-byte swizzle); Q K^T runs K = 80 (five
+// K = 16 steps), P V runs as an N = 64 and an N = 16 instruction, O keeps 80 TMEM columns of
+// which the first 72 are stored.
+constexpr int kAtom32 = 128 * 16 * 2;  // 128 rows x 16 fp16: one 32-byte-swizzle column block
+
 template <int DH>
 struct PpLayout {
-  static constexpr int kAtoms = DH / 64;
-  static constexpr int kQ = 0;                        // Q tile t: atoms at kQ + (t kAtoms + a) kAtom
-  static constexpr int kKV = 2 * kAtoms * kAtom;      // stage s: K atoms, then V atoms
-  static constexpr int kStage = 2 * kAtoms * kAtom;
+  static constexpr bool kPad = DH == 72;
+  static constexpr int kA64 = DH / 64;                // 64-column atoms per tile
+  static constexpr int kA16 = kPad ? 1 : 0;           // 16-column atoms per tile
+  static constexpr int kDP = 64 * kA64 + 16 * kA16;   // head width the MMAs see
+  static constexpr int kTile = kA64 * kAtom + kA16 * kAtom32;
+  static constexpr int kQ = 0;                        // Q tile t at kQ + t kTile
+  static constexpr int kKV = 2 * kTile;               // stage s: the K tile, then the V tile
+  static constexpr int kStage = 2 * kTile;
   static constexpr int kBar = kKV + 2 * kStage;
   static constexpr int kBytes = kBar + 256 + 1024;
   static constexpr uint32_t kTmemS = 0;               // S_t at columns 128 t
-  static constexpr uint32_t kTmemO = 256;             // O_t at columns 256 + DH t
+  static constexpr uint32_t kTmemO = 256;             // O_t at columns 256 + kDP t
   static_assert(kBytes <= 232448, "shared memory");
+  static_assert(kTmemO + 2 * kDP <= 512, "tensor memory");
 };
 
 template <int DH>
@@ -615,22 +633,25 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
 
   if (warp == 0) {
     if (lane == 0) {
-      mbar_arrive_expect_tx(q_full, 2 * L::kAtoms * kAtom);
+      const int col0 = h * a.head_stride;
+      // one 128-row operand tile: its 64-column atoms, then (d_h 72) its 16-column atom
+      auto load_tile = [&](uint8_t* dst, const CUtensorMap* m64, const CUtensorMap* m16, uint64_t* bar,
+                           int row) {
+        for (int at = 0; at < L::kA64; ++at) tma_load_2d(dst + at * kAtom, m64, bar, col0 + at * 64, row);
+        if (L::kPad) tma_load_2d(dst + L::kA64 * kAtom, m16, bar, col0 + 64, row);
+      };
+      mbar_arrive_expect_tx(q_full, 2 * L::kTile);
       for (int t = 0; t < 2; ++t)
-        for (int at = 0; at < L::kAtoms; ++at)
-          tma_load_2d(sm + L::kQ + (t * L::kAtoms + at) * kAtom, &a.tmap_q, q_full, h * DH + at * 64,
-                      b * a.n_q + (2 * qt + t) * kTcBQ);
+        load_tile(sm + L::kQ + t * L::kTile, &a.tmap_q, &a.tmap_q16, q_full, b * a.n_q + (2 * qt + t) * kTcBQ);
       int j = 0;
       for (; j < nt; ++j) {
         const int s = j & 1;
         if (!mbar_wait(&kv_empty[s], ((j >> 1) & 1) ^ 1u, abort_flag, a.status, 21)) break;
         uint8_t* st = sm + L::kKV + s * L::kStage;
-        mbar_arrive_expect_tx(&kv_full[s], 2 * L::kAtoms * kAtom);
+        mbar_arrive_expect_tx(&kv_full[s], 2 * L::kTile);
         const int row = b * a.n_kv + j * kTcBK;
-        for (int at = 0; at < L::kAtoms; ++at) {
-          tma_load_2d(st + at * kAtom, &a.tmap_k, &kv_full[s], h * DH + at * 64, row);
-          tma_load_2d(st + (L::kAtoms + at) * kAtom, &a.tmap_v, &kv_full[s], h * DH + at * 64, row);
-        }
+        load_tile(st, &a.tmap_k, &a.tmap_k16, &kv_full[s], row);
+        load_tile(st + L::kTile, &a.tmap_v, &a.tmap_v16, &kv_full[s], row);
       }
       if (*abort_flag) {
         drain_bar(q_full, 0);
@@ -640,28 +661,39 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc_qk = umma_idesc_f16(kTcBQ, kTcBK);
-      const uint32_t idesc_pv = umma_idesc_f16_bmn(kTcBQ, DH);
+      const uint32_t idesc_pv = umma_idesc_f16_bmn(kTcBQ, 64 * L::kA64);
+      const uint32_t idesc_pv16 = umma_idesc_f16_bmn(kTcBQ, 16);
       bool ok = mbar_wait(q_full, 0, abort_flag, a.status, 22);
       auto issue_qk = [&](int t, int j) {
         const int s = j & 1;
-        const uint32_t qa = smem_u32(sm + L::kQ + t * L::kAtoms * kAtom);
+        const uint32_t qa = smem_u32(sm + L::kQ + t * L::kTile);
         const uint32_t ka = smem_u32(sm + L::kKV + s * L::kStage);
 #pragma unroll
-        for (int ks = 0; ks < DH / 16; ++ks) {
+        for (int ks = 0; ks < 4 * L::kA64; ++ks) {
           const uint32_t off = (ks >> 2) * kAtom + (ks & 3) * 32;
           umma_f16(tmem + L::kTmemS + t * kTcBK, smem_desc_sw128(qa + off), smem_desc_sw128(ka + off),
                    idesc_qk, ks > 0 ? 1u : 0u);
+        }
+        if (L::kPad) {  // head columns 64..79 (Q's 72..79 are zero)
+          const uint32_t off = L::kA64 * kAtom;
+          umma_f16(tmem + L::kTmemS + t * kTcBK, smem_desc_sw32(qa + off), smem_desc_sw32(ka + off),
+                   idesc_qk, 1u);
         }
         umma_commit(&s_full[t]);
       };
       auto issue_pv = [&](int t, int j) {
         const int s = j & 1;
-        const uint32_t va = smem_u32(sm + L::kKV + s * L::kStage + L::kAtoms * kAtom);
+        const uint32_t va = smem_u32(sm + L::kKV + s * L::kStage + L::kTile);
 #pragma unroll
         for (int ks = 0; ks < kTcBK / 16; ++ks) {
           const uint64_t bd = smem_desc_sw128_mn(va + ks * 2048, kAtom, 1024);
-          umma_f16_ts(tmem + L::kTmemO + t * DH, tmem + L::kTmemS + t * kTcBK + 8 * ks, bd, idesc_pv,
-                      (j > 0 || ks > 0) ? 1u : 0u);
+          const uint32_t pa = tmem + L::kTmemS + t * kTcBK + 8 * ks;
+          umma_f16_ts(tmem + L::kTmemO + t * L::kDP, pa, bd, idesc_pv, (j > 0 || ks > 0) ? 1u : 0u);
+          if (L::kPad) {  // O columns 64..79 from the 16-column V atom (8-key-row groups 256 B apart)
+            const uint64_t bd16 = smem_desc_sw32_mn(va + L::kA64 * kAtom + ks * 512, kAtom32, 256);
+            umma_f16_ts(tmem + L::kTmemO + t * L::kDP + 64 * L::kA64, pa, bd16, idesc_pv16,
+                        (j > 0 || ks > 0) ? 1u : 0u);
+          }
         }
         umma_commit(&o_done[t]);
       };
@@ -695,7 +727,7 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
     const int row = q * 32 + lane;
     const uint32_t lane_base = static_cast<uint32_t>(q * 32) << 16;
     const uint32_t s_col = tmem + lane_base + L::kTmemS + t * kTcBK;
-    const uint32_t o_col = tmem + lane_base + L::kTmemO + t * DH;
+    const uint32_t o_col = tmem + lane_base + L::kTmemO + t * L::kDP;
     float m2 = -INFINITY, l = 0.f;
     bool ok = true;
     uint32_t r[kTcBK];
@@ -732,7 +764,7 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
         const float corr = exp2f(m2 - mnew);
         uint32_t o16[16];
 #pragma unroll 1
-        for (int c = 0; c < DH; c += 16) {
+        for (int c = 0; c < L::kDP; c += 16) {
           tmem_ld16(o_col + c, o16);
           tmem_ld_wait16(o16);
 #pragma unroll
@@ -773,7 +805,7 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
       const int qrow = (2 * qt + t) * kTcBQ + row;
       f16* orow = a.o + (static_cast<int64_t>(b) * a.n_q + qrow) * a.ldo + h * DH;
 #pragma unroll
-      for (int c = 0; c < DH; c += 16) {
+      for (int c = 0; c < L::kDP; c += 16) {
         tmem_ld16(o_col + c, r);
         tmem_ld_wait16(r);
         float f[16];
@@ -781,7 +813,7 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
         for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(r[i]) * inv;
         if (qrow < a.n_q) {
           reinterpret_cast<uint4*>(orow + c)[0] = pack_f16x8(f);
-          reinterpret_cast<uint4*>(orow + c)[1] = pack_f16x8(f + 8);
+          if (c + 16 <= DH) reinterpret_cast<uint4*>(orow + c)[1] = pack_f16x8(f + 8);
         }
       }
     }
@@ -812,6 +844,10 @@ cudaError_t launch_pp(const AttnPlan& plan, cudaStream_t s) {
   memcpy(&a.tmap_q, &plan.tmap_q, sizeof(CUtensorMap));
   memcpy(&a.tmap_k, &plan.tmap_kv, sizeof(CUtensorMap));
   memcpy(&a.tmap_v, &plan.tmap_v, sizeof(CUtensorMap));
+  memcpy(&a.tmap_q16, &plan.tmap_q16, sizeof(CUtensorMap));
+  memcpy(&a.tmap_k16, &plan.tmap_k16, sizeof(CUtensorMap));
+  memcpy(&a.tmap_v16, &plan.tmap_v16, sizeof(CUtensorMap));
+  a.head_stride = p.head_stride > 0 ? p.head_stride : DH;
   a.o = p.o;
   a.ldo = p.ldo;
   a.n_q = p.n_q;
@@ -841,6 +877,7 @@ cudaError_t launch_tc(const AttnPlan& plan, cudaStream_t s) {
   memcpy(&a.tmap_q, &plan.tmap_q, sizeof(CUtensorMap));
   memcpy(&a.tmap_k, &plan.tmap_kv, sizeof(CUtensorMap));
   memcpy(&a.tmap_v, &plan.tmap_v, sizeof(CUtensorMap));
+  a.head_stride = p.head_stride > 0 ? p.head_stride : DH;
   a.o = p.o;
   a.ldo = p.ldo;
   a.n_q = p.n_q;
@@ -893,6 +930,15 @@ int attn_check(const AttnParams& p, const char** why) {
     *why = "attention: batch * heads exceeds the grid limit";
     return -2;
   }
+  if (p.head_stride != 0 && (p.head_stride < p.d_head || p.head_stride % 8)) {
+    *why = "attention: head_stride must be >= d_head and a multiple of 8";
+    return -2;
+  }
+  const int hs = p.head_stride > 0 ? p.head_stride : p.d_head;
+  if (p.ldq < (p.n_heads - 1) * hs + p.d_head || p.ldkv < (p.n_heads - 1) * hs + p.d_head) {
+    *why = "attention: ldq / ldkv smaller than the heads' columns";
+    return -2;
+  }
   return 0;
 }
 
@@ -900,16 +946,26 @@ int attn_plan(AttnPlan& plan, const char** why) {
   const AttnParams& p = plan.p;
   int rc = attn_check(p, why);
   if (rc) return rc;
-  const bool tc_dh = p.d_head == 64 || p.d_head == 128;
+  const int hs = p.head_stride > 0 ? p.head_stride : p.d_head;
+  // d_h 72 runs on tcgen05 only from a head-padded layout (>= 80 columns per head, Q's
+  // columns 72..79 zero), with two query tiles per CTA
+  const bool pad72 = p.d_head == 72 && hs >= 80;
+  const bool tc_dh = p.d_head == 64 || p.d_head == 128 || (pad72 && p.impl != 2);
   plan.tc = (p.impl == 0 || p.impl == 2 || p.impl == 3) && tc_dh;
   if (!plan.tc) return 0;
   // two query tiles per CTA (ping-pong) unless one tile per CTA is forced: faster on every
   // measured shape, short and ragged ones included (258 tokens: 37.8 against 55.2 us)
   plan.pp = p.impl == 0 || p.impl == 3;
-  const int cols = p.n_heads * p.d_head;
+  const int cols = (p.n_heads - 1) * hs + (pad72 ? 80 : p.d_head);
   if (!make_tmap_f16(&plan.tmap_q, p.q, p.batch * p.n_q, cols, p.ldq, kTcBQ) ||
       !make_tmap_f16(&plan.tmap_kv, p.k, p.batch * p.n_kv, cols, p.ldkv, kTcBK) ||
       !make_tmap_f16(&plan.tmap_v, p.v, p.batch * p.n_kv, cols, p.ldkv, kTcBK)) {
+    *why = "attention: cuTensorMapEncodeTiled failed";
+    return -5;
+  }
+  if (pad72 && (!make_tmap_f16(&plan.tmap_q16, p.q, p.batch * p.n_q, cols, p.ldq, kTcBQ, 16) ||
+                !make_tmap_f16(&plan.tmap_k16, p.k, p.batch * p.n_kv, cols, p.ldkv, kTcBK, 16) ||
+                !make_tmap_f16(&plan.tmap_v16, p.v, p.batch * p.n_kv, cols, p.ldkv, kTcBK, 16))) {
     *why = "attention: cuTensorMapEncodeTiled failed";
     return -5;
   }
@@ -918,7 +974,8 @@ int attn_plan(AttnPlan& plan, const char** why) {
 
 cudaError_t attn_launch(const AttnPlan& plan, cudaStream_t s) {
   const AttnParams& p = plan.p;
-  if (plan.tc && plan.pp) return p.d_head == 64 ? launch_pp<64>(plan, s) : launch_pp<128>(plan, s);
+  if (plan.tc && plan.pp)
+    return p.d_head == 64 ? launch_pp<64>(plan, s) : (p.d_head == 72 ? launch_pp<72>(plan, s) : launch_pp<128>(plan, s));
   if (plan.tc) return p.d_head == 64 ? launch_tc<64>(plan, s) : launch_tc<128>(plan, s);
   switch (p.d_head) {
     case 64: return launch_dh<64, 64>(p, s);

@@ -314,6 +314,30 @@ __device__ __forceinline__ uint64_t smem_desc_sw64(uint32_t saddr) {
   return d;
 }
 
+// Same for 32-byte rows written with 32-byte swizzling (8-row groups 256 B apart, layout
+// SWIZZLE_32B): one K = 16 slice per 32-byte row.
+__device__ __forceinline__ uint64_t smem_desc_sw32(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(1) << 16;
+  d |= static_cast<uint64_t>(256 >> 4) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(6) << 61;                   // SWIZZLE_32B
+  return d;
+}
+
+// MN-major operand in 32-byte swizzle atoms of 8 K-rows x 16 fp16: `lbo` = bytes between
+// atoms along N, `sbo` = bytes between 8-row groups along K.
+__device__ __forceinline__ uint64_t smem_desc_sw32_mn(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(6) << 61;
+  return d;
+}
+
 // Shared-memory descriptor for an MN-major operand (the N index contiguous) stored as
 // 128-byte swizzle atoms of 8 K-rows x 64 fp16: `lbo` = bytes between atoms along N,
 // `sbo` = bytes between 8-row groups along K.

@@ -92,6 +92,8 @@ __device__ __forceinline__ void epi_store8(const EpiParams& e, void* out, int ro
                                            float* v) {
   switch (e.kind) {
     case SGD_EPI_F16:
+      store8_f16(out, e.ldo, row, e.pad_src ? (col / e.pad_src) * e.pad_dst + col % e.pad_src : col, v);
+      break;
     case SGD_EPI_ROPE:
     case SGD_EPI_GATED:
       store8_f16(out, e.ldo, row, col, v);
@@ -873,10 +875,11 @@ __global__ void gemm_simt_kernel(const SimtArgs a) {
     default:
       break;
   }
+  const int oc = (e.kind == SGD_EPI_F16 && e.pad_src) ? (col / e.pad_src) * e.pad_dst + col % e.pad_src : col;
   if (e.kind == SGD_EPI_F32)
     reinterpret_cast<float*>(out)[static_cast<int64_t>(row) * e.ldo + col] = v;
   else
-    reinterpret_cast<f16*>(out)[static_cast<int64_t>(row) * e.ldo + col] = __float2half_rn(sat_f16(v));
+    reinterpret_cast<f16*>(out)[static_cast<int64_t>(row) * e.ldo + oc] = __float2half_rn(sat_f16(v));
 }
 
 // ----------------------------------------------------------------------------
@@ -904,7 +907,7 @@ EncodeTiledFn get_encode_fn() {
 
 }  // namespace
 
-// fp16 [rows, cols] with row stride ld elements; box = box_cols (64 or 32) columns x
+// fp16 [rows, cols] with row stride ld elements; box = box_cols (64, 32 or 16) columns x
 // box_rows rows, 128- or 64-byte swizzle to match, out-of-range elements read as zero.
 bool make_tmap_f16(CUtensorMap* m, const void* base, int rows, int cols, int ld, int box_rows,
                    int box_cols) {
@@ -916,7 +919,8 @@ bool make_tmap_f16(CUtensorMap* m, const void* base, int rows, int cols, int ld,
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides,
                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                  box_cols == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
+                  box_cols == 64 ? CU_TENSOR_MAP_SWIZZLE_128B
+                                 : (box_cols == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B),
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
@@ -1059,6 +1063,14 @@ int gemm_plan(GemmPlan& p, const char** why) {
         (e.norm == SGD_FNORM_LN && (!e.colsum || !e.colbias)) || e.kind == SGD_EPI_DELTA) {
       *why = "gemm: folded norm needs row statistics (1..64 slots, stat_ld >= M), LN column "
              "vectors, and a non-residual epilogue";
+      return -2;
+    }
+  }
+  if (e.pad_src) {
+    if (e.kind != SGD_EPI_F16 || e.pad_src % 8 || e.pad_dst < e.pad_src || e.pad_dst % 8 ||
+        e.ldo < ((p.N + e.pad_src - 1) / e.pad_src) * e.pad_dst) {
+      *why = "gemm: head padding needs an F16 epilogue, pad_src and pad_dst multiples of 8, and ldo "
+             "covering the padded width";
       return -2;
     }
   }

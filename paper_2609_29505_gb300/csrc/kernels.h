@@ -57,6 +57,9 @@ struct EpiParams {
   f16* h16;
   float* stat_out;
   int stat_out_ld;
+  // SGD_EPI_F16 only: output column c goes to (c / pad_src) pad_dst + c % pad_src (heads of
+  // pad_src columns written pad_dst apart; the gaps are never written).  0 = off.
+  int pad_src, pad_dst;
 };
 
 // Row-statistics buffer: kStatSlots slots of sums of squares, then kStatSlots of sums.
@@ -118,8 +121,10 @@ struct AttnParams {
   f16* o;
   int ldo;
   int batch, n_q, n_kv, n_heads, d_head;
-  int impl;  // 0: tcgen05 with two query tiles per CTA where d_head is 64 or 128, else
-             //    mma.sync; 1: mma.sync; 2: tcgen05, one query tile per CTA; 3: same as 0
+  int impl;  // 0: tcgen05 with two query tiles per CTA where d_head is 64 or 128 (72 from a
+             //    head-padded layout), else mma.sync; 1: mma.sync; 2: tcgen05, one query
+             //    tile per CTA; 3: same as 0
+  int head_stride;  // input (q, k, v) columns between heads; 0 = d_head.  Outputs: d_head.
 };
 // A planned attention launch: parameters plus TMA descriptors for the tcgen05 kernel.
 struct AttnPlan {
@@ -129,6 +134,9 @@ struct AttnPlan {
   CUtensorMap tmap_q;
   CUtensorMap tmap_kv;
   CUtensorMap tmap_v;
+  CUtensorMap tmap_q16;  // d_h 72: 16-column boxes (32-byte swizzle)
+  CUtensorMap tmap_k16;
+  CUtensorMap tmap_v16;
 };
 int attn_check(const AttnParams& p, const char** why);
 int attn_plan(AttnPlan& plan, const char** why);

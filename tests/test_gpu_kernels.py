@@ -476,3 +476,44 @@ def test_gemm_residual_writer_emits_h16_and_row_sums(B, kind, variant):
     s1 = st[64:64 + slots].double().sum(dim=0)
     torch.testing.assert_close(ss, (hv * hv).sum(dim=1), rtol=2e-5, atol=1e-3)
     torch.testing.assert_close(s1, hv.sum(dim=1), rtol=2e-5, atol=1e-2)
+
+
+def _padded_heads(x, H, dh, hs, rng=None):
+    """[rows, H dh] -> [rows, H hs]: head h at columns [h hs, h hs + dh); the gap columns
+    hold zeros (rng None) or random finite values."""
+    rows = x.shape[0]
+    out = np.zeros((rows, H * hs), np.float32) if rng is None else \
+        rng.standard_normal((rows, H * hs)).astype(np.float32) * 3.0
+    for h in range(H):
+        out[:, h * hs:h * hs + dh] = x[:, h * dh:(h + 1) * dh]
+    return out
+
+
+@pytest.mark.parametrize("impl", [0, 3, 1], ids=["tcgen05", "tcgen05_2tile", "mma_sync"])
+@pytest.mark.parametrize("H,nq,nkv,bsz", [(16, 256, 256, 2), (3, 136, 136, 2), (2, 300, 77, 3),
+                                          (4, 640, 640, 1)])
+def test_attention_dh72_head_padded(B, H, nq, nkv, bsz, impl):
+    """d_h = 72 (DiT-XL/2) from a head-padded layout (80 columns per head): the tcgen05
+    kernel reads each head as a 64- and a 16-column block, with zeros after every Q head and
+    arbitrary finite values after K and V heads, against the oracle's attention; O is
+    written with 72 columns per head."""
+    rng = np.random.default_rng(H + nq + nkv)
+    dh, hs = 72, 80
+    d = H * dh
+    q = (rng.standard_normal((bsz * nq, d)) * 1.5).astype(np.float32)
+    k = (rng.standard_normal((bsz * nkv, d)) * 1.5).astype(np.float32)
+    v = rng.standard_normal((bsz * nkv, d)).astype(np.float32)
+    q, k, v = (torch.from_numpy(t).half().float().numpy() for t in (q, k, v))
+    qp = torch.from_numpy(_padded_heads(q, H, dh, hs)).half().cuda()
+    kp = torch.from_numpy(_padded_heads(k, H, dh, hs, rng)).half().cuda()
+    vp = torch.from_numpy(_padded_heads(v, H, dh, hs, rng)).half().cuda()
+    o = torch.full((bsz * nq, d), float("nan"), dtype=torch.float16, device="cuda")
+    B.sgd_kernel_attention_hs(qp, H * hs, kp, vp, H * hs, hs, o, d, bsz, nq, nkv, H, dh, impl=impl)
+    torch.cuda.synchronize()
+    want = odn.attention(q.reshape(bsz, nq, d), k.reshape(bsz, nkv, d), v.reshape(bsz, nkv, d),
+                         H).reshape(bsz * nq, d)
+    got = _f(o)
+    err = np.linalg.norm(got - want) / np.linalg.norm(want)
+    assert err < 1.5e-3, err
+    assert np.max(np.abs(got - want)) < 5e-3 * float(np.abs(want).max())
+    assert B.sgd_kernel_status() == 0

@@ -134,4 +134,5 @@ def test_static_ws_validates_on_host():
     assert L.sgd_kernel_gemm_static_ws(None, 8, None, 8, 8, 8, 8, C.byref(epi), 0, None) == binding.SGD_ERR_ARG
     epi = binding.sgd_epilogue_args(kind=binding.EPI_F16, out=64, ldo=8)
     assert L.sgd_kernel_gemm_static_ws(64, 12, 64, 12, 8, 8, 12, C.byref(epi), 0, None) == binding.SGD_ERR_SHAPE
-    assert L.sgd_kernel_gemm_static_ws(64, 8, 64, 8, 8, 8, 8, C.byref(epi), 11, None) == binding.SGD_ERR_ARG
+    for bad_variant in (2, 4, 13, -1):  # not a variant code
+        assert L.sgd_kernel_gemm_static_ws(64, 8, 64, 8, 8, 8, 8, C.byref(epi), bad_variant, None) == binding.SGD_ERR_ARG
