@@ -19,7 +19,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libsgd.so")
 
-SOURCES = ["gemm.cu", "attention.cu", "elementwise.cu", "api.cu"]
+SOURCES = ["gemm_tc_plain.cu", "gemm_tc_rms.cu", "gemm_tc_ln.cu", "gemm_tc_h16.cu", "gemm.cu",
+           "attention.cu", "elementwise.cu", "api.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fno-strict-aliasing",
          "-Xcompiler", "-fvisibility=hidden",

@@ -27,6 +27,24 @@
 
 using namespace sgd;
 
+namespace sgd {
+
+namespace {
+std::vector<unsigned int* (*)()>& clamp_registry() {
+  static std::vector<unsigned int* (*)()> r;
+  return r;
+}
+}  // namespace
+
+int register_f16_clamp_flag(unsigned int* (*accessor)()) {
+  clamp_registry().push_back(accessor);
+  return 1;
+}
+
+const std::vector<unsigned int* (*)()>& f16_clamp_flags() { return clamp_registry(); }
+
+}  // namespace sgd
+
 namespace {
 
 thread_local std::string g_err;
@@ -1813,9 +1831,8 @@ int sgd_kernel_gemm_stat_slots(int M, int N, int K, const sgd_epilogue_args* ea,
 int sgd_kernel_f16_clamped(int* clamped_host) {
   if (!clamped_host) return fail(SGD_ERR_ARG, "null argument");
   *clamped_host = 0;
-  unsigned int* flags[3] = {f16_clamp_flag_gemm(), f16_clamp_flag_attention(),
-                            f16_clamp_flag_elementwise()};
-  for (unsigned int* p : flags) {
+  for (auto accessor : f16_clamp_flags()) {
+    unsigned int* p = accessor();
     if (!p) return fail(SGD_ERR_CUDA, "fp16 clamp flag unavailable");
     unsigned int v = 0;
     CUDA_TRY(cudaMemcpy(&v, p, sizeof(v), cudaMemcpyDeviceToHost));

@@ -984,6 +984,4 @@ cudaError_t attn_launch(const AttnPlan& plan, cudaStream_t s) {
   }
 }
 
-unsigned int* f16_clamp_flag_attention() { return f16_clamp_flag_here(); }
-
 }  // namespace sgd

@@ -366,6 +366,10 @@ __host__ __device__ constexpr uint32_t umma_idesc_f16_bmn(int M, int N) {
   return umma_idesc_f16(M, N) | (1u << 16);
 }
 
+// Every translation unit registers its clamp flag's accessor at load time; the host reads
+// them all (sgd_kernel_f16_clamped).  Defined in api.cu.
+int register_f16_clamp_flag(unsigned int* (*accessor)());
+
 // Device address of this translation unit's clamp flag on the current device (cached per
 // device; nullptr if it cannot be obtained).
 static inline unsigned int* f16_clamp_flag_here() {
@@ -379,5 +383,7 @@ static inline unsigned int* f16_clamp_flag_here() {
   }
   return ptr[dev];
 }
+
+static const int g_f16_clamp_registered = register_f16_clamp_flag(&f16_clamp_flag_here);
 
 }  // namespace sgd

@@ -756,6 +756,4 @@ cudaError_t sampler_launch(float* z, const float* eps, float alpha, float beta, 
   return cudaGetLastError();
 }
 
-unsigned int* f16_clamp_flag_elementwise() { return f16_clamp_flag_here(); }
-
 }  // namespace sgd

@@ -7,6 +7,8 @@
 #include <cuda_fp16.h>
 #include <stdint.h>
 
+#include <vector>
+
 #include "../../include/sgd.h"
 #include "../../include/sgd_kernels.h"
 
@@ -101,10 +103,8 @@ size_t gemm_ws_floats(const GemmPlan& p);
 // capacity; returns 0, or -1 with `why` set when its address cannot be obtained.
 int gemm_static_scratch(float** ws, size_t* ws_floats, int** tickets, int* n_tickets, const char** why);
 int* device_status_ptr();  // device address of the shared status word
-// Device addresses of the fp16 clamp flags of the kernel translation units (one each).
-unsigned int* f16_clamp_flag_gemm();
-unsigned int* f16_clamp_flag_attention();
-unsigned int* f16_clamp_flag_elementwise();
+// Accessors of the fp16 clamp flags of every kernel translation unit (registered at load).
+const std::vector<unsigned int* (*)()>& f16_clamp_flags();
 int num_sms();
 // 2-D fp16 tensor map: [rows, cols] with row stride ld elements, box 64 x box_rows,
 // 128-byte swizzle (defined in gemm.cu).

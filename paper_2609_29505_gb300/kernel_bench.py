@@ -7,6 +7,7 @@ command that the committed ncu summaries under profiles/ were captured from.
 
     python -m paper_2609_29505_gb300.kernel_bench gemm --M 4096 --N 12288 --K 4096 --epi rope
     python -m paper_2609_29505_gb300.kernel_bench attention --batch 4 --heads 32 --tokens 1024 --dh 128
+    python -m paper_2609_29505_gb300.kernel_bench attention --batch 8 --heads 16 --tokens 256 --dh 72 --head-stride 80
     python -m paper_2609_29505_gb300.kernel_bench frozen --rows 4096 --d 4096 --caches 8
     python -m paper_2609_29505_gb300.kernel_bench norm --rows 4096 --d 4096
 """
@@ -71,12 +72,15 @@ def case_gemm(a):
 
 def case_attention(a):
     B, H, N, dh = a.batch, a.heads, a.tokens, a.dh
-    d = H * dh
-    qkv = torch.randn(B * N, 3 * d, device="cuda").half()
+    hs = a.head_stride or dh  # input columns per head (80: d_h 72 padded for tcgen05)
+    d, w = H * dh, H * hs
+    qkv = torch.randn(B * N, 3 * w, device="cuda").half()
+    if hs > dh:  # the gaps after every head are zero, as the QKV epilogue leaves them
+        qkv.view(B * N, 3 * H, hs)[:, :, dh:] = 0
     o = torch.empty(B * N, d, device="cuda", dtype=torch.float16)
-    q, k, v = qkv[:, :d], qkv[:, d:2 * d], qkv[:, 2 * d:]
-    ms = _time(lambda: binding.sgd_kernel_attention(q, 3 * d, k, v, 3 * d, o, d, B, N, N, H, dh,
-                                                    impl=a.impl), a.iters, a.warmup)
+    q, k, v = qkv[:, :w], qkv[:, w:2 * w], qkv[:, 2 * w:]
+    ms = _time(lambda: binding.sgd_kernel_attention_hs(q, 3 * w, k, v, 3 * w, hs, o, d, B, N, N, H, dh,
+                                                       impl=a.impl), a.iters, a.warmup)
     flops = 4.0 * B * H * N * N * dh
     return dict(case="attention", impl=["tcgen05", "mma_sync", "tcgen05_1tile", "tcgen05_2tile"][a.impl], batch=B, heads=H,
                 tokens=N, dh=dh, ms=ms, tflops=flops / ms / 1e9)
@@ -115,6 +119,8 @@ def main():
     ap.add_argument("--batch", type=int, default=4)
     ap.add_argument("--heads", type=int, default=32)
     ap.add_argument("--dh", type=int, default=128)
+    ap.add_argument("--head-stride", type=int, default=0,
+                    help="attention: input columns per head (0: d_h; 80 runs d_h 72 on tcgen05)")
     ap.add_argument("--impl", type=int, default=0, help="attention: 0 tcgen05 (auto), 1 mma.sync, 2 tcgen05 one query tile per CTA, "
                          "3 tcgen05 two query tiles per CTA")
     ap.add_argument("--rows", type=int, default=4096)

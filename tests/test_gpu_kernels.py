@@ -417,26 +417,42 @@ def test_gemm_folded_norm(B, norm, epi, variant):
     B.sgd_kernel_gemm(A, Wg.cuda(), M, N, K, e, use_simt=variant)
     torch.cuda.synchronize()
     assert B.sgd_kernel_status() == 0
+    def finish(u):
+        if epi == "gated":
+            return odn.silu(u[:, :N]) * u[:, N:]
+        if epi == "gelu":
+            return odn.gelu_erf(u)
+        if epi == "rope":
+            qkv = u.reshape(bsz, n_tok, 3, H, dh)
+            r = qkv.copy()
+            for j in range(2):
+                t = qkv[:, :, j].transpose(0, 2, 1, 3)
+                r[:, :, j] = odn.rope(t, np.arange(n_tok), 10000.0).transpose(0, 2, 1, 3)
+            return r.reshape(M, N)
+        return u
+
+    # (1) the oracle: norm, then the linear map and the epilogue function, unrounded operands
     if norm == "rms":
         xn = odn.rms_norm(x, g.float().numpy(), 1e-6)
     else:
         xn = odn.layer_norm(x, g.float().numpy(), bsh.float().numpy(), 1e-6)
-    u = odn.linear(xn, W.float().numpy())
-    if epi == "gated":
-        want = odn.silu(u[:, :N]) * u[:, N:]
-    elif epi == "gelu":
-        want = odn.gelu_erf(u)
-    elif epi == "rope":
-        qkv = u.reshape(bsz, n_tok, 3, H, dh)
-        want = qkv.copy()
-        for j in range(2):
-            t = qkv[:, :, j].transpose(0, 2, 1, 3)
-            want[:, :, j] = odn.rope(t, np.arange(n_tok), 10000.0).transpose(0, 2, 1, 3)
-        want = want.reshape(M, N)
+    want = finish(odn.linear(xn, W.float().numpy()))
+    got = _f(out).astype(np.float64)
+    err = np.linalg.norm(got - want) / np.linalg.norm(want)
+    assert err < 2e-3, err  # fp16 rounding of x and of W g (2^-11 each) and of the output
+    # (2) element-wise: the same algebra on the operands the kernel multiplies (fp16 x, fp16
+    # W g), so that only accumulation order and the output rounding remain
+    xr = A.double().cpu().numpy()
+    acc = xr @ Wg.double().numpy().T
+    ss, s1 = np.sum(x.astype(np.float64) ** 2, axis=1), np.sum(x.astype(np.float64), axis=1)
+    if norm == "rms":
+        u = acc / np.sqrt(ss / K + 1e-6)[:, None]
     else:
-        want = u
-    # fp16 rounding of x and of W g (2^-11 each) on top of the fp16 output rounding
-    _check_f16(out, want, extra_abs=3e-3 * float(np.sqrt(np.mean(want.astype(np.float64) ** 2))))
+        mean = s1 / K
+        rstd = 1.0 / np.sqrt(ss / K - mean ** 2 + 1e-6)
+        u = rstd[:, None] * (acc - mean[:, None] * colsum[None, :b_rows]) + colbias[None, :b_rows]
+    tight = finish(u.astype(np.float32))
+    _check_f16(out, tight, extra_abs=2e-4 * float(np.sqrt(np.mean(tight.astype(np.float64) ** 2))))
 
 
 @pytest.mark.parametrize("variant", [0, 5, 7, 9, 10], ids=["tcgen05", "epi4", "bn128", "streamk", "bn224"])
