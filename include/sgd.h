@@ -101,6 +101,10 @@ typedef enum {
 /* (Flag bit 4 is not defined; sgd_create rejects it.) */
 /* Use 64-element K-blocks (4 stages, 128-byte swizzle) in the tcgen05 GEMMs. */
 #define SGD_FLAG_GEMM_BK64 8
+/* Launch a step's kernels without programmatic dependent launch (each kernel then starts
+ * only after the previous one has finished; by default its launch and prologue overlap the
+ * previous kernel's tail). */
+#define SGD_FLAG_NO_PDL 16
 
 typedef struct {
   int stem, block, norm, mlp, head;   /* enums above                                   */

@@ -43,6 +43,11 @@ int register_f16_clamp_flag(unsigned int* (*accessor)()) {
 
 const std::vector<unsigned int* (*)()>& f16_clamp_flags() { return clamp_registry(); }
 
+bool& pdl_flag() {
+  thread_local bool on = false;
+  return on;
+}
+
 }  // namespace sgd
 
 namespace {
@@ -150,6 +155,7 @@ struct sgd_ctx {
   int M = 0, U = 0, nbr = 0;
   int attn_impl = 0;  // 1: mma.sync attention everywhere (SGD_FLAG_MMA_SYNC_ATTENTION)
   int head_stride = 0;  // columns per head in qkv: d_head, or 80 for d_head 72 on tcgen05
+  bool pdl = true;      // programmatic dependent launch between a step program's kernels
   int gemm_bk = 64;   // default K-block of the tcgen05 GEMM
   int exec_mode = SGD_EXEC_JAGGED_GRAPH;
   float* h_pad = nullptr;  // padded mode: residual that discarded branch updates land in
@@ -776,7 +782,15 @@ int ensure_sk_ws(sgd_ctx* c) {
   return SGD_OK;
 }
 
-int run_ops(const std::vector<Op>& ops, cudaStream_t s) {
+// Launch a program's ops in order on `s`; with `pdl`, each kernel may begin launching while
+// the one before finishes (programmatic dependent launch; every kernel waits for its
+// predecessor's results before touching global memory).
+int run_ops(const std::vector<Op>& ops, cudaStream_t s, bool pdl) {
+  struct Scope {
+    bool prev;
+    explicit Scope(bool on) : prev(pdl_flag()) { pdl_flag() = on; }
+    ~Scope() { pdl_flag() = prev; }
+  } scope(pdl);
   for (const Op& op : ops) {
     cudaError_t e = op.run(s);
     if (e != cudaSuccess) return fail(SGD_ERR_CUDA, op.name + ": " + cudaGetErrorString(e));
@@ -1080,7 +1094,7 @@ int prepare_step(sgd_ctx* c, const void* in, void* out, float t, const sgd_cond*
     std::vector<Op> ops;
     int rc = ctx_kv_ops(c, cond->ctx, ops);
     if (rc) return rc;
-    if ((rc = ensure_sk_ws(c)) || (rc = run_ops(ops, s))) return rc;
+    if ((rc = ensure_sk_ws(c)) || (rc = run_ops(ops, s, c->pdl))) return rc;
   }
   return SGD_OK;
 }
@@ -1098,7 +1112,7 @@ const char* sgd_last_error(void) { return g_err.c_str(); }
 int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out) {
   if (!desc || !w || !out) return fail(SGD_ERR_ARG, "null argument");
   *out = nullptr;
-  if (desc->flags & ~(SGD_FLAG_SIMT_GEMM | SGD_FLAG_MMA_SYNC_ATTENTION | SGD_FLAG_GEMM_BK64))
+  if (desc->flags & ~(SGD_FLAG_SIMT_GEMM | SGD_FLAG_MMA_SYNC_ATTENTION | SGD_FLAG_GEMM_BK64 | SGD_FLAG_NO_PDL))
     return fail(SGD_ERR_ARG, "unknown flag bits");
   int rc = check_shape(*desc, *w);
   if (rc) return rc;
@@ -1116,6 +1130,7 @@ int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out) 
   }
   c->M = desc->batch * desc->n_tokens;
   c->attn_impl = (desc->flags & SGD_FLAG_MMA_SYNC_ATTENTION) ? 1 : 0;
+  c->pdl = !(desc->flags & SGD_FLAG_NO_PDL);
   // RMSNorm / LayerNorm pre-norms fold into the GEMMs that follow them; the AdaLN
   // modulation (a per-sample scale of the weight's columns) and the SIMT debug GEMM do not
   c->fold = (desc->norm == SGD_NORM_RMS || desc->norm == SGD_NORM_LN) &&
@@ -1154,7 +1169,7 @@ int sgd_compile_schedule(int T, int n_units, const int32_t* lifetimes, const int
 static int capture_program(sgd_ctx* c, std::vector<Op>&& ops, int* gid) {
   cudaGraph_t g = nullptr;
   CUDA_TRY(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeRelaxed));
-  int rc = run_ops(ops, c->cap_stream);
+  int rc = run_ops(ops, c->cap_stream, c->pdl);
   cudaError_t ce = cudaStreamEndCapture(c->cap_stream, &g);
   if (rc) {
     if (g) cudaGraphDestroy(g);
@@ -1367,7 +1382,7 @@ int drift_step(sgd_ctx* c, int step, cudaStream_t s) {
     ++c->graph_steps;
   } else {
     if (it != c->drift_graph_of.end()) {
-      if ((rc = run_ops(c->programs[it->second], s))) return rc;
+      if ((rc = run_ops(c->programs[it->second], s, c->pdl))) return rc;
     } else {
       auto e = c->drift_eager.find(mask);
       if (e == c->drift_eager.end()) {
@@ -1375,7 +1390,7 @@ int drift_step(sgd_ctx* c, int step, cudaStream_t s) {
         if ((rc = build_program(c, mask, mask, ops)) || (rc = ensure_sk_ws(c))) return rc;
         e = c->drift_eager.emplace(mask, std::move(ops)).first;
       }
-      if ((rc = run_ops(e->second, s))) return rc;
+      if ((rc = run_ops(e->second, s, c->pdl))) return rc;
     }
     ++c->eager_steps;
   }
@@ -1399,7 +1414,7 @@ int sgd_step(sgd_ctx* c, const void* in, void* out, float t, const sgd_cond* con
     return SGD_OK;
   }
   if (c->exec_mode == SGD_EXEC_EAGER) {
-    if ((rc = run_ops(c->programs[c->graph_of_step[step]], s))) return rc;  // one launch per op
+    if ((rc = run_ops(c->programs[c->graph_of_step[step]], s, c->pdl))) return rc;  // one launch per op
   } else {
     CUDA_TRY(cudaGraphLaunch(c->execs[c->graph_of_step[step]], s));
   }

@@ -77,6 +77,7 @@ __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnParams p) {
   f16* sK = sQ + kBQ * kPitch;            // [2][kBKV][kPitch]
   f16* sV = sK + 2 * kBKV * kPitch;       // [2][kBKV][kPitch]
 
+  pdl_wait_and_trigger();
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
   const int q0 = blockIdx.x * kBQ;
@@ -360,6 +361,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(const __grid_con
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_wait_and_trigger();  // the prologue above touched only shared memory and TMEM
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
@@ -629,6 +631,7 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_wait_and_trigger();  // the prologue above touched only shared memory and TMEM
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
@@ -856,8 +859,7 @@ cudaError_t launch_pp(const AttnPlan& plan, cudaStream_t s) {
   a.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(DH));
   a.status = device_status_ptr();
   dim3 grid((p.n_q + kPpBQ - 1) / kPpBQ, p.batch * p.n_heads);
-  attn_pp_kernel<DH><<<grid, kPpThreads, L::kBytes, s>>>(a);
-  return cudaGetLastError();
+  return launch_k(attn_pp_kernel<DH>, grid, dim3(kPpThreads), L::kBytes, s, a);
 }
 
 template <int DH>
@@ -886,8 +888,7 @@ cudaError_t launch_tc(const AttnPlan& plan, cudaStream_t s) {
   a.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(DH));
   a.status = device_status_ptr();
   dim3 grid((p.n_q + kTcBQ - 1) / kTcBQ, p.batch * p.n_heads);
-  attn_tc_kernel<DH><<<grid, kTcThreads, L::kBytes, s>>>(a);
-  return cudaGetLastError();
+  return launch_k(attn_tc_kernel<DH>, grid, dim3(kTcThreads), L::kBytes, s, a);
 }
 
 template <int DH, int DP>
@@ -904,8 +905,7 @@ cudaError_t launch_dh(const AttnParams& p, cudaStream_t s) {
     done[dev] = true;
   }
   dim3 grid((p.n_q + kBQ - 1) / kBQ, p.batch * p.n_heads);
-  attn_kernel<DH, DP><<<grid, kWarps * 32, smem, s>>>(p);
-  return cudaGetLastError();
+  return launch_k(attn_kernel<DH, DP>, grid, dim3(kWarps * 32), static_cast<size_t>(smem), s, p);
 }
 
 }  // namespace

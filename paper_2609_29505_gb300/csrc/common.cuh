@@ -112,6 +112,20 @@ __device__ __forceinline__ uint32_t lane_id() {
 }
 
 // ----------------------------------------------------------------------------
+// programmatic dependent launch (PTX griddepcontrol)
+// ----------------------------------------------------------------------------
+
+// Wait until the grids this grid depends on have completed and their memory is visible
+// (returns at once for a grid launched without programmatic serialization), then let the
+// next grid in the stream begin launching (its CTAs run their own prologue and wait here in
+// turn).  Every kernel of a step program calls this after its shared-memory / TMEM-only
+// prologue and before its first global-memory access.
+__device__ __forceinline__ void pdl_wait_and_trigger() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// ----------------------------------------------------------------------------
 // mbarrier
 // ----------------------------------------------------------------------------
 
@@ -385,5 +399,28 @@ static inline unsigned int* f16_clamp_flag_here() {
 }
 
 static const int g_f16_clamp_registered = register_f16_clamp_flag(&f16_clamp_flag_here);
+
+// Host: launches made while pdl_flag() is set (the kernels of a step program, see run_ops in
+// api.cu) carry the programmatic-stream-serialization attribute, so that in a captured graph
+// each kernel's launch and prologue overlap the tail of the one before (programmatic edges).
+bool& pdl_flag();
+
+template <typename... KArgs, typename... Args>
+static inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                                   cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  if (pdl_flag()) {
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+  }
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
 
 }  // namespace sgd

@@ -43,6 +43,7 @@ __device__ __forceinline__ void load_bf16x4(const bf16* p, float* f) {
 
 __global__ void __launch_bounds__(kNormThreads) norm_kernel(const NormParams p) {
   __shared__ float red[kNormThreads / 32];
+  pdl_wait_and_trigger();
   const int row = blockIdx.x;
   const int nv = p.d >> 2;
   const float4* hr = reinterpret_cast<const float4*>(p.h + static_cast<int64_t>(row) * p.d);
@@ -118,6 +119,7 @@ __global__ void __launch_bounds__(kNormThreads) norm_kernel(const NormParams p) 
 // models a 128-thread block per row would leave each thread two vectors of work.
 constexpr int kNormWarpMaxVec = 16;
 __global__ void __launch_bounds__(256) norm_warp_kernel(const NormParams p) {
+  pdl_wait_and_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row = blockIdx.x * (blockDim.x >> 5) + warp;
   if (row >= p.rows) return;
@@ -193,6 +195,7 @@ __device__ __forceinline__ void drift_acc(const float4 x, const float4 y, float&
 
 __global__ void __launch_bounds__(256) drift_kernel(const DriftParams p) {
   __shared__ float red[8];
+  pdl_wait_and_trigger();
   const int64_t nv = p.n >> 2;
   const float4* h4 = reinterpret_cast<const float4*>(p.h);
   float4* s4 = reinterpret_cast<float4*>(p.snap);
@@ -222,6 +225,7 @@ __global__ void __launch_bounds__(256) drift_kernel(const DriftParams p) {
 // One warp per group: lane l sums partials l, l + 32, ... in double, then a fixed xor tree
 // combines the lanes (the order is the same on every run).
 __global__ void drift_reduce_kernel(const float* partials, double* sums) {
+  pdl_wait_and_trigger();
   const float* p = partials + static_cast<size_t>(blockIdx.x) * 2 * kDriftBlocks;
   double dd = 0.0, hh = 0.0;
   for (int b = threadIdx.x; b < kDriftBlocks; b += 32) {
@@ -255,6 +259,7 @@ __global__ void wait_selftest_kernel(int* status, int code) {
 }
 
 __global__ void __launch_bounds__(256) frozen_kernel(const __grid_constant__ FrozenParams p) {
+  pdl_wait_and_trigger();
   const int64_t n8 = p.n >> 3;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n8; i += stride) {
@@ -279,6 +284,7 @@ __global__ void __launch_bounds__(256) frozen_kernel(const __grid_constant__ Fro
 // cache order (the same fp32 arithmetic as frozen_kernel), stores h and fp16(h), and the
 // warp reduces its sums with a fixed xor tree into stat slot ch.
 __global__ void __launch_bounds__(256) frozen_rows_kernel(const __grid_constant__ FrozenParams p) {
+  pdl_wait_and_trigger();
   const int nch = (p.d + kStatChunk - 1) / kStatChunk;
   const int64_t wid = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (wid >= static_cast<int64_t>(p.rows) * nch) return;
@@ -332,6 +338,7 @@ __device__ __forceinline__ float sinusoid_at(double t, int dim, int c) {
 }
 
 __global__ void stem_kernel(const StemParams p) {
+  pdl_wait_and_trigger();
   const int64_t total = static_cast<int64_t>(p.batch) * p.n_tokens * p.d;
   const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (idx >= total) return;
@@ -385,6 +392,7 @@ constexpr int kGemvCols = 4;
 template <int RMAX>
 __global__ void __launch_bounds__(256) gemv_kernel(const GemvParams p) {
   extern __shared__ float xs[];  // [xrows][K]
+  pdl_wait_and_trigger();
   const int xrows = p.x_sinusoid ? 1 : (p.ldx == 0 ? 1 : p.rows);
   for (int r = 0; r < xrows; ++r) {
     for (int k = threadIdx.x; k < p.K; k += blockDim.x) {
@@ -472,6 +480,7 @@ __device__ __forceinline__ float warp_sum(float v) {
 }
 
 __global__ void __launch_bounds__(256) head_small_kernel(const HeadParams p) {
+  pdl_wait_and_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t r = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + warp;
   const int64_t rows = static_cast<int64_t>(p.batch) * p.n_tokens;
@@ -526,6 +535,7 @@ __global__ void __launch_bounds__(256) head_small_kernel(const HeadParams p) {
 }
 
 __global__ void copy_out_kernel(const IoSlot* slot, const float* h, int64_t n4) {
+  pdl_wait_and_trigger();
   float4* o = reinterpret_cast<float4*>(slot->out);
   const float4* s = reinterpret_cast<const float4*>(h);
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -534,6 +544,7 @@ __global__ void copy_out_kernel(const IoSlot* slot, const float* h, int64_t n4) 
 }
 
 __global__ void pack_f16_kernel(f16* dst, int ld_dst, int col0, const float* h, int rows, int d) {
+  pdl_wait_and_trigger();
   const int64_t n4 = static_cast<int64_t>(rows) * d / 4;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
@@ -635,10 +646,9 @@ cudaError_t norm_launch(const NormParams& p, cudaStream_t s) {
   // warp per row up to d = 2048; wider rows (LLaDA's 4096) measured faster with the block
   // per row (4.2 against 2.3 TB/s inside the step)
   if (p.d <= 32 * 4 * kNormWarpMaxVec)
-    norm_warp_kernel<<<(p.rows + 7) / 8, 256, 0, s>>>(p);
+    return launch_k(norm_warp_kernel, dim3((p.rows + 7) / 8), dim3(256), 0, s, p);
   else
-    norm_kernel<<<p.rows, kNormThreads, 0, s>>>(p);
-  return cudaGetLastError();
+    return launch_k(norm_kernel, dim3(p.rows), dim3(kNormThreads), 0, s, p);
 }
 
 cudaError_t wait_selftest_launch(int* status, int code, cudaStream_t s) {
@@ -647,24 +657,20 @@ cudaError_t wait_selftest_launch(int* status, int code, cudaStream_t s) {
 }
 
 cudaError_t drift_launch(const DriftParams& p, cudaStream_t s) {
-  drift_kernel<<<kDriftBlocks, 256, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_k(drift_kernel, dim3(kDriftBlocks), dim3(256), 0, s, p);
 }
 
 cudaError_t drift_reduce_launch(const float* partials, int n_groups, double* sums, cudaStream_t s) {
-  drift_reduce_kernel<<<n_groups, 32, 0, s>>>(partials, sums);
-  return cudaGetLastError();
+  return launch_k(drift_reduce_kernel, dim3(n_groups), dim3(32), 0, s, partials, sums);
 }
 
 cudaError_t frozen_launch(const FrozenParams& p, cudaStream_t s) {
   if (p.h16) {
     if (!p.stat || p.d % 8 || p.rows < 1 || frozen_stat_slots(p.d) > kStatSlots) return cudaErrorInvalidValue;
     const int64_t warps = static_cast<int64_t>(p.rows) * frozen_stat_slots(p.d);
-    frozen_rows_kernel<<<static_cast<unsigned>((warps + 7) / 8), 256, 0, s>>>(p);
-    return cudaGetLastError();
+    return launch_k(frozen_rows_kernel, dim3(static_cast<unsigned>((warps + 7) / 8)), dim3(256), 0, s, p);
   }
-  frozen_kernel<<<grid_for(p.n / 8, 256), 256, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_k(frozen_kernel, dim3(grid_for(p.n / 8, 256)), dim3(256), 0, s, p);
 }
 
 cudaError_t io_set_launch(IoSlot* slot, const IoSlot& v, cudaStream_t s) {
@@ -674,8 +680,7 @@ cudaError_t io_set_launch(IoSlot* slot, const IoSlot& v, cudaStream_t s) {
 
 cudaError_t stem_launch(const StemParams& p, cudaStream_t s) {
   const int64_t total = static_cast<int64_t>(p.batch) * p.n_tokens * p.d;
-  stem_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_k(stem_kernel, dim3(static_cast<unsigned>((total + 255) / 256)), dim3(256), 0, s, p);
 }
 
 template <int RMAX>
@@ -686,8 +691,7 @@ cudaError_t gemv_launch_r(const GemvParams& p, size_t smem, cudaStream_t s) {
     if (e != cudaSuccess) return e;
   }
   const int cols_per_block = 8 * kGemvCols;
-  gemv_kernel<RMAX><<<(p.N + cols_per_block - 1) / cols_per_block, 256, smem, s>>>(p);
-  return cudaGetLastError();
+  return launch_k(gemv_kernel<RMAX>, dim3((p.N + cols_per_block - 1) / cols_per_block), dim3(256), smem, s, p);
 }
 
 cudaError_t gemv_launch(const GemvParams& p, cudaStream_t s) {
@@ -701,20 +705,17 @@ cudaError_t gemv_launch(const GemvParams& p, cudaStream_t s) {
 
 cudaError_t head_small_launch(const HeadParams& p, cudaStream_t s) {
   const int64_t rows = static_cast<int64_t>(p.batch) * p.n_tokens;
-  head_small_kernel<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_k(head_small_kernel, dim3(static_cast<unsigned>((rows + 7) / 8)), dim3(256), 0, s, p);
 }
 
 cudaError_t copy_out_launch(const IoSlot* slot, const float* h, int64_t n, cudaStream_t s) {
-  copy_out_kernel<<<grid_for(n / 4, 256), 256, 0, s>>>(slot, h, n / 4);
-  return cudaGetLastError();
+  return launch_k(copy_out_kernel, dim3(grid_for(n / 4, 256)), dim3(256), 0, s, slot, h, n / 4);
 }
 
 cudaError_t pack_f16_launch(f16* dst, int ld_dst, int col0, const float* h, int rows, int d,
                             cudaStream_t s) {
-  pack_f16_kernel<<<grid_for(static_cast<int64_t>(rows) * d / 4, 256), 256, 0, s>>>(dst, ld_dst,
-                                                                                  col0, h, rows, d);
-  return cudaGetLastError();
+  return launch_k(pack_f16_kernel, dim3(grid_for(static_cast<int64_t>(rows) * d / 4, 256)), dim3(256), 0, s,
+                  dst, ld_dst, col0, h, rows, d);
 }
 
 cudaError_t absmax_bf16_launch(const bf16* w, int64_t n, float* out, cudaStream_t s) {

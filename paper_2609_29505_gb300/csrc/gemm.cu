@@ -60,6 +60,7 @@ __device__ __forceinline__ float dot_f16(const f16* a, const f16* b, int K) {
 }
 
 __global__ void gemm_simt_kernel(const SimtArgs a) {
+  pdl_wait_and_trigger();
   const int col = blockIdx.x * blockDim.x + threadIdx.x;
   const int row = blockIdx.y;
   if (col >= a.N || row >= a.M) return;
@@ -390,8 +391,7 @@ cudaError_t gemm_launch(const GemmPlan& p, cudaStream_t s) {
   if (p.simt) {
     SimtArgs a{p.A, p.lda, p.B, p.ldb, p.M, p.N, p.K, p.epi};
     dim3 grid((p.N + 127) / 128, p.M);
-    gemm_simt_kernel<<<grid, 128, 0, s>>>(a);
-    return cudaGetLastError();
+    return launch_k(gemm_simt_kernel, grid, dim3(128), 0, s, a);
   }
   TcArgs a;
   memcpy(&a.tmap_a, &p.tmap_a, sizeof(CUtensorMap));

@@ -661,6 +661,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_wait_and_trigger();  // the prologue above touched only shared memory and TMEM
   const uint32_t tmem_base = *tmem_slot;
   const int num_mu = a.num_m;
   const int num_tiles = num_mu * a.num_n;
@@ -839,8 +840,7 @@ cudaError_t launch_tc(const GemmPlan& p, const TcArgs& a, cudaStream_t s) {
     if (err != cudaSuccess) return err;
     attr_done[dev] = true;
   }
-  gemm_tc_kernel<BK, BN, EPIW, FEAT><<<p.grid, kThreads, kSmemBytes, s>>>(a);
-  return cudaGetLastError();
+  return launch_k(gemm_tc_kernel<BK, BN, EPIW, FEAT>, dim3(p.grid), dim3(kThreads), kSmemBytes, s, a);
 }
 
 

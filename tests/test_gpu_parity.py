@@ -323,3 +323,29 @@ def test_long_context_4096_tokens(B):
         assert rel(out.float().cpu().numpy(), ref["outputs"][s - 1]) <= STEP_TOL
     m.check_device()
     m.close()
+
+
+@pytest.mark.parametrize("name", ["dit_small", "llada_small", "uvit_small", "sdxl_small"])
+def test_programmatic_dependent_launch_is_bit_identical(B, name):
+    """Step programs launched with programmatic dependent launch (each kernel's launch and
+    prologue overlapping its predecessor's tail, in graphs and eagerly) give the same bits as
+    fully serialised launches (SGD_FLAG_NO_PDL)."""
+    c = case(name, 0.5)
+    results = []
+    for flags, mode in ((0, B.EXEC_JAGGED_GRAPH), (B.FLAG_NO_PDL, B.EXEC_JAGGED_GRAPH),
+                        (0, B.EXEC_EAGER)):
+        m = B.Denoiser(c.cfg, c.w_dev, flags=flags)
+        m.set_schedule(c.T, c.sched["lifetimes"], c.sched["groups"])
+        m.set_exec_mode(mode)
+        out = c.out_buffer()
+        res = []
+        for s in range(1, c.T + 1):
+            x = c.ids_at(s).cuda() if c.cfg.stem == "embed" else torch.from_numpy(c.ref["states"][s - 1]).cuda()
+            m.step(x, out, otj.timestep(c.T, s), s, class_ids=c.cls, ctx=c.ctx)
+            res.append(out.cpu().clone())
+        m.check_device()
+        m.close()
+        results.append(res)
+    for other in results[1:]:
+        for a, b in zip(results[0], other):
+            assert torch.equal(a, b)
