@@ -48,6 +48,9 @@ def parse():
     ap.add_argument("--rankings", action="store_true",
                     help="also time one trajectory per static ranking of Table tab:cross-ablation "
                          "and for branch granularity, all at the same budget (adds key 'rankings')")
+    ap.add_argument("--flags", type=int, default=0,
+                    help="sgd_model_desc flags for ablations (e.g. 16: no programmatic dependent "
+                         "launch, 32: norms not folded into the GEMMs)")
     ap.add_argument("--policies", action="store_true",
                     help="also time the static schedule against the activation-drift policy of "
                          "App. B.1 at the same budget (adds key 'policies')")
@@ -234,7 +237,7 @@ def run_native(args):
     K = args.steps if args.steps is not None else T
     W = args.warmup if args.warmup is not None else T
     W = max(W, 3)
-    model = binding.Denoiser(cfg, weights)
+    model = binding.Denoiser(cfg, weights, flags=args.flags)
     t0 = time.time()
     model.set_schedule(T, sched["lifetimes"], sched["groups"])
     setup_t["capture_s"] = round(time.time() - t0, 2)
@@ -421,7 +424,7 @@ def run_native(args):
                    "tokens_per_s": round(value * cfg.batch * cfg.n_tokens, 1),
                    "parallelism": f"replicas{world}" if world > 1 else "single",
                    "l2": "inputs larger than L2 (bf16 weights ~16 GB per step)",
-                   "n_patterns": info["n_patterns"], "n_graphs": info["n_graphs"],
+                   "n_patterns": info["n_patterns"], "n_graphs": info["n_graphs"], "flags": args.flags,
                    "cache_gb": round(info["cache_bytes"] / 2 ** 30, 2), "setup": setup_t},
         "roofline": roofline, "step_roofline": step_roof, "kernels": kernels,
         "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(gpu_launches),

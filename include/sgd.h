@@ -105,6 +105,9 @@ typedef enum {
  * only after the previous one has finished; by default its launch and prologue overlap the
  * previous kernel's tail). */
 #define SGD_FLAG_NO_PDL 16
+/* Keep RMSNorm / LayerNorm pre-norms as separate norm kernels instead of folding them into
+ * the GEMMs that follow them (an ablation switch; results agree within fp16 rounding). */
+#define SGD_FLAG_NO_FOLD 32
 
 typedef struct {
   int stem, block, norm, mlp, head;   /* enums above                                   */

@@ -1112,7 +1112,8 @@ const char* sgd_last_error(void) { return g_err.c_str(); }
 int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out) {
   if (!desc || !w || !out) return fail(SGD_ERR_ARG, "null argument");
   *out = nullptr;
-  if (desc->flags & ~(SGD_FLAG_SIMT_GEMM | SGD_FLAG_MMA_SYNC_ATTENTION | SGD_FLAG_GEMM_BK64 | SGD_FLAG_NO_PDL))
+  if (desc->flags & ~(SGD_FLAG_SIMT_GEMM | SGD_FLAG_MMA_SYNC_ATTENTION | SGD_FLAG_GEMM_BK64 | SGD_FLAG_NO_PDL |
+                      SGD_FLAG_NO_FOLD))
     return fail(SGD_ERR_ARG, "unknown flag bits");
   int rc = check_shape(*desc, *w);
   if (rc) return rc;
@@ -1134,7 +1135,7 @@ int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out) 
   // RMSNorm / LayerNorm pre-norms fold into the GEMMs that follow them; the AdaLN
   // modulation (a per-sample scale of the weight's columns) and the SIMT debug GEMM do not
   c->fold = (desc->norm == SGD_NORM_RMS || desc->norm == SGD_NORM_LN) &&
-            !(desc->flags & SGD_FLAG_SIMT_GEMM);
+            !(desc->flags & (SGD_FLAG_SIMT_GEMM | SGD_FLAG_NO_FOLD));
   c->nbr = desc->block == SGD_BLOCK_XATTN ? 3 : 2;
   c->U = desc->n_blocks * c->nbr;
   if ((rc = ensure_alloc(c)) || (rc = prep_weights(c))) {

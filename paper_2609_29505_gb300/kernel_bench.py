@@ -65,9 +65,24 @@ def case_gemm(a):
         epi.d_head, epi.rope_cols = 128, 2 * N // 3
         keep += [cos, sin]
     epi.act = 0
+    if a.norm:  # pre-norm folded in: row statistics as a residual writer with 38 slots leaves them
+        slots = 38
+        rstat = torch.rand(128, M, device="cuda", generator=g) * (K / slots)
+        colsum = torch.randn(rows_b + 512, device="cuda", generator=g)
+        colbias = torch.randn(rows_b + 512, device="cuda", generator=g)
+        epi.norm = 1 if a.norm == "rms" else 2
+        epi.rstat, epi.stat_slots, epi.stat_ld, epi.norm_eps = rstat.data_ptr(), slots, M, 1e-6
+        epi.colsum, epi.colbias = colsum.data_ptr(), colbias.data_ptr()
+        keep += [rstat, colsum, colbias]
+    if a.h16:  # residual writer: fp16 copy of h and row sums
+        h16 = torch.empty(M, N, device="cuda", dtype=torch.float16)
+        st = torch.empty(128, M, device="cuda")
+        epi.h16, epi.stat_out, epi.stat_out_ld = h16.data_ptr(), st.data_ptr(), M
+        keep += [h16, st]
     ms = _time(lambda: binding.sgd_kernel_gemm(A, B, M, N, K, epi, use_simt=a.simt), a.iters, a.warmup)
     flops = 2.0 * M * rows_b * K
-    return dict(case="gemm", M=M, N=N, K=K, epi=a.epi, ms=ms, tflops=flops / ms / 1e9)
+    return dict(case="gemm", M=M, N=N, K=K, epi=a.epi, norm=a.norm, h16=a.h16, ms=ms,
+                tflops=flops / ms / 1e9)
 
 
 def case_attention(a):
@@ -111,6 +126,10 @@ def main():
     ap.add_argument("--K", type=int, default=4096)
     ap.add_argument("--epi", default="f16", choices=list(EPI))
     ap.add_argument("--store-cache", action="store_true")
+    ap.add_argument("--norm", default="", choices=["", "rms", "ln"],
+                    help="gemm: pre-norm folded into the GEMM (row statistics in 38 slots)")
+    ap.add_argument("--h16", action="store_true",
+                    help="gemm (delta / f32): also write the fp16 copy of h and the row sums")
     ap.add_argument("--simt", type=int, default=0,
                     help="sgd_kernel_gemm variant: 0 tcgen05 (auto), 1 SIMT, 3 BK 32, "
                          "5 4 epilogue warps, 6 8 warps, 7 128-column tiles, 8 no stream-K, "
