@@ -290,6 +290,10 @@ int gemm_plan(GemmPlan& p, const char** why) {
       return -2;
     }
   }
+  if (e.norm == SGD_FNORM_LN && e.kind == SGD_EPI_ROPE) {
+    *why = "gemm: a folded LayerNorm has no RoPE epilogue (RoPE models use RMSNorm)";
+    return -2;
+  }
   if (e.norm != SGD_FNORM_NONE && e.h16) {
     *why = "gemm: a folded-norm GEMM cannot also write the residual stream";
     return -2;
@@ -303,9 +307,9 @@ int gemm_plan(GemmPlan& p, const char** why) {
     }
   }
   if (e.h16) {
-    if ((e.kind != SGD_EPI_DELTA && e.kind != SGD_EPI_F32) || !e.stat_out || e.stat_out_ld < p.M ||
+    if ((e.kind != SGD_EPI_DELTA && e.kind != SGD_EPI_F32) || e.gate || !e.stat_out || e.stat_out_ld < p.M ||
         !aligned16(e.h16)) {
-      *why = "gemm: the fp16 copy of h needs a DELTA or F32 epilogue and a statistics buffer";
+      *why = "gemm: the fp16 copy of h needs a DELTA (without gate) or F32 epilogue and a statistics buffer";
       return -2;
     }
   }

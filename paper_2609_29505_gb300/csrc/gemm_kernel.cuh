@@ -315,11 +315,14 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
                                               const Src& src, int cb, int ce, int part, int halves) {
   constexpr int kBN = BN;
   constexpr bool kH16 = FEAT == kFeatH16;
+  // compile-time pruning of paths a feature set never takes (gemm_plan enforces it): a
+  // folded-norm GEMM has no residual (DELTA) epilogue, a residual writer is DELTA or F32
+  constexpr bool kNormFeat = FEAT == kFeatRms || FEAT == kFeatLn;  // (and LayerNorm: no RoPE)
   const EpiParams& e = a.epi;
   const bool row_ok = row < a.M;
   const RowNorm rn = row_norm<FEAT>(e, row, row_ok);
   float x[16], y[16];
-  if (a.gated) {
+  if (!kH16 && a.gated) {
     const int n0 = n_blk * (kBN / 2);
     for (int c = cb; c < ce; c += 16) {
       if (n0 + c >= a.N) break;
@@ -336,7 +339,7 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
     return;
   }
   const int n0 = n_blk * kBN;
-  if (e.kind == SGD_EPI_ROPE && kFastRope) {
+  if (!kH16 && FEAT != kFeatLn && e.kind == SGD_EPI_ROPE && kFastRope) {
     // every head of the tile shares the row's position, so each 16-wide chunk of the cos /
     // sin tables is read once for all of them and the next chunk is fetched ahead (the
     // 4-epilogue-warp kernel, which has the registers for it)
@@ -392,7 +395,7 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
     }
     return;
   }
-  if (e.kind == SGD_EPI_ROPE && !kFastRope) {
+  if (!kH16 && FEAT != kFeatLn && e.kind == SGD_EPI_ROPE && !kFastRope) {
     const int dh = e.d_head, hd = dh >> 1;
     const int pos = row_ok ? row % e.rope_tokens : 0;
     for (int hb = cb; hb < ce; hb += dh) {
@@ -424,11 +427,13 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
     }
     return;
   }
-  if (e.kind == SGD_EPI_DELTA) {
+  if (!kNormFeat && e.kind == SGD_EPI_DELTA) {
     // residual update: the chunk's h (and gate) loads are issued together, ahead of the
     // accumulator reads, instead of one dependent load per 8 columns
+    // the residual writer (kFeatH16) serves folded-norm models, which have no AdaLN gate
     const float* grow =
-        e.gate ? e.gate + static_cast<int64_t>(row_ok ? row / e.rows_per_batch : 0) * e.ld_gate + n0 : nullptr;
+        (!kH16 && e.gate) ? e.gate + static_cast<int64_t>(row_ok ? row / e.rows_per_batch : 0) * e.ld_gate + n0
+                          : nullptr;
     float* hrow = e.h + static_cast<int64_t>(row) * e.ldh + n0;
     float st_ss = 0.f, st_s1 = 0.f;
     for (int c = cb; c < ce; c += 32) {
@@ -441,7 +446,8 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
       for (int q = 0; q < 8; ++q) {
         const int col = min(c + 4 * q, a.N - n0 - 4);
         hv[q] = *reinterpret_cast<const float4*>(hrow + static_cast<int64_t>(hr) * e.ldh + col);
-        gv[q] = grow ? *reinterpret_cast<const float4*>(grow + col) : make_float4(1.f, 1.f, 1.f, 1.f);
+        if constexpr (!kH16)
+          gv[q] = grow ? *reinterpret_cast<const float4*>(grow + col) : make_float4(1.f, 1.f, 1.f, 1.f);
       }
       src.load2(c, c + 16, x, y);
       if (row_ok) {
@@ -449,7 +455,7 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
         for (int g = 0; g < 4; ++g) {
           if (n0 + c + 8 * g >= a.N) continue;
           float* v = g < 2 ? x + 8 * g : y + 8 * (g - 2);  // constant once unrolled
-          if (grow) {
+          if (!kH16 && grow) {
             v[0] *= gv[2 * g].x; v[1] *= gv[2 * g].y; v[2] *= gv[2 * g].z; v[3] *= gv[2 * g].w;
             v[4] *= gv[2 * g + 1].x; v[5] *= gv[2 * g + 1].y; v[6] *= gv[2 * g + 1].z; v[7] *= gv[2 * g + 1].w;
           }
@@ -479,18 +485,20 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
   for (int c = cb; c < ce; c += 32) {
     if (n0 + c >= a.N) break;
     src.load2(c, c + 16, x, y);
-    apply_norm16<FEAT>(e, rn, n0 + c, x);
-    apply_norm16<FEAT>(e, rn, n0 + c + 16, y);
-    if (row_ok) {
+    // the first 16 columns are normalised and stored before the second 16 are touched (the
+    // LayerNorm column vectors of one half at a time)
 #pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        if (n0 + c + 8 * q < a.N) {
-          epi_store8(e, out, row, n0 + c + 8 * q, x + 8 * q);
-          if constexpr (kH16) emit_h8(e, e.ldo, row, n0 + c + 8 * q, x + 8 * q, st_ss, st_s1);
-        }
-        if (n0 + c + 16 + 8 * q < a.N) {
-          epi_store8(e, out, row, n0 + c + 16 + 8 * q, y + 8 * q);
-          if constexpr (kH16) emit_h8(e, e.ldo, row, n0 + c + 16 + 8 * q, y + 8 * q, st_ss, st_s1);
+    for (int half = 0; half < 2; ++half) {
+      float* v = half ? y : x;
+      const int c0 = n0 + c + 16 * half;
+      apply_norm16<FEAT>(e, rn, c0, v);
+      if (row_ok) {
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          if (c0 + 8 * q < a.N) {
+            epi_store8(e, out, row, c0 + 8 * q, v + 8 * q);
+            if constexpr (kH16) emit_h8(e, e.ldo, row, c0 + 8 * q, v + 8 * q, st_ss, st_s1);
+          }
         }
       }
     }

@@ -414,9 +414,15 @@ def test_gemm_folded_norm(B, norm, epi, variant):
         sin = torch.from_numpy(np.sin(pos * freq).astype(np.float32)).cuda()
         e.rope_cos, e.rope_sin = cos.data_ptr(), sin.data_ptr()
         e.rope_tokens, e.d_head, e.rope_cols = n_tok, dh, 2 * K
+    if norm == "ln" and epi == "rope":  # not a model combination (RoPE models use RMSNorm)
+        with pytest.raises(B.SgdError) as err:
+            B.sgd_kernel_gemm(A, Wg.cuda(), M, N, K, e, use_simt=variant)
+        assert err.value.code == B.SGD_ERR_SHAPE
+        return
     B.sgd_kernel_gemm(A, Wg.cuda(), M, N, K, e, use_simt=variant)
     torch.cuda.synchronize()
     assert B.sgd_kernel_status() == 0
+
     def finish(u):
         if epi == "gated":
             return odn.silu(u[:, :N]) * u[:, N:]
