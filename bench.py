@@ -49,7 +49,7 @@ def parse():
                     help="also time one trajectory per static ranking of Table tab:cross-ablation "
                          "and for branch granularity, all at the same budget (adds key 'rankings')")
     ap.add_argument("--flags", type=int, default=0,
-                    help="sgd_model_desc flags for ablations (e.g. 16: no programmatic dependent "
+                    help="sgd_model_desc flags for ablations (e.g. 16: programmatic dependent "
                          "launch, 32: norms not folded into the GEMMs)")
     ap.add_argument("--policies", action="store_true",
                     help="also time the static schedule against the activation-drift policy of "
@@ -330,8 +330,8 @@ def run_native(args):
                 "frac": round(achieved / peaks["bf16_sus"], 4),
                 "peak_source": f"{peaks['source']} bf16 sustained x 1 (fp16 and bf16 share the "
                                "kind::f16 dense rate)", "traffic": gemm_traffic(cfg, T, args.budget),
-                "traffic_unit": "DRAM bytes per launch (ncu launch list in profiles/, averaged over "
-                                "the step's GEMM launches)",
+                "traffic_unit": "DRAM bytes per launch (ncu, one cold launch of each GEMM of the step, "
+                                "averaged with the step's launch mix; profiles/gemm_tcgen05_llada_dram.md)",
                 "algorithmic_bytes_per_launch": round(gemm["bytes"] / gemm["launches"]),
                 "launches_in_timed_steps": gemm["launches"],
                 "measured_over": "the timed positions, one eager op-by-op launch per op with "
@@ -579,23 +579,30 @@ def run_policies(binding, model, cfg, T, xs, out, cls, ctx, stream):
     return rows
 
 
+GEMM_SOURCES = ("gemm_kernel.cuh", "gemm.cu", "common.cuh")
+
+
+def gemm_source_hash():
+    import hashlib
+    h = hashlib.sha256()
+    for f in GEMM_SOURCES:
+        with open(os.path.join(ROOT, "paper_2609_29505_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
 def gemm_traffic(cfg, T, budget):
     """DRAM bytes per GEMM launch (read + write, averaged over the step's GEMM launches) from
-    the committed ncu launch list of this workload, or None when the workload differs or the
-    GEMM sources changed since the counters were taken."""
-    import hashlib
+    the committed ncu summary of this workload's GEMMs, or None when the workload differs or
+    the GEMM sources changed since the counters were taken."""
     import re
-    path = os.path.join(ROOT, "profiles", "launches_llada_b4_n1024_T64_budget50.md")
+    path = os.path.join(ROOT, "profiles", "gemm_tcgen05_llada_dram.md")
     if cfg.name != "llada" or T != 64 or abs(budget - 0.5) > 1e-9 or not os.path.exists(path):
         return None
     m = re.search(r"traffic_bytes_per_launch: (\d+) sources: ([0-9a-f]{16})", open(path).read())
     if not m:
         return None
-    h = hashlib.sha256()
-    for f in ("gemm.cu", "common.cuh"):
-        with open(os.path.join(ROOT, "paper_2609_29505_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
-    return int(m.group(1)) if h.hexdigest()[:16] == m.group(2) else None
+    return int(m.group(1)) if gemm_source_hash() == m.group(2) else None
 
 
 def workload_name(cfg, T, budget):

@@ -40,7 +40,7 @@ HEAD = {"linear": 0, "adaln_linear": 1, "identity": 2, "logits": 3}
 FLAG_SIMT_GEMM = 1
 FLAG_MMA_SYNC_ATTENTION = 2
 FLAG_GEMM_BK64 = 8
-FLAG_NO_PDL = 16
+FLAG_PDL = 16
 FLAG_NO_FOLD = 32
 
 EPI_F16, EPI_F32, EPI_DELTA, EPI_GATED, EPI_GELU, EPI_ROPE = range(6)

@@ -155,7 +155,7 @@ struct sgd_ctx {
   int M = 0, U = 0, nbr = 0;
   int attn_impl = 0;  // 1: mma.sync attention everywhere (SGD_FLAG_MMA_SYNC_ATTENTION)
   int head_stride = 0;  // columns per head in qkv: d_head, or 80 for d_head 72 on tcgen05
-  bool pdl = true;      // programmatic dependent launch between a step program's kernels
+  bool pdl = false;     // programmatic dependent launch between a step program's kernels
   int gemm_bk = 64;   // default K-block of the tcgen05 GEMM
   int exec_mode = SGD_EXEC_JAGGED_GRAPH;
   float* h_pad = nullptr;  // padded mode: residual that discarded branch updates land in
@@ -1112,7 +1112,7 @@ const char* sgd_last_error(void) { return g_err.c_str(); }
 int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out) {
   if (!desc || !w || !out) return fail(SGD_ERR_ARG, "null argument");
   *out = nullptr;
-  if (desc->flags & ~(SGD_FLAG_SIMT_GEMM | SGD_FLAG_MMA_SYNC_ATTENTION | SGD_FLAG_GEMM_BK64 | SGD_FLAG_NO_PDL |
+  if (desc->flags & ~(SGD_FLAG_SIMT_GEMM | SGD_FLAG_MMA_SYNC_ATTENTION | SGD_FLAG_GEMM_BK64 | SGD_FLAG_PDL |
                       SGD_FLAG_NO_FOLD))
     return fail(SGD_ERR_ARG, "unknown flag bits");
   int rc = check_shape(*desc, *w);
@@ -1131,7 +1131,7 @@ int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out) 
   }
   c->M = desc->batch * desc->n_tokens;
   c->attn_impl = (desc->flags & SGD_FLAG_MMA_SYNC_ATTENTION) ? 1 : 0;
-  c->pdl = !(desc->flags & SGD_FLAG_NO_PDL);
+  c->pdl = (desc->flags & SGD_FLAG_PDL) != 0;
   // RMSNorm / LayerNorm pre-norms fold into the GEMMs that follow them; the AdaLN
   // modulation (a per-sample scale of the weight's columns) and the SIMT debug GEMM do not
   c->fold = (desc->norm == SGD_NORM_RMS || desc->norm == SGD_NORM_LN) &&

@@ -246,19 +246,32 @@ struct RowNorm {
   float rstd, mean;
 };
 
+// Sum of `n` slots of a row's partial sums, slot order (the same bits on every run): eight
+// loads are issued together and then added one after another (a zero past the last slot
+// leaves the sum unchanged), instead of one load latency per slot.
+__device__ __forceinline__ float sum_slots(const float* base, int64_t ld, int n) {
+  float s = 0.f;
+  for (int p = 0; p < n; p += 8) {
+    float v[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = (p + i < n) ? __ldcg(base + static_cast<int64_t>(p + i) * ld) : 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) s += v[i];
+  }
+  return s;
+}
+
 template <int FEAT>
 __device__ __forceinline__ RowNorm row_norm(const EpiParams& e, int row, bool row_ok) {
   RowNorm n{1.f, 0.f};
   if constexpr (FEAT == kFeatRms || FEAT == kFeatLn) {
     const int r = row_ok ? row : 0;
-    float ss = 0.f;
-    for (int p = 0; p < e.stat_slots; ++p) ss += e.rstat[static_cast<int64_t>(p) * e.stat_ld + r];
+    const float ss = sum_slots(e.rstat + r, e.stat_ld, e.stat_slots);
     if constexpr (FEAT == kFeatRms) {
       n.rstd = rsqrtf(ss * e.norm_inv_d + e.norm_eps);
     } else {
-      float s1 = 0.f;
-      for (int p = 0; p < e.stat_slots; ++p)
-        s1 += e.rstat[static_cast<int64_t>(kStatSlots + p) * e.stat_ld + r];
+      const float s1 = sum_slots(e.rstat + static_cast<int64_t>(kStatSlots) * e.stat_ld + r, e.stat_ld,
+                                 e.stat_slots);
       const double mean = static_cast<double>(s1) * e.norm_inv_d;
       const double var = fmax(static_cast<double>(ss) * e.norm_inv_d - mean * mean, 0.0);
       n.mean = static_cast<float>(mean);
@@ -266,6 +279,18 @@ __device__ __forceinline__ RowNorm row_norm(const EpiParams& e, int row, bool ro
     }
   }
   return n;
+}
+
+// Residual (DELTA) epilogue: pull this thread's part of the tile's h rows into L2 before
+// waiting for the accumulator, so that the epilogue reads them from L2 (the wait is idle
+// time; for a CTA's last tile no mainloop hides the DRAM latency otherwise).
+__device__ __forceinline__ void prefetch_h_row(const EpiParams& e, int row, int M, int N, int n0, int cb,
+                                               int ce) {
+  if (e.kind != SGD_EPI_DELTA || row >= M) return;
+  const int c1 = min(n0 + ce, N);
+  const float* hr = e.h + static_cast<int64_t>(row) * e.ldh;
+  for (int c = n0 + cb; c < c1; c += 32)  // 128-byte lines
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(hr + c));
 }
 
 // Apply the folded norm to 16 accumulator values whose B rows are brow .. brow + 15
@@ -770,6 +795,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
       const int row = m_blk * kBM + q * 32 + lane;
       const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * kBN;
       if (u >= w.n_sk) {  // data-parallel tile
+        prefetch_h_row(a.epi, row, a.M, a.N, n_blk * kBN, cb, ce);
         if (!warp_wait(&tfull[acc], aph, abort_flag, a.status, 4)) break;
         tc_fence_after();
         epilogue_tile<kBN, kEpiWarps == 4, FEAT>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce, part,

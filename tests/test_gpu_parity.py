@@ -327,13 +327,13 @@ def test_long_context_4096_tokens(B):
 
 @pytest.mark.parametrize("name", ["dit_small", "llada_small", "uvit_small", "sdxl_small"])
 def test_programmatic_dependent_launch_is_bit_identical(B, name):
-    """Step programs launched with programmatic dependent launch (each kernel's launch and
-    prologue overlapping its predecessor's tail, in graphs and eagerly) give the same bits as
-    fully serialised launches (SGD_FLAG_NO_PDL)."""
+    """Step programs launched with programmatic dependent launch (SGD_FLAG_PDL: each kernel's
+    launch and prologue overlapping its predecessor's tail, in graphs and eagerly) give the
+    same bits as fully serialised launches."""
     c = case(name, 0.5)
     results = []
-    for flags, mode in ((0, B.EXEC_JAGGED_GRAPH), (B.FLAG_NO_PDL, B.EXEC_JAGGED_GRAPH),
-                        (0, B.EXEC_EAGER)):
+    for flags, mode in ((0, B.EXEC_JAGGED_GRAPH), (B.FLAG_PDL, B.EXEC_JAGGED_GRAPH),
+                        (B.FLAG_PDL, B.EXEC_EAGER)):
         m = B.Denoiser(c.cfg, c.w_dev, flags=flags)
         m.set_schedule(c.T, c.sched["lifetimes"], c.sched["groups"])
         m.set_exec_mode(mode)
