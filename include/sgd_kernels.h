@@ -86,6 +86,13 @@ typedef struct {
   void* h16;
   float* stat_out;
   int stat_out_ld;
+  /* Optional, with h16: the CTA that completes the last column tile of a 128-row block
+   * (tickets in stat_cnt, one int per row block, zero before the launch and left zero after
+   * it; no CTA waits for another) adds that block's slots in slot order and stores each row's
+   * totals in slot 0 of stat_final (same layout as rstat, 256-byte aligned like any device
+   * allocation), so that a following SGD_FNORM_* GEMM reads stat_slots = 1 of stat_final. */
+  int* stat_cnt;
+  float* stat_final;
 } sgd_epilogue_args;
 
 /* Partial-sum slots a residual writer with these arguments fills (see h16 above). */

@@ -109,7 +109,7 @@ class sgd_epilogue_args(C.Structure):
                 ("norm", C.c_int), ("rstat", C.c_void_p), ("stat_slots", C.c_int),
                 ("stat_ld", C.c_int), ("norm_eps", C.c_float), ("colsum", C.c_void_p),
                 ("colbias", C.c_void_p), ("h16", C.c_void_p), ("stat_out", C.c_void_p),
-                ("stat_out_ld", C.c_int)]
+                ("stat_out_ld", C.c_int), ("stat_cnt", C.c_void_p), ("stat_final", C.c_void_p)]
 
 
 _lib = None

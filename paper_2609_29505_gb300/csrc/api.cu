@@ -165,6 +165,9 @@ struct sgd_ctx {
   bool fold = false;
   f16* h16 = nullptr;
   float* rstat = nullptr;
+  float* rstat_final = nullptr;  // row totals finalised by a writer GEMM (slot 0)
+  int* stat_cnt = nullptr;       // per 128-row block tickets of that finalisation
+  const float* prog_stat = nullptr;  // statistics buffer of the current writer of h
   int prog_slots = 0;
   // stream-K GEMM workspace, shared by every GEMM of this context (they run one after
   // another on one stream); grown when a new plan needs more, the old buffers stay
@@ -317,7 +320,13 @@ int make_gemm_op(sgd_ctx* c, std::vector<Op>& ops, const std::string& name, cons
   if (epi.h16) {  // writer of h: its fp16 copy and row sums (slots of this plan's column tiles)
     const int num_n = (N + plan->bn - 1) / plan->bn;
     out_b += 2.0 * M * N + 16.0 * M * num_n;
-    c->prog_slots = 2 * num_n;
+    if (epi.stat_cnt) {  // finalised by the writer: the next GEMM reads one slot
+      c->prog_stat = epi.stat_final;
+      c->prog_slots = 1;
+    } else {
+      c->prog_stat = epi.stat_out;
+      c->prog_slots = 2 * num_n;
+    }
   }
   if (epi.norm != SGD_FNORM_NONE) out_b += 8.0 * M * epi.stat_slots * (epi.norm == SGD_FNORM_LN ? 2 : 1);
   Op op;
@@ -342,7 +351,7 @@ EpiParams epi_base(int kind) {
 // the statistics of the current writer of h.
 void set_folded_norm(sgd_ctx* c, EpiParams& e, int norm_kind) {
   e.norm = norm_kind == SGD_NORM_RMS ? SGD_FNORM_RMS : SGD_FNORM_LN;
-  e.rstat = c->rstat;
+  e.rstat = c->prog_stat;
   e.stat_slots = c->prog_slots;
   e.stat_ld = c->M;
   e.norm_eps = c->d.eps;
@@ -354,6 +363,8 @@ void set_h_writer(sgd_ctx* c, EpiParams& e) {
   e.h16 = c->h16;
   e.stat_out = c->rstat;
   e.stat_out_ld = c->M;
+  e.stat_cnt = c->stat_cnt;
+  e.stat_final = c->rstat_final;
 }
 
 // h16 and row sums of h as it stands (after the stem): a frozen run of no units.
@@ -372,6 +383,7 @@ void make_hstat_op(sgd_ctx* c, std::vector<Op>& ops) {
   op.bytes = 6.0 * p.n;
   op.run = [p](cudaStream_t s) { return frozen_launch(p, s); };
   ops.push_back(std::move(op));
+  c->prog_stat = c->rstat;
   c->prog_slots = frozen_stat_slots(c->d.d);
 }
 
@@ -437,6 +449,7 @@ void flush_run(sgd_ctx* c, std::vector<Op>& ops, std::vector<const f16*>& run, i
     if (c->fold) {
       p.h16 = c->h16;
       p.stat = c->rstat;
+      c->prog_stat = c->rstat;
       c->prog_slots = frozen_stat_slots(c->d.d);
     }
     while (i < run.size() && p.n_caches < kMaxRun) p.caches[p.n_caches++] = run[i++];
@@ -893,6 +906,11 @@ int ensure_alloc(sgd_ctx* c) {
     if ((rc = c->alloc(&c->h16, M * D, &c->ws_bytes))) return rc;
     if ((rc = c->alloc(&c->rstat, 2 * static_cast<size_t>(kStatSlots) * M, &c->ws_bytes))) return rc;
     CUDA_TRY(cudaMemset(c->rstat, 0, 2 * sizeof(float) * kStatSlots * M));
+    if ((rc = c->alloc(&c->rstat_final, 2 * static_cast<size_t>(kStatSlots) * M, &c->ws_bytes))) return rc;
+    CUDA_TRY(cudaMemset(c->rstat_final, 0, 2 * sizeof(float) * kStatSlots * M));
+    const size_t blocks = (M + 127) / 128;
+    if ((rc = c->alloc(&c->stat_cnt, blocks, &c->ws_bytes))) return rc;
+    CUDA_TRY(cudaMemset(c->stat_cnt, 0, blocks * sizeof(int)));
   }
   if (d.block == SGD_BLOCK_ADALN) {
     if ((rc = c->alloc(&c->t_hidden, D, &c->ws_bytes))) return rc;
@@ -1721,6 +1739,8 @@ int kernel_gemm_plan(const void* A, int lda, const void* B, int ldb, int M, int 
   e.h16 = static_cast<f16*>(ea->h16);
   e.stat_out = ea->stat_out;
   e.stat_out_ld = ea->stat_out_ld;
+  e.stat_cnt = ea->stat_cnt;
+  e.stat_final = ea->stat_final;
   const char* why = "";
   const int rc = gemm_plan(p, &why);
   if (rc) return fail(rc == -5 ? SGD_ERR_CUDA : (rc == -1 ? SGD_ERR_ARG : SGD_ERR_SHAPE), why);

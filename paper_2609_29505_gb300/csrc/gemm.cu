@@ -290,6 +290,10 @@ int gemm_plan(GemmPlan& p, const char** why) {
       return -2;
     }
   }
+  if (e.stat_cnt && (!e.h16 || !e.stat_final || !aligned16(e.stat_final))) {
+    *why = "gemm: row-statistics finalisation needs the residual writer and a final buffer";
+    return -2;
+  }
   if (e.norm == SGD_FNORM_LN && e.kind == SGD_EPI_ROPE) {
     *why = "gemm: a folded LayerNorm has no RoPE epilogue (RoPE models use RMSNorm)";
     return -2;

@@ -62,7 +62,7 @@ struct TileCfg {
   static constexpr int kStages = BN == 224 ? 5 : (192 * 1024) / kStageBytes;
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
   static_assert(kSmemBytes <= 232448, "shared memory");
-  static_assert((2 * kStages + 5) * 8 + 3 * 4 <= 256, "barrier block");
+  static_assert((2 * kStages + 5) * 8 + 4 * 4 <= 256, "barrier block");
 };
 
 template <int BK>
@@ -642,6 +642,35 @@ __device__ __forceinline__ void unit_at(const TcArgs& a, const CtaWork& w, int u
   }
 }
 
+// Residual writer with finalisation (EpiParams::stat_cnt): after the epilogue of a tile, every
+// epilogue thread takes part (also after an expired wait, so that all leave together; returns
+// false then).  The tile's partial sums are published (fence), one thread draws a ticket for
+// the tile's row block, and the CTA holding the last ticket sums the block's slots per row
+// (one thread per row) into stat_final and resets the counter.
+template <int kEpiThreads>
+__device__ __forceinline__ bool finalize_row_stats(const TcArgs& a, bool ok, int m_blk, int row, bool row_owner,
+                                                   volatile int* fin_flag) {
+  const EpiParams& e = a.epi;
+  __threadfence();
+  if (!epi_bar_and(ok, kEpiThreads)) return false;
+  if (threadIdx.x == 64) *fin_flag = atomicAdd(&e.stat_cnt[m_blk], 1) == a.num_n - 1 ? 1 : 0;
+  epi_bar(kEpiThreads);
+  if (*fin_flag != 0) {
+    __threadfence();
+    if (row_owner && row < a.M) {
+      const int slots = 2 * a.num_n;
+      const int64_t ld = e.stat_out_ld;
+      e.stat_final[row] = sum_slots(e.stat_out + row, ld, slots);
+      e.stat_final[static_cast<int64_t>(kStatSlots) * ld + row] =
+          sum_slots(e.stat_out + static_cast<int64_t>(kStatSlots) * ld + row, ld, slots);
+    }
+    if (threadIdx.x == 64) e.stat_cnt[m_blk] = 0;
+  }
+  // fin_flag is rewritten (next tile) only after every epilogue thread has read it: each
+  // reads it before it reaches the next tile's first barrier
+  return true;
+}
+
 // Stream-K (sk_tiles > 0): the K iterations of the first sk_tiles tiles are
 // spread evenly over sk_ctas CTAs (at most kMaxSeg per tile), so that the tiles left over
 // after the last full wave do not leave most SMs idle.  A CTA whose segment does not cover
@@ -668,6 +697,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* last_flag = reinterpret_cast<volatile int*>(tmem_slot + 2);
+  volatile int* fin_flag = reinterpret_cast<volatile int*>(tmem_slot + 3);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -796,6 +826,19 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
       const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * kBN;
       if (u >= w.n_sk) {  // data-parallel tile
         prefetch_h_row(a.epi, row, a.M, a.N, n_blk * kBN, cb, ce);
+        if (FEAT == kFeatH16 && a.epi.stat_cnt) {  // every epilogue thread reaches the barriers
+          const bool ok = warp_wait(&tfull[acc], aph, abort_flag, a.status, 4);
+          if (ok) {
+            tc_fence_after();
+            epilogue_tile<kBN, kEpiWarps == 4, FEAT>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce,
+                                                     part, kEpiWarps == 8 ? 2 : 1);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[acc]);
+          }
+          if (!finalize_row_stats<kEpiThreads>(a, ok, m_blk, row, part == 0, fin_flag)) break;
+          continue;
+        }
         if (!warp_wait(&tfull[acc], aph, abort_flag, a.status, 4)) break;
         tc_fence_after();
         epilogue_tile<kBN, kEpiWarps == 4, FEAT>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce, part,
@@ -816,6 +859,10 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&tempty[acc]);
+        }
+        if (FEAT == kFeatH16 && a.epi.stat_cnt) {
+          if (!finalize_row_stats<kEpiThreads>(a, ok, m_blk, row, part == 0, fin_flag)) break;
+          continue;
         }
         if (!epi_bar_and(ok, kEpiThreads)) break;
         continue;
@@ -847,6 +894,10 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
         epilogue_tile<kBN, kEpiWarps == 4, FEAT>(a, out, row, n_blk, WsSrc<kBN>{slot0, nseg, q * 32 + lane, a.epi.alpha},
                                            cb, ce, part, kEpiWarps == 8 ? 2 : 1);
         if (threadIdx.x == 64) a.sk_cnt[tile] = 0;
+      }
+      // the CTA that finished the tile (last_flag is CTA-uniform) draws its row block's ticket
+      if (FEAT == kFeatH16 && a.epi.stat_cnt && *last_flag != 0) {
+        if (!finalize_row_stats<kEpiThreads>(a, true, m_blk, row, part == 0, fin_flag)) break;
       }
     }
   }

@@ -59,6 +59,13 @@ struct EpiParams {
   f16* h16;
   float* stat_out;
   int stat_out_ld;
+  // Optional finalisation by the writer: the CTA that completes the last column tile of a
+  // 128-row block (ticket from stat_cnt[row block], zero between launches, put back to zero
+  // by that CTA; no CTA waits) adds the block's slots in slot order and stores the row
+  // totals in slot 0 of stat_final (same layout as rstat, ld stat_out_ld): a following
+  // folded-norm GEMM then reads one slot instead of 2 ceil(N / tile width).
+  int* stat_cnt;
+  float* stat_final;
   // SGD_EPI_F16 only: output column c goes to (c / pad_src) pad_dst + c % pad_src (heads of
   // pad_src columns written pad_dst apart; the gaps are never written).  0 = off.
   int pad_src, pad_dst;

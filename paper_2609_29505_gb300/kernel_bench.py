@@ -65,8 +65,8 @@ def case_gemm(a):
         epi.d_head, epi.rope_cols = 128, 2 * N // 3
         keep += [cos, sin]
     epi.act = 0
-    if a.norm:  # pre-norm folded in: row statistics as a residual writer with 38 slots leaves them
-        slots = 38
+    if a.norm:  # pre-norm folded in: row statistics in a.slots slots (1: finalised by the writer)
+        slots = a.slots
         rstat = torch.rand(128, M, device="cuda", generator=g) * (K / slots)
         colsum = torch.randn(rows_b + 512, device="cuda", generator=g)
         colbias = torch.randn(rows_b + 512, device="cuda", generator=g)
@@ -77,8 +77,11 @@ def case_gemm(a):
     if a.h16:  # residual writer: fp16 copy of h and row sums
         h16 = torch.empty(M, N, device="cuda", dtype=torch.float16)
         st = torch.empty(128, M, device="cuda")
+        fin = torch.empty(128, M, device="cuda")
+        cnt = torch.zeros((M + 127) // 128, dtype=torch.int32, device="cuda")
         epi.h16, epi.stat_out, epi.stat_out_ld = h16.data_ptr(), st.data_ptr(), M
-        keep += [h16, st]
+        epi.stat_cnt, epi.stat_final = cnt.data_ptr(), fin.data_ptr()
+        keep += [h16, st, fin, cnt]
     ms = _time(lambda: binding.sgd_kernel_gemm(A, B, M, N, K, epi, use_simt=a.simt), a.iters, a.warmup)
     flops = 2.0 * M * rows_b * K
     return dict(case="gemm", M=M, N=N, K=K, epi=a.epi, norm=a.norm, h16=a.h16, ms=ms,
@@ -128,6 +131,9 @@ def main():
     ap.add_argument("--store-cache", action="store_true")
     ap.add_argument("--norm", default="", choices=["", "rms", "ln"],
                     help="gemm: pre-norm folded into the GEMM (row statistics in 38 slots)")
+    ap.add_argument("--slots", type=int, default=1,
+                    help="gemm --norm: row-statistic slots the GEMM reads (1: finalised by the writer, "
+                         "up to 64: partial sums)")
     ap.add_argument("--h16", action="store_true",
                     help="gemm (delta / f32): also write the fp16 copy of h and the row sums")
     ap.add_argument("--simt", type=int, default=0,

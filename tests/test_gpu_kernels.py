@@ -461,12 +461,15 @@ def test_gemm_folded_norm(B, norm, epi, variant):
     _check_f16(out, tight, extra_abs=2e-4 * float(np.sqrt(np.mean(tight.astype(np.float64) ** 2))))
 
 
+@pytest.mark.parametrize("finalise", [False, True], ids=["slots", "finalised"])
 @pytest.mark.parametrize("variant", [0, 5, 7, 9, 10], ids=["tcgen05", "epi4", "bn128", "streamk", "bn224"])
 @pytest.mark.parametrize("kind", ["delta", "f32"])
-def test_gemm_residual_writer_emits_h16_and_row_sums(B, kind, variant):
+def test_gemm_residual_writer_emits_h16_and_row_sums(B, kind, variant, finalise):
     """A writer of the residual stream also stores fp16(h_new) (bit-exact against torch's
     rounding of the same fp32 values) and, per row, partial sums of h_new^2 and h_new whose
-    slot sums equal the full row sums."""
+    slot sums equal the full row sums.  Finalised: the CTA completing each 128-row block
+    stores the slot-order fp32 sum of its slots (bit-exact against that sum on the host) in
+    slot 0 of the final buffer and leaves the tickets at zero."""
     rng = np.random.default_rng(41 + variant)
     M, N, K = 300, 1032 if variant != 10 else 4096, 512
     if variant == 9:
@@ -476,12 +479,16 @@ def test_gemm_residual_writer_emits_h16_and_row_sums(B, kind, variant):
     h = torch.from_numpy(rng.standard_normal((M, N)).astype(np.float32)).cuda()
     h16 = torch.empty(M, N, dtype=torch.float16, device="cuda")
     st = torch.full((128, M), float("nan"), device="cuda")
+    fin = torch.full((128, M), float("nan"), device="cuda")
+    cnt = torch.zeros((M + 127) // 128, dtype=torch.int32, device="cuda")
     if kind == "delta":
         e = B.sgd_epilogue_args(kind=B.EPI_DELTA, h=h.data_ptr(), ldh=N, h16=h16.data_ptr(),
                                 stat_out=st.data_ptr(), stat_out_ld=M)
     else:
         e = B.sgd_epilogue_args(kind=B.EPI_F32, out=h.data_ptr(), ldo=N, h16=h16.data_ptr(),
                                 stat_out=st.data_ptr(), stat_out_ld=M)
+    if finalise:
+        e.stat_cnt, e.stat_final = cnt.data_ptr(), fin.data_ptr()
     slots = B.sgd_kernel_gemm_stat_slots(M, N, K, e, variant)
     assert 2 <= slots <= 64 and slots % 2 == 0
     h0 = h.clone()
@@ -498,6 +505,17 @@ def test_gemm_residual_writer_emits_h16_and_row_sums(B, kind, variant):
     s1 = st[64:64 + slots].double().sum(dim=0)
     torch.testing.assert_close(ss, (hv * hv).sum(dim=1), rtol=2e-5, atol=1e-3)
     torch.testing.assert_close(s1, hv.sum(dim=1), rtol=2e-5, atol=1e-2)
+    if finalise:
+        slots_h = st[:slots].cpu().numpy()
+        sums_h = st[64:64 + slots].cpu().numpy()
+        want_ss = np.zeros(M, np.float32)
+        want_s1 = np.zeros(M, np.float32)
+        for p in range(slots):  # slot order, fp32
+            want_ss = (want_ss + slots_h[p]).astype(np.float32)
+            want_s1 = (want_s1 + sums_h[p]).astype(np.float32)
+        np.testing.assert_array_equal(fin[0].cpu().numpy(), want_ss)
+        np.testing.assert_array_equal(fin[64].cpu().numpy(), want_s1)
+        assert int(cnt.abs().sum()) == 0
 
 
 def _padded_heads(x, H, dh, hs, rng=None):
