@@ -50,7 +50,7 @@ def parse():
                          "and for branch granularity, all at the same budget (adds key 'rankings')")
     ap.add_argument("--flags", type=int, default=0,
                     help="sgd_model_desc flags for ablations (e.g. 16: programmatic dependent "
-                         "launch, 32: norms not folded into the GEMMs)")
+                         "launch, 32: pre-norms folded into the GEMMs)")
     ap.add_argument("--policies", action="store_true",
                     help="also time the static schedule against the activation-drift policy of "
                          "App. B.1 at the same budget (adds key 'policies')")

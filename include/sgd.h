@@ -106,9 +106,13 @@ typedef enum {
  * previous one has finished).  Measured on GB300 it gains nothing on the mid-size models
  * and loses 1.5% on the LLaDA-8B-shaped step, whose clock falls under the power cap. */
 #define SGD_FLAG_PDL 16
-/* Keep RMSNorm / LayerNorm pre-norms as separate norm kernels instead of folding them into
- * the GEMMs that follow them (an ablation switch; results agree within fp16 rounding). */
-#define SGD_FLAG_NO_FOLD 32
+/* Fold RMSNorm / LayerNorm pre-norms into the GEMMs that follow them (Algorithm 2's
+ * Norm -> projection as one tcgen05 GEMM: the gain folded into the weight, the row
+ * statistics applied in the epilogue, emitted by the previous writer of the residual stream
+ * with an fp16 copy of it) instead of running a norm kernel first.  Off by default: measured
+ * on GB300 it is slower (LLaDA-8B-shaped step -2% under the power cap, U-ViT / SDXL-shaped
+ * -7 to -8%); results agree with the default path within fp16 rounding. */
+#define SGD_FLAG_FOLD_NORM 32
 
 typedef struct {
   int stem, block, norm, mlp, head;   /* enums above                                   */

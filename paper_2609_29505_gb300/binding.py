@@ -41,7 +41,7 @@ FLAG_SIMT_GEMM = 1
 FLAG_MMA_SYNC_ATTENTION = 2
 FLAG_GEMM_BK64 = 8
 FLAG_PDL = 16
-FLAG_NO_FOLD = 32
+FLAG_FOLD_NORM = 32
 
 EPI_F16, EPI_F32, EPI_DELTA, EPI_GATED, EPI_GELU, EPI_ROPE = range(6)
 KERNEL_NAMES = ["gemm_tc", "gemm_simt", "attention", "norm", "frozen_run", "small"]

@@ -1131,7 +1131,7 @@ int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out) 
   if (!desc || !w || !out) return fail(SGD_ERR_ARG, "null argument");
   *out = nullptr;
   if (desc->flags & ~(SGD_FLAG_SIMT_GEMM | SGD_FLAG_MMA_SYNC_ATTENTION | SGD_FLAG_GEMM_BK64 | SGD_FLAG_PDL |
-                      SGD_FLAG_NO_FOLD))
+                      SGD_FLAG_FOLD_NORM))
     return fail(SGD_ERR_ARG, "unknown flag bits");
   int rc = check_shape(*desc, *w);
   if (rc) return rc;
@@ -1150,10 +1150,10 @@ int sgd_create(const sgd_model_desc* desc, const sgd_weights* w, sgd_ctx** out) 
   c->M = desc->batch * desc->n_tokens;
   c->attn_impl = (desc->flags & SGD_FLAG_MMA_SYNC_ATTENTION) ? 1 : 0;
   c->pdl = (desc->flags & SGD_FLAG_PDL) != 0;
-  // RMSNorm / LayerNorm pre-norms fold into the GEMMs that follow them; the AdaLN
+  // RMSNorm / LayerNorm pre-norms fold into the GEMMs that follow them on request; the AdaLN
   // modulation (a per-sample scale of the weight's columns) and the SIMT debug GEMM do not
   c->fold = (desc->norm == SGD_NORM_RMS || desc->norm == SGD_NORM_LN) &&
-            !(desc->flags & (SGD_FLAG_SIMT_GEMM | SGD_FLAG_NO_FOLD));
+            (desc->flags & SGD_FLAG_FOLD_NORM) && !(desc->flags & SGD_FLAG_SIMT_GEMM);
   c->nbr = desc->block == SGD_BLOCK_XATTN ? 3 : 2;
   c->U = desc->n_blocks * c->nbr;
   if ((rc = ensure_alloc(c)) || (rc = prep_weights(c))) {

@@ -151,6 +151,22 @@ def test_full_size_row0(B, name, T, budget):
     model.check_device()
     assert max(errs) <= STEP_TOL, f"per-step rel L2 {['%.2e' % e for e in errs]}"
 
+    if cfg.norm in ("rms", "ln") and budget == 0.5:  # the same with the pre-norms folded in
+        fm = B.Denoiser(cfg, w, flags=B.FLAG_FOLD_NORM)
+        fm.set_schedule(T, S, sched["groups"])
+        ferrs = []
+        for s in range(1, T + 1):
+            if token:
+                x = ids_at(s).to(dev)
+            else:
+                x = inp.z0.clone()
+                x[0] = torch.from_numpy(ref["states"][s - 1][0]).to(dev)
+            fm.step(x, out, otj.timestep(T, s), s, class_ids=cls, ctx=ctx)
+            ferrs.append(rel(out[0].float().cpu().numpy(), ref["outputs"][s - 1][0]))
+        fm.check_device()
+        fm.close()
+        assert max(ferrs) <= STEP_TOL, f"folded norms: per-step rel L2 {['%.2e' % e for e in ferrs]}"
+
     if not token:  # closed loop on the GPU's own states
         z = inp.z0.clone()
         model.reset()

@@ -349,3 +349,45 @@ def test_programmatic_dependent_launch_is_bit_identical(B, name):
     for other in results[1:]:
         for a, b in zip(results[0], other):
             assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("budget", [1.0, 0.5])
+@pytest.mark.parametrize("name", ["tiny", "uvit_small", "sdxl_small", "llada_small"])
+def test_folded_norm_path_against_oracle(B, name, budget):
+    """The pre-norm folded into the GEMMs (SGD_FLAG_FOLD_NORM; RMSNorm and LayerNorm models):
+    bit-exact active sets and per-step relative L2 <= 5e-3 teacher forced, under jagged graphs,
+    eager launches and padded graphs (which give the same bits), and the closed-loop final
+    state within 1e-2."""
+    c = case(name, budget)
+    want_masks = osp.active_sets(c.osched["lifetimes"], c.T)
+    results = {}
+    for mode in (B.EXEC_JAGGED_GRAPH, B.EXEC_EAGER, B.EXEC_PADDED_GRAPH):
+        m = B.Denoiser(c.cfg, c.w_dev, flags=B.FLAG_FOLD_NORM)
+        m.set_schedule(c.T, c.sched["lifetimes"], c.sched["groups"])
+        m.set_exec_mode(mode)
+        out = c.out_buffer()
+        res, errs = [], []
+        for s in range(1, c.T + 1):
+            np.testing.assert_array_equal(m.active_mask(s), want_masks[s - 1])
+            x = c.ids_at(s).cuda() if c.cfg.stem == "embed" else torch.from_numpy(c.ref["states"][s - 1]).cuda()
+            m.step(x, out, otj.timestep(c.T, s), s, class_ids=c.cls, ctx=c.ctx)
+            res.append(out.cpu().clone())
+            errs.append(rel(res[-1].float().numpy(), c.ref["outputs"][s - 1]))
+        m.check_device()
+        m.close()
+        results[mode] = res
+        assert max(errs) <= STEP_TOL, f"mode {mode}: per-step rel L2 {['%.2e' % e for e in errs]}"
+    for mode in (B.EXEC_EAGER, B.EXEC_PADDED_GRAPH):
+        for a, b in zip(results[B.EXEC_JAGGED_GRAPH], results[mode]):
+            assert torch.equal(a, b)
+    if c.cfg.stem != "embed":
+        m = B.Denoiser(c.cfg, c.w_dev, flags=B.FLAG_FOLD_NORM)
+        m.set_schedule(c.T, c.sched["lifetimes"], c.sched["groups"])
+        out = c.out_buffer()
+        z = c.inp.z0.clone().cuda()
+        for s in range(1, c.T + 1):
+            m.step(z, out, otj.timestep(c.T, s), s, class_ids=c.cls, ctx=c.ctx)
+            B.sgd_sampler_update(z, out, 1.0, 1.0 / c.T)
+        torch.cuda.synchronize()
+        m.close()
+        assert rel(z.cpu().numpy(), c.ref["states"][-1]) <= FINAL_TOL
