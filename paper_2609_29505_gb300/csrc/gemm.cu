@@ -366,10 +366,19 @@ int gemm_plan(GemmPlan& p, const char** why) {
   }
   const int units = num_m * num_n;
   p.grid = units < sms ? units : sms;
-  // tile order: groups of 16 row-blocks where there are several groups and several waves
-  // (a 152-tile wave then spans ~16 x 9.5 tiles, about balanced between A and B bytes for
-  // 224- and 256-column tiles); M-fastest otherwise
-  if (p.group_m < 0) p.group_m = (num_m >= 32 && num_n >= 4 && units >= 2 * sms) ? 16 : 0;
+  // tile order.  M-fastest keeps A (the activations) in L2 while B streams through once,
+  // which is the least DRAM traffic whenever A fits in L2 with room to spare (QKV, up, head
+  // and attention-output projections: A = 33.5 MB).  When neither operand fits (the down
+  // projection: 100 MB each), groups of 16 row-blocks (a 152-tile wave spanning ~16 x 9.5
+  // tiles, about balanced between A and B bytes) read less than M-fastest.
+  if (p.group_m < 0) {
+    const double a_bytes = 2.0 * p.M * p.K, b_bytes = 2.0 * b_rows * p.K;
+    constexpr double kL2Resident = 48e6;  // of 129 MB of L2, split between two dies
+    p.group_m = (num_m >= 32 && num_n >= 4 && units >= 2 * sms && a_bytes > kL2Resident &&
+                 b_bytes > kL2Resident)
+                    ? 16
+                    : 0;
+  }
   p.sk_tiles = p.sk_ctas = p.max_seg = 0;
   if (p.sk != 0) {
     const SkSplit k = sk_split(units, num_k, sms, p.sk == 1);
