@@ -370,20 +370,22 @@ def run_native(args):
         n_e2e = len(plan) * T  # whole trajectories: every step of each, in order
         barrier(world)
         _t.cuda.synchronize()
-        t0 = time.perf_counter()
-        for i in range(n_e2e):
-            s = i % T + 1
-            if s == 1:
-                model.reset()
-            model.step_host_async(xs_h[s - 1], outs_h[i % 2], timestep(cfg, s, T), s,
-                                  class_ids_host=cls_h, ctx_host=ctx_h, stream=stream)
-        model.host_wait()
-        _t.cuda.synchronize()
-        e2e_s = max_over_ranks(time.perf_counter() - t0, world)
+        with ClockSampler(dev.index if dev.index is not None else 0) as clk_e2e:
+            t0 = time.perf_counter()
+            for i in range(n_e2e):
+                s = i % T + 1
+                if s == 1:
+                    model.reset()
+                model.step_host_async(xs_h[s - 1], outs_h[i % 2], timestep(cfg, s, T), s,
+                                      class_ids_host=cls_h, ctx_host=ctx_h, stream=stream)
+            model.host_wait()
+            _t.cuda.synchronize()
+            e2e_s = max_over_ranks(time.perf_counter() - t0, world)
         h2d = xs_h[0].numel() * xs_h[0].element_size() + (0 if cls_h is None else cls_h.numel() * 4)
         e2e = {"value": round(n_e2e * world / e2e_s, 3), "unit": "steps/s", "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(outs_h[0].numel() * outs_h[0].element_size()),
                "steps": n_e2e, "over": f"{len(plan)} whole trajectory(ies) of T={T} steps",
+               "clocks": clk_e2e.summary(),
                "api": "sgd_step_host_async + sgd_host_wait (output copy overlaps the next step)"}
 
     sweep = None
