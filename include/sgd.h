@@ -131,7 +131,8 @@ typedef struct {
   int flags;                          /* SGD_FLAG_*                                     */
 } sgd_model_desc;
 
-/* Per-block weights (device, bf16).  Unused entries may be NULL. */
+/* Per-block weights (device, bf16, every pointer 16-byte aligned, else sgd_create returns
+ * SGD_ERR_ARG).  Unused entries may be NULL. */
 typedef struct {
   const void* norm1_w; const void* norm1_b;   /* [d]                                  */
   const void* w_qkv;                          /* [3d, d]: rows Q, then K, then V      */
@@ -146,6 +147,7 @@ typedef struct {
   const void* w_mod;                          /* [6d, d] AdaLN: shift1 scale1 gate1 shift2 scale2 gate2 */
 } sgd_block_weights;
 
+/* Model weights (device, bf16, 16-byte aligned like the per-block ones). */
 typedef struct {
   const sgd_block_weights* blocks;  /* host array of n_blocks entries (copied)     */
   const void* w_stem;               /* [d, d_in]                                   */

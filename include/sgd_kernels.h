@@ -174,6 +174,7 @@ SGD_API int sgd_kernel_attention_hs(const void* q, int ldq, const void* k, const
  * out fp16 [rows, d] = norm(h fp32 [rows, d]); kind = sgd_norm_kind.  g, b: bf16 [d]
  * (NULL allowed for LN_PLAIN).  shift/scale: optional fp32 AdaLN modulation
  * [B, ld_mod]: out = norm(h) * (1 + scale[r / rows_per_batch]) + shift[...].
+ * h 16-byte and out 8-byte aligned (else SGD_ERR_ARG).
  */
 SGD_API int sgd_kernel_norm(const float* h, void* out, int rows, int d, int kind, const void* g,
                     const void* b, const float* shift, const float* scale, int ld_mod,

@@ -431,8 +431,9 @@ void make_gemv_op(std::vector<Op>& ops, const std::string& name, const GemvParam
   Op op;
   op.name = name;
   op.kernel = SGD_KERNEL_SMALL;
-  op.flops = 2.0 * p.rows * p.N * p.K;
-  op.bytes = 2.0 * p.N * p.K + 4.0 * p.rows * (p.N + p.K);
+  const double seg = p.n_seg > 0 ? p.n_seg : 1;
+  op.flops = 2.0 * seg * p.rows * p.N * p.K;
+  op.bytes = seg * (2.0 * p.N * p.K + 4.0 * p.rows * p.N) + 4.0 * p.rows * p.K;
   op.run = [p](cudaStream_t s) { return gemv_launch(p, s); };
   ops.push_back(std::move(op));
 }
@@ -605,23 +606,26 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
     g2.n_classes = d.n_classes;
     g2.out_silu = c->cond_silu;
     make_gemv_op(ops, "cond.t2", g2);
+    // the modulation of every block with an active branch, in one launch (it depends on c
+    // only): per-block launches of a 16 MB weight each left most of the GPU idle
+    GemvParams gm{};
+    gm.ldo = 6 * D;
+    gm.x = c->cond_silu;
+    gm.ldx = D;
+    gm.slot = c->slot;
+    gm.in_silu = 0;
+    gm.N = 6 * D;
+    gm.K = D;
+    gm.rows = d.batch;
     for (int b = 0; b < d.n_blocks; ++b) {
       bool any = false;
       for (int k = 0; k < c->nbr; ++k) any = any || active[b * c->nbr + k];
       if (!any) continue;  // modulation only for active blocks
-      GemvParams gm{};
-      gm.out = c->mod + static_cast<size_t>(b) * d.batch * 6 * D;
-      gm.ldo = 6 * D;
-      gm.x = c->cond_silu;
-      gm.ldx = D;
-      gm.slot = c->slot;
-      gm.in_silu = 0;
-      gm.W = B16(c->blk[b].w_mod);
-      gm.N = 6 * D;
-      gm.K = D;
-      gm.rows = d.batch;
-      make_gemv_op(ops, "b" + std::to_string(b) + ".mod", gm);
+      gm.w_seg[gm.n_seg] = B16(c->blk[b].w_mod);
+      gm.out_seg[gm.n_seg] = c->mod + static_cast<size_t>(b) * d.batch * 6 * D;
+      ++gm.n_seg;
     }
+    if (gm.n_seg > 0) make_gemv_op(ops, "mod", gm);
   }
   std::vector<const f16*> run;
   int run_first = 0;
@@ -869,8 +873,20 @@ int check_shape(const sgd_model_desc& d, const sgd_weights& w) {
       break;
   }
   if (!w.blocks) return fail(SGD_ERR_ARG, "null block weights");
+  // every weight is read with 8- or 16-byte vector loads
+  {
+    const void* top[] = {w.w_stem, w.pos_emb, w.w_t1, w.w_t2, w.class_emb, w.normf_w,
+                         w.normf_b, w.w_modf, w.w_head, w.embed};
+    for (const void* p : top)
+      if (p && !al16(p)) return fail(SGD_ERR_ARG, "misaligned weight (16-byte alignment needed)");
+    for (int i = 0; w.skip_w && i < d.n_skips; ++i)
+      if (w.skip_w[i] && !al16(w.skip_w[i])) return fail(SGD_ERR_ARG, "misaligned skip weight");
+  }
   for (int b = 0; b < d.n_blocks; ++b) {
     const sgd_block_weights& W = w.blocks[b];
+    const void* all[] = {W.norm1_w, W.norm1_b, W.normx_w, W.normx_b, W.wx_q, W.wx_o, W.norm2_w, W.norm2_b};
+    for (const void* p : all)
+      if (p && !al16(p)) return fail(SGD_ERR_ARG, "block " + std::to_string(b) + ": misaligned weight");
     const void* need[] = {W.w_qkv, W.w_o, W.w_1, W.w_2};
     for (const void* p : need)
       if (!p || !al16(p)) return fail(SGD_ERR_ARG, "block " + std::to_string(b) + ": missing or misaligned weight");
@@ -1823,6 +1839,8 @@ int sgd_kernel_norm(const float* h, void* out, int rows, int d, int kind, const 
     return fail(SGD_ERR_ARG, "norm: bad arguments (d must be a multiple of 4, <= 4096)");
   if ((shift == nullptr) != (scale == nullptr) || (shift && rows_per_batch < 1))
     return fail(SGD_ERR_ARG, "norm: shift and scale go together, rows_per_batch >= 1");
+  if (!al16(h) || (reinterpret_cast<uintptr_t>(out) & 7u))
+    return fail(SGD_ERR_ARG, "norm: h must be 16-byte and out 8-byte aligned");
   NormParams p{h, static_cast<f16*>(out), rows, d, kind, B16(g), B16(b), shift, scale, ld_mod,
                rows_per_batch > 0 ? rows_per_batch : 1, eps};
   CUDA_TRY(norm_launch(p, static_cast<cudaStream_t>(stream)));

@@ -607,6 +607,9 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
   const int qt = blockIdx.x, bh = blockIdx.y;
   const int b = bh / a.n_heads, h = bh % a.n_heads;
   const int nt = (a.n_kv + kTcBK - 1) / kTcBK;
+  // the second query tile of the last pair may hold no query (n_q % 256 in (0, 128], e.g. 258
+  // tokens): that CTA then runs tile 0 alone (CTA-uniform)
+  const bool two = (2 * qt + 1) * kTcBQ < a.n_q;
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
@@ -643,8 +646,8 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
         for (int at = 0; at < L::kA64; ++at) tma_load_2d(dst + at * kAtom, m64, bar, col0 + at * 64, row);
         if (L::kPad) tma_load_2d(dst + L::kA64 * kAtom, m16, bar, col0 + 64, row);
       };
-      mbar_arrive_expect_tx(q_full, 2 * L::kTile);
-      for (int t = 0; t < 2; ++t)
+      mbar_arrive_expect_tx(q_full, (two ? 2 : 1) * L::kTile);
+      for (int t = 0; t < (two ? 2 : 1); ++t)
         load_tile(sm + L::kQ + t * L::kTile, &a.tmap_q, &a.tmap_q16, q_full, b * a.n_q + (2 * qt + t) * kTcBQ);
       int j = 0;
       for (; j < nt; ++j) {
@@ -703,7 +706,7 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
       if (ok && (ok = mbar_wait(&kv_full[0], 0, abort_flag, a.status, 23))) {
         tc_fence_after();
         issue_qk(0, 0);
-        issue_qk(1, 0);
+        if (two) issue_qk(1, 0);
       }
       for (int j = 0; j < nt && ok; ++j) {
         const uint32_t ph = j & 1;
@@ -715,11 +718,13 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
           tc_fence_after();
           issue_qk(0, j + 1);
         }
-        if (!(ok = mbar_wait(&p_full[1], ph, abort_flag, a.status, 26))) break;
-        tc_fence_after();
-        issue_pv(1, j);
+        if (two) {
+          if (!(ok = mbar_wait(&p_full[1], ph, abort_flag, a.status, 26))) break;
+          tc_fence_after();
+          issue_pv(1, j);
+        }
         umma_commit(&kv_empty[j & 1]);
-        if (j + 1 < nt) issue_qk(1, j + 1);
+        if (two && j + 1 < nt) issue_qk(1, j + 1);
       }
       umma_commit(drain);
       drain_bar(drain, 0);
@@ -732,9 +737,9 @@ __global__ void __launch_bounds__(kPpThreads, 1) attn_pp_kernel(const __grid_con
     const uint32_t s_col = tmem + lane_base + L::kTmemS + t * kTcBK;
     const uint32_t o_col = tmem + lane_base + L::kTmemO + t * L::kDP;
     float m2 = -INFINITY, l = 0.f;
-    bool ok = true;
+    bool ok = t == 0 || two;  // the warpgroup of an empty second tile has nothing to do
     uint32_t r[kTcBK];
-    for (int j = 0; j < nt; ++j) {
+    for (int j = 0; j < nt && ok; ++j) {
       if (!(ok = warp_wait_bar(&s_full[t], j & 1, abort_flag, a.status, 27))) break;
       tc_fence_after();
       const int kb = j * kTcBK;

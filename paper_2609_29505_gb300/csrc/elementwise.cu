@@ -41,6 +41,65 @@ __device__ __forceinline__ void load_bf16x4(const bf16* p, float* f) {
   f[0] = a.x; f[1] = a.y; f[2] = c.x; f[3] = c.y;
 }
 
+// y = ((x - mean) * rstd) * g + b, then * (1 + scale) + shift (AdaLN), for the 4 columns
+// 4 i .. 4 i + 3 of a row; sc / sh point at the row's sample's modulation (or are null).
+template <class P>  // NormParams or HeadParams (g, b: bf16 [d] or null)
+__device__ __forceinline__ float4 norm_affine4(const P& p, int i, float4 v, float mean, float rstd,
+                                               const float* sc, const float* sh) {
+  float y[4] = {(v.x - mean) * rstd, (v.y - mean) * rstd, (v.z - mean) * rstd, (v.w - mean) * rstd};
+  if (p.g) {
+    float g[4];
+    load_bf16x4(p.g + 4 * i, g);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) y[k] *= g[k];
+  }
+  if (p.b) {
+    float b[4];
+    load_bf16x4(p.b + 4 * i, b);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) y[k] += b[k];
+  }
+  if (sc) {
+    const float4 s4 = *reinterpret_cast<const float4*>(sc + 4 * i);
+    const float4 h4 = *reinterpret_cast<const float4*>(sh + 4 * i);
+    y[0] = y[0] * (1.f + s4.x) + h4.x;
+    y[1] = y[1] * (1.f + s4.y) + h4.y;
+    y[2] = y[2] * (1.f + s4.z) + h4.z;
+    y[3] = y[3] * (1.f + s4.w) + h4.w;
+  }
+  return make_float4(y[0], y[1], y[2], y[3]);
+}
+
+// The same with the AdaLN modulation read as scalars (any alignment of shift / scale).
+__device__ __forceinline__ float4 norm_affine_s(const NormParams& p, int i, float4 v, float mean, float rstd,
+                                                const float* sc, const float* sh) {
+  float y[4] = {(v.x - mean) * rstd, (v.y - mean) * rstd, (v.z - mean) * rstd, (v.w - mean) * rstd};
+  if (p.g) {
+    float g[4];
+    load_bf16x4(p.g + 4 * i, g);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) y[k] *= g[k];
+  }
+  if (p.b) {
+    float b[4];
+    load_bf16x4(p.b + 4 * i, b);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) y[k] += b[k];
+  }
+  if (sc) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) y[k] = y[k] * (1.f + sc[4 * i + k]) + sh[4 * i + k];
+  }
+  return make_float4(y[0], y[1], y[2], y[3]);
+}
+
+__device__ __forceinline__ void store_f16x4(f16* p, float4 v) {
+  uint2 u;
+  u.x = pack_f16x2(v.x, v.y);
+  u.y = pack_f16x2(v.z, v.w);
+  *reinterpret_cast<uint2*>(p) = u;
+}
+
 __global__ void __launch_bounds__(kNormThreads) norm_kernel(const NormParams p) {
   __shared__ float red[kNormThreads / 32];
   pdl_wait_and_trigger();
@@ -84,33 +143,13 @@ __global__ void __launch_bounds__(kNormThreads) norm_kernel(const NormParams p) 
   const float* sh = p.shift ? p.shift + static_cast<int64_t>(row / p.rows_per_batch) * p.ld_mod : nullptr;
   const float* sc = p.scale ? p.scale + static_cast<int64_t>(row / p.rows_per_batch) * p.ld_mod : nullptr;
   f16* orow = p.out + static_cast<int64_t>(row) * p.d;
+  // (the fp16 stores cannot alias the fp32 / bf16 parameter loads, so the compiler issues
+  // those loads ahead of the stores; transforming every vector before the first store
+  // measured slower)
 #pragma unroll
   for (int j = 0; j < kNormMaxVec; ++j) {
     const int i = threadIdx.x + j * kNormThreads;
-    if (i < nv) {
-      float y[4] = {(v[j].x - mean) * rstd, (v[j].y - mean) * rstd, (v[j].z - mean) * rstd,
-                    (v[j].w - mean) * rstd};
-      if (p.g) {
-        float g[4];
-        load_bf16x4(p.g + 4 * i, g);
-#pragma unroll
-        for (int k = 0; k < 4; ++k) y[k] *= g[k];
-      }
-      if (p.b) {
-        float b[4];
-        load_bf16x4(p.b + 4 * i, b);
-#pragma unroll
-        for (int k = 0; k < 4; ++k) y[k] += b[k];
-      }
-      if (sc) {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) y[k] = y[k] * (1.f + sc[4 * i + k]) + sh[4 * i + k];
-      }
-      uint2 u;
-      u.x = pack_f16x2(y[0], y[1]);
-      u.y = pack_f16x2(y[2], y[3]);
-      *reinterpret_cast<uint2*>(orow + 4 * i) = u;
-    }
+    if (i < nv) store_f16x4(orow + 4 * i, norm_affine_s(p, i, v[j], mean, rstd, sc, sh));
   }
 }
 
@@ -155,30 +194,7 @@ __global__ void __launch_bounds__(256) norm_warp_kernel(const NormParams p) {
 #pragma unroll
   for (int j = 0; j < kNormWarpMaxVec; ++j) {
     const int i = lane + 32 * j;
-    if (i < nv) {
-      float y[4] = {(v[j].x - mean) * rstd, (v[j].y - mean) * rstd, (v[j].z - mean) * rstd,
-                    (v[j].w - mean) * rstd};
-      if (p.g) {
-        float g[4];
-        load_bf16x4(p.g + 4 * i, g);
-#pragma unroll
-        for (int k = 0; k < 4; ++k) y[k] *= g[k];
-      }
-      if (p.b) {
-        float b[4];
-        load_bf16x4(p.b + 4 * i, b);
-#pragma unroll
-        for (int k = 0; k < 4; ++k) y[k] += b[k];
-      }
-      if (sc) {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) y[k] = y[k] * (1.f + sc[4 * i + k]) + sh[4 * i + k];
-      }
-      uint2 u;
-      u.x = pack_f16x2(y[0], y[1]);
-      u.y = pack_f16x2(y[2], y[3]);
-      *reinterpret_cast<uint2*>(orow + 4 * i) = u;
-    }
+    if (i < nv) store_f16x4(orow + 4 * i, norm_affine_s(p, i, v[j], mean, rstd, sc, sh));
   }
 }
 
@@ -384,6 +400,54 @@ __global__ void stem_kernel(const StemParams p) {
   p.h[idx] = v;
 }
 
+// The patch stems with one thread per (token row, 4 channels): the row's d_in patch values
+// and the 4 channels' weight rows are read as 16-byte vectors (d_in % 8 == 0, d % 4 == 0),
+// each channel's dot product is summed in k order exactly as in stem_kernel, and the 4
+// results go out as one float4.
+__global__ void stem_patch_kernel(const StemParams p) {
+  pdl_wait_and_trigger();
+  const int d4 = p.d >> 2;
+  const int64_t total = static_cast<int64_t>(p.batch) * p.n_tokens * d4;
+  const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (idx >= total) return;
+  const int c0 = static_cast<int>(idx % d4) * 4;
+  const int64_t r = idx / d4;
+  const int n = static_cast<int>(r % p.n_tokens);
+  const int b = static_cast<int>(r / p.n_tokens);
+  const IoSlot* s = p.slot;
+  float v[4];
+  const int np = n - p.n_prefix;
+  if (np < 0) {
+    const int cls = min(max(s->class_ids[b], 0), p.n_classes - 1);
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      v[q] = (n == 0) ? sinusoid_at(s->t, p.d, c0 + q)
+                      : __bfloat162float(p.class_emb[static_cast<int64_t>(cls) * p.d + c0 + q]);
+  } else {
+    const float4* z = reinterpret_cast<const float4*>(
+        reinterpret_cast<const float*>(s->state) + (static_cast<int64_t>(b) * (p.n_tokens - p.n_prefix) + np) * p.d_in);
+    const uint4* w = reinterpret_cast<const uint4*>(p.w_stem + static_cast<int64_t>(c0) * p.d_in);
+    const int w_ld = p.d_in >> 3;  // uint4 per weight row
+#pragma unroll
+    for (int q = 0; q < 4; ++q) v[q] = 0.f;
+    for (int k8 = 0; k8 < w_ld; ++k8) {
+      const float4 za = __ldg(z + 2 * k8), zb = __ldg(z + 2 * k8 + 1);
+      const float zf[8] = {za.x, za.y, za.z, za.w, zb.x, zb.y, zb.z, zb.w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float wf[8];
+        unpack_bf16x8(__ldg(w + q * w_ld + k8), wf);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[q] = fmaf(zf[e], wf[e], v[q]);
+      }
+    }
+  }
+  const uint2 pu = __ldg(reinterpret_cast<const uint2*>(p.pos + static_cast<int64_t>(n) * p.d + c0));
+  const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&pu);
+  const float2 p01 = __bfloat1622float2(pb[0]), p23 = __bfloat1622float2(pb[1]);
+  reinterpret_cast<float4*>(p.h)[idx] = make_float4(v[0] + p01.x, v[1] + p01.y, v[2] + p23.x, v[3] + p23.y);
+}
+
 // out[r, j] = sum_k act(x[r, k]) W[j, k] for R <= RMAX rows (conditioning and AdaLN
 // modulation: a few rows against a large weight, bound by reading W once).  Each warp owns
 // 4 consecutive columns; a lane streams 16-byte chunks of the 4 weight rows and reuses
@@ -394,17 +458,51 @@ __global__ void __launch_bounds__(256) gemv_kernel(const GemvParams p) {
   extern __shared__ float xs[];  // [xrows][K]
   pdl_wait_and_trigger();
   const int xrows = p.x_sinusoid ? 1 : (p.ldx == 0 ? 1 : p.rows);
-  for (int r = 0; r < xrows; ++r) {
+  if (p.x_sinusoid) {
     for (int k = threadIdx.x; k < p.K; k += blockDim.x) {
-      float x = p.x_sinusoid ? sinusoid_at(p.slot->t, p.K, k) : p.x[static_cast<int64_t>(r) * p.ldx + k];
+      float x = sinusoid_at(p.slot->t, p.K, k);
       if (p.in_silu) x = silu_f(x);
-      xs[r * p.K + k] = x;
+      xs[k] = x;
+    }
+  } else {
+    // float4 loads (K % 8 == 0, rows 16-byte aligned) in batches of 8 per thread, every load
+    // of a batch issued before its first shared-memory store: x is a generic pointer that
+    // the compiler cannot tell apart from xs, so a store in between would make each load
+    // wait for the previous element's round trip
+    const int k4 = p.K >> 2, n4 = xrows * k4;
+    constexpr int kBatch = 8;
+    for (int i0 = threadIdx.x; i0 < n4; i0 += kBatch * blockDim.x) {
+      float4 v[kBatch];
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const int i = i0 + j * blockDim.x;
+        if (i < n4) {
+          const int r = i / k4, k = (i - r * k4) << 2;
+          v[j] = __ldg(reinterpret_cast<const float4*>(p.x + static_cast<int64_t>(r) * p.ldx + k));
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const int i = i0 + j * blockDim.x;
+        if (i < n4) {
+          float4 x = v[j];
+          if (p.in_silu) {
+            x.x = silu_f(x.x);
+            x.y = silu_f(x.y);
+            x.z = silu_f(x.z);
+            x.w = silu_f(x.w);
+          }
+          *reinterpret_cast<float4*>(xs + i * 4) = x;  // = xs[r * K + k]
+        }
+      }
     }
   }
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int j0 = (blockIdx.x * (blockDim.x >> 5) + warp) * kGemvCols;
   if (j0 >= p.N) return;
+  const bf16* W = p.n_seg ? p.w_seg[blockIdx.y] : p.W;
+  float* out = p.n_seg ? p.out_seg[blockIdx.y] : p.out;
   float acc[kGemvCols][RMAX];
 #pragma unroll
   for (int c = 0; c < kGemvCols; ++c)
@@ -417,7 +515,7 @@ __global__ void __launch_bounds__(256) gemv_kernel(const GemvParams p) {
 #pragma unroll
     for (int c = 0; c < kGemvCols; ++c) {
       if (j0 + c < p.N)
-        unpack_bf16x8(*reinterpret_cast<const uint4*>(p.W + static_cast<int64_t>(j0 + c) * p.K + k), w[c]);
+        unpack_bf16x8(*reinterpret_cast<const uint4*>(W + static_cast<int64_t>(j0 + c) * p.K + k), w[c]);
       else
 #pragma unroll
         for (int q = 0; q < 8; ++q) w[c][q] = 0.f;
@@ -464,21 +562,25 @@ __global__ void __launch_bounds__(256) gemv_kernel(const GemvParams p) {
         v += __bfloat162float(p.add_class[static_cast<int64_t>(cls) * p.N + j]);
       }
       if (p.add_vec) v += p.add_vec[j];
-      p.out[static_cast<int64_t>(r) * p.ldo + j] = v;
+      out[static_cast<int64_t>(r) * p.ldo + j] = v;
       if (p.out_silu) p.out_silu[static_cast<int64_t>(r) * p.ldo + j] = silu_f(v);
     }
   }
 }
 
-// One warp per row: the row's mean and rstd from the fp32 residual stream (two passes, as the
-// norm kernels), then every output channel's dot product with the normalised row formed on
-// the fly (fp32; W rows re-read from L1).
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
 }
 
+// One warp per row: the fp32 row is read once into registers (lane l holds columns 4 (l + 32 j)
+// .. + 3), its mean and rstd are reduced across the warp, the row is normalised (and AdaLN
+// modulated) in place, and then every output channel's dot product with it is formed from
+// the channel's bf16 weight row (read through the read-only cache: out_channels x K x 2
+// bytes, shared by all rows) and reduced across the warp; lane c keeps channel c (and
+// c + 32), and the row's outputs are stored together at the end.
+template <int MAXV>  // float4 per lane: K <= 128 MAXV
 __global__ void __launch_bounds__(256) head_small_kernel(const HeadParams p) {
   pdl_wait_and_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -490,48 +592,61 @@ __global__ void __launch_bounds__(256) head_small_kernel(const HeadParams p) {
   float* out = reinterpret_cast<float*>(p.slot->out) +
                (static_cast<int64_t>(b) * (p.n_tokens - p.n_prefix) + (n - p.n_prefix)) *
                    p.out_channels;
-  const float* x = p.h + r * p.ldx;
-  float mean = 0.f;
-  if (p.norm_kind != SGD_NORM_RMS) {
-    float s1 = 0.f;
-    for (int k = lane * 4; k < p.K; k += 128) {
-      const float4 v = *reinterpret_cast<const float4*>(x + k);
-      s1 += (v.x + v.y) + (v.z + v.w);
+  const float4* x = reinterpret_cast<const float4*>(p.h + r * p.ldx);
+  const int nv = p.K >> 2;
+  float4 v[MAXV];
+  float s1 = 0.f;
+#pragma unroll
+  for (int j = 0; j < MAXV; ++j) {
+    const int i = lane + 32 * j;
+    if (i < nv) {
+      v[j] = __ldg(x + i);
+      s1 += (v[j].x + v[j].y) + (v[j].z + v[j].w);
     }
-    mean = warp_sum(s1) / p.K;
   }
+  const float mean = p.norm_kind != SGD_NORM_RMS ? warp_sum(s1) / p.K : 0.f;
   float sq = 0.f;
-  for (int k = lane * 4; k < p.K; k += 128) {
-    const float4 v = *reinterpret_cast<const float4*>(x + k);
-    const float a0 = v.x - mean, a1 = v.y - mean, a2 = v.z - mean, a3 = v.w - mean;
-    sq += (a0 * a0 + a1 * a1) + (a2 * a2 + a3 * a3);
+#pragma unroll
+  for (int j = 0; j < MAXV; ++j) {
+    const int i = lane + 32 * j;
+    if (i < nv) {
+      const float a0 = v[j].x - mean, a1 = v[j].y - mean, a2 = v[j].z - mean, a3 = v[j].w - mean;
+      sq += (a0 * a0 + a1 * a1) + (a2 * a2 + a3 * a3);
+    }
   }
   const float rstd = rsqrtf(warp_sum(sq) / p.K + p.eps);
   const float* sh = p.shift ? p.shift + static_cast<int64_t>(b) * p.ld_mod : nullptr;
   const float* sc = p.scale ? p.scale + static_cast<int64_t>(b) * p.ld_mod : nullptr;
-  for (int j = 0; j < p.out_channels; ++j) {
-    const bf16* w = p.W + static_cast<int64_t>(j) * p.K;
-    float acc = 0.f;
-    for (int k = lane * 8; k < p.K; k += 256) {
-      const float4 va = *reinterpret_cast<const float4*>(x + k);
-      const float4 vb = *reinterpret_cast<const float4*>(x + k + 4);
-      float fx[8] = {va.x, va.y, va.z, va.w, vb.x, vb.y, vb.z, vb.w}, fw[8];
-      unpack_bf16x8(*reinterpret_cast<const uint4*>(w + k), fw);
-      float g[8], bb[8];
-      if (p.g) unpack_bf16x8(*reinterpret_cast<const uint4*>(p.g + k), g);
-      if (p.b) unpack_bf16x8(*reinterpret_cast<const uint4*>(p.b + k), bb);
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        float y = (fx[q] - mean) * rstd;
-        if (p.g) y *= g[q];
-        if (p.b) y += bb[q];
-        if (sc) y = y * (1.f + sc[k + q]) + sh[k + q];
-        acc = fmaf(y, fw[q], acc);
+  for (int j = 0; j < MAXV; ++j) {
+    const int i = lane + 32 * j;
+    if (i < nv) v[j] = norm_affine4(p, i, v[j], mean, rstd, sc, sh);
+  }
+  float res0 = 0.f, res1 = 0.f;
+  for (int c = 0; c < p.out_channels; ++c) {
+    const uint2* w = reinterpret_cast<const uint2*>(p.W + static_cast<int64_t>(c) * p.K);
+    float acc = 0.f;
+#pragma unroll
+    for (int j = 0; j < MAXV; ++j) {
+      const int i = lane + 32 * j;
+      if (i < nv) {
+        const uint2 u = __ldg(w + i);
+        const __nv_bfloat162* wb = reinterpret_cast<const __nv_bfloat162*>(&u);
+        const float2 w01 = __bfloat1622float2(wb[0]), w23 = __bfloat1622float2(wb[1]);
+        acc = fmaf(v[j].x, w01.x, acc);
+        acc = fmaf(v[j].y, w01.y, acc);
+        acc = fmaf(v[j].z, w23.x, acc);
+        acc = fmaf(v[j].w, w23.y, acc);
       }
     }
     acc = warp_sum(acc);
-    if (lane == 0) out[j] = acc;
+    if (c < 32)
+      res0 = lane == c ? acc : res0;
+    else
+      res1 = lane == c - 32 ? acc : res1;
   }
+  if (lane < p.out_channels) out[lane] = res0;
+  if (lane + 32 < p.out_channels) out[lane + 32] = res1;
 }
 
 __global__ void copy_out_kernel(const IoSlot* slot, const float* h, int64_t n4) {
@@ -679,6 +794,11 @@ cudaError_t io_set_launch(IoSlot* slot, const IoSlot& v, cudaStream_t s) {
 }
 
 cudaError_t stem_launch(const StemParams& p, cudaStream_t s) {
+  if ((p.kind == SGD_STEM_PATCH || p.kind == SGD_STEM_PATCH_TOKENS) && p.d % 4 == 0 && p.d_in % 8 == 0 &&
+      p.d_in > 0) {
+    const int64_t total4 = static_cast<int64_t>(p.batch) * p.n_tokens * (p.d / 4);
+    return launch_k(stem_patch_kernel, dim3(static_cast<unsigned>((total4 + 255) / 256)), dim3(256), 0, s, p);
+  }
   const int64_t total = static_cast<int64_t>(p.batch) * p.n_tokens * p.d;
   return launch_k(stem_kernel, dim3(static_cast<unsigned>((total + 255) / 256)), dim3(256), 0, s, p);
 }
@@ -691,13 +811,17 @@ cudaError_t gemv_launch_r(const GemvParams& p, size_t smem, cudaStream_t s) {
     if (e != cudaSuccess) return e;
   }
   const int cols_per_block = 8 * kGemvCols;
-  return launch_k(gemv_kernel<RMAX>, dim3((p.N + cols_per_block - 1) / cols_per_block), dim3(256), smem, s, p);
+  const dim3 grid((p.N + cols_per_block - 1) / cols_per_block, p.n_seg > 0 ? p.n_seg : 1);
+  return launch_k(gemv_kernel<RMAX>, grid, dim3(256), smem, s, p);
 }
 
 cudaError_t gemv_launch(const GemvParams& p, cudaStream_t s) {
   const int xrows = p.x_sinusoid ? 1 : (p.ldx == 0 ? 1 : p.rows);
   const size_t smem = static_cast<size_t>(xrows) * p.K * sizeof(float);
-  if (p.rows > 16 || smem > 200 * 1024 || (p.K % 8)) return cudaErrorInvalidValue;
+  if (p.rows > 16 || smem > 200 * 1024 || (p.K % 8) || p.n_seg < 0 || p.n_seg > kGemvMaxSeg ||
+      (p.n_seg > 0 && (p.out_silu || p.add_class || p.add_vec)) ||
+      (!p.x_sinusoid && ((p.ldx % 4) || (reinterpret_cast<uintptr_t>(p.x) & 15u))))
+    return cudaErrorInvalidValue;
   if (xrows == 1) return gemv_launch_r<1>(p, smem, s);
   if (xrows <= 8) return gemv_launch_r<8>(p, smem, s);
   return gemv_launch_r<16>(p, smem, s);
@@ -705,7 +829,15 @@ cudaError_t gemv_launch(const GemvParams& p, cudaStream_t s) {
 
 cudaError_t head_small_launch(const HeadParams& p, cudaStream_t s) {
   const int64_t rows = static_cast<int64_t>(p.batch) * p.n_tokens;
-  return launch_k(head_small_kernel, dim3(static_cast<unsigned>((rows + 7) / 8)), dim3(256), 0, s, p);
+  const dim3 grid(static_cast<unsigned>((rows + 7) / 8));
+  if (p.K % 4 || p.K > 4096 || p.out_channels > 64 || p.out_channels > p.N || p.ldx % 4 ||
+      (p.shift && p.ld_mod % 4))
+    return cudaErrorInvalidValue;
+  if (p.K <= 512) return launch_k(head_small_kernel<4>, grid, dim3(256), 0, s, p);
+  if (p.K <= 1024) return launch_k(head_small_kernel<8>, grid, dim3(256), 0, s, p);
+  if (p.K <= 1536) return launch_k(head_small_kernel<12>, grid, dim3(256), 0, s, p);
+  if (p.K <= 2048) return launch_k(head_small_kernel<16>, grid, dim3(256), 0, s, p);
+  return launch_k(head_small_kernel<32>, grid, dim3(256), 0, s, p);
 }
 
 cudaError_t copy_out_launch(const IoSlot* slot, const float* h, int64_t n, cudaStream_t s) {

@@ -332,8 +332,7 @@ int gemm_plan(GemmPlan& p, const char** why) {
   // tile shape: 128-column tiles when they need clearly fewer tile-times than 256-column
   // tiles (a 128-column tile takes half the time of a 256-column one, at about 3/4 of its
   // efficiency, so: 2 * waves_128 < 3 * waves_256) and stream-K does not already even out
-  // the last wave; they need a plain epilogue and one-CTA launches.  4 epilogue warps for
-  // RoPE and gated epilogues.
+  // the last wave; they need a plain epilogue and one-CTA launches.
   const bool small_ok = !gated && e.kind != SGD_EPI_ROPE && p.bk == 64;
   // 128 x 224 tiles where they fill whole waves exactly, K is long and the last column of
   // tiles wastes under a tenth of N (e.g. M = N = 4096 at K >= 3072: 608 tiles = 4 waves;
@@ -352,7 +351,12 @@ int gemm_plan(GemmPlan& p, const char** why) {
   }
   if ((p.bn != 128 && p.bn != 224) || !small_ok) p.bn = 256;
   if (p.bn == 224) p.sk = 0;
-  if (p.epiw == 0) p.epiw = (e.kind == SGD_EPI_ROPE || gated) ? 4 : 8;
+  // 8 epilogue warps (two per TMEM lane quarter, staged stores) except for RoPE, whose
+  // per-thread state needs the 4-warp kernel's registers, and long-K gated MLPs, whose
+  // epilogue hides behind the main loop (device time per launch: gated 2048 x 5120 x 1280
+  // 44.9 against 65.0 us with 4 warps, 4096 x 12288 x 4096 495 against 491 us; RoPE
+  // 4096 x 12288 x 4096 259 against 305 us with 8)
+  if (p.epiw == 0) p.epiw = (e.kind == SGD_EPI_ROPE || (gated && p.K >= 3072)) ? 4 : 8;
   if (p.bn == 128 || p.bn == 224 || p.bk == 32) p.epiw = 8;
   if (p.encode && (!make_tmap_f16(&p.tmap_a, p.A, p.M, p.K, p.lda, 128, p.bk) ||
                    !make_tmap_f16(&p.tmap_b, p.B, b_rows, p.K, p.ldb, p.bn == 224 ? 224 : 128, p.bk))) {

@@ -59,8 +59,12 @@ struct TileCfg {
   static constexpr int kTileBHalf = 128 * BK * 2;
   static constexpr int kTileB = BN * BK * 2;
   static constexpr int kStageBytes = kTileA + kTileB;
-  static constexpr int kStages = BN == 224 ? 5 : (192 * 1024) / kStageBytes;
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+  // epilogue staging: 4 KB per epilogue warp (32 rows x 32 fp32 columns) for the residual
+  // epilogue's coalesced read-modify-write of h; none at BN 224, whose 5 stages fill the rest,
+// nor in the 4-warp kernel
+  static constexpr int kStaging = (BN == 224 || EPIW != 8) ? 0 : EPIW * 4096;
+  static constexpr int kStages = BN == 224 ? 5 : (224 * 1024 - kStaging) / kStageBytes;
+  static constexpr int kSmemBytes = kStages * kStageBytes + kStaging + 1024 /*align*/ + 256 /*barriers*/;
   static_assert(kSmemBytes <= 232448, "shared memory");
   static_assert((2 * kStages + 5) * 8 + 4 * 4 <= 256, "barrier block");
 };
@@ -330,6 +334,143 @@ __device__ __forceinline__ void emit_stats(const EpiParams& e, int row, int slot
   e.stat_out[static_cast<int64_t>(kStatSlots + slot) * e.stat_out_ld + row] = s1;
 }
 
+// Residual epilogue through this warp's 4 KB staging buffer `stg` (32 rows x 8 float4,
+// 16-byte chunk j of row r at r * 8 + (j ^ (r & 7)), so that both access patterns below are
+// free of bank conflicts).  Per 32-column chunk: the warp loads its 32 rows of h coalesced
+// (8 lanes per 128-byte row segment), each thread adds its row's accumulator (times the
+// AdaLN gate) in shared memory, and the warp stores h and the fp16 cache coalesced.  With
+// one thread per row the same accesses touch 32 rows per instruction, which made the
+// epilogue of a short-K projection take longer than its main loop.
+template <class Src>
+__device__ __forceinline__ void delta_staged(const TcArgs& a, int row, int n0, const Src& src, int cb, int ce,
+                                             float4* stg) {
+  const EpiParams& e = a.epi;
+  const int lane = threadIdx.x & 31;
+  const int row0 = row - lane;  // the warp's first row
+  const int lr = lane >> 3, lc = lane & 7;
+  const bool row_ok = row < a.M;
+  const float* grow =
+      e.gate ? e.gate + static_cast<int64_t>(row_ok ? row / e.rows_per_batch : 0) * e.ld_gate + n0 : nullptr;
+#pragma unroll 1
+  for (int c = cb; c < ce; c += 32) {
+    const int col0 = n0 + c;
+    if (col0 >= a.N) break;
+    const bool c_ok = col0 + 4 * lc < a.N;  // this lane's float4 in the coalesced phases (N % 8 == 0)
+    {
+      float4 hv[8];
+#pragma unroll
+      for (int it = 0; it < 8; ++it) {
+        const int r = row0 + it * 4 + lr;
+        hv[it] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (r < a.M && c_ok)
+          hv[it] = *reinterpret_cast<const float4*>(e.h + static_cast<int64_t>(r) * e.ldh + col0 + 4 * lc);
+      }
+#pragma unroll
+      for (int it = 0; it < 8; ++it) {
+        const int r = it * 4 + lr;
+        stg[r * 8 + (lc ^ (r & 7))] = hv[it];
+      }
+    }
+    __syncwarp();
+    float x[16], y[16];
+    src.load2(c, c + 16, x, y);
+    if (grow) {  // columns past N (the tile's edge) read the row's last four, never stored
+#pragma unroll
+      for (int g = 0; g < 8; ++g) {
+        const float4 gv = *reinterpret_cast<const float4*>(grow + min(c + 4 * g, a.N - n0 - 4));
+        float* v = g < 4 ? x + 4 * g : y + 4 * (g - 4);
+        v[0] *= gv.x; v[1] *= gv.y; v[2] *= gv.z; v[3] *= gv.w;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float* v = j < 4 ? x + 4 * j : y + 4 * (j - 4);
+      float4& hs = stg[lane * 8 + (j ^ (lane & 7))];
+      float4 h4 = hs;
+      h4.x += v[0]; h4.y += v[1]; h4.z += v[2]; h4.w += v[3];
+      hs = h4;
+    }
+    __syncwarp();
+#pragma unroll
+    for (int it = 0; it < 8; ++it) {
+      const int r = it * 4 + lr;
+      if (row0 + r < a.M && c_ok)
+        *reinterpret_cast<float4*>(e.h + static_cast<int64_t>(row0 + r) * e.ldh + col0 + 4 * lc) =
+            stg[r * 8 + (lc ^ (r & 7))];
+    }
+    if (e.cache) {
+      __syncwarp();
+      uint4* su = reinterpret_cast<uint4*>(stg);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) su[lane * 8 + (j ^ (lane & 7))] = pack_f16x8(j < 2 ? x + 8 * j : y + 8 * (j - 2));
+      __syncwarp();
+      const int lr4 = lane >> 2, lc4 = lane & 3;
+      const bool c8_ok = col0 + 8 * lc4 < a.N;
+#pragma unroll
+      for (int it = 0; it < 4; ++it) {
+        const int r = it * 8 + lr4;
+        if (row0 + r < a.M && c8_ok)
+          *reinterpret_cast<uint4*>(e.cache + static_cast<int64_t>(row0 + r) * e.ld_cache + col0 + 8 * lc4) =
+              su[r * 8 + (lc4 ^ (r & 7))];
+      }
+    }
+    __syncwarp();  // the next chunk overwrites the staging buffer
+  }
+}
+
+// Coalesced stores through this warp's staging buffer (layout as in delta_staged): every
+// thread puts 32 consecutive output values of its row (columns col0 .. col0 + 31), 16 at a
+// time (put16 with half 0, then 1), and flush stores rows row0 .. row0 + 31.  fp16: 64
+// bytes per row, stored as 4 lanes x 16 bytes per row (head-padded layouts remap each
+// 8-column group); fp32: 128 bytes per row, 8 lanes per row.
+__device__ __forceinline__ void stage_put16_f16(float4* stg, int half, const float* v) {
+  const int lane = threadIdx.x & 31;
+  uint4* su = reinterpret_cast<uint4*>(stg);
+  su[lane * 8 + ((2 * half) ^ (lane & 7))] = pack_f16x8(v);
+  su[lane * 8 + ((2 * half + 1) ^ (lane & 7))] = pack_f16x8(v + 8);
+}
+
+__device__ __forceinline__ void stage_flush_f16(const EpiParams& e, void* out, int row0, int M, int N, int col0,
+                                                float4* stg) {
+  const int lane = threadIdx.x & 31;
+  const uint4* su = reinterpret_cast<const uint4*>(stg);
+  __syncwarp();
+  const int lr4 = lane >> 2, lc4 = lane & 3;
+  const int col = col0 + 8 * lc4;
+  const int dcol = e.pad_src ? (col / e.pad_src) * e.pad_dst + col % e.pad_src : col;
+  f16* o = reinterpret_cast<f16*>(out);
+#pragma unroll
+  for (int it = 0; it < 4; ++it) {
+    const int r = it * 8 + lr4;
+    if (row0 + r < M && col < N)
+      *reinterpret_cast<uint4*>(o + static_cast<int64_t>(row0 + r) * e.ldo + dcol) = su[r * 8 + (lc4 ^ (r & 7))];
+  }
+  __syncwarp();  // the next chunk overwrites the staging buffer
+}
+
+__device__ __forceinline__ void stage_put16_f32(float4* stg, int half, const float* v) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    stg[lane * 8 + ((4 * half + j) ^ (lane & 7))] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+}
+
+__device__ __forceinline__ void stage_flush_f32(const EpiParams& e, void* out, int row0, int M, int N, int col0,
+                                                float4* stg) {
+  const int lane = threadIdx.x & 31;
+  __syncwarp();
+  const int lr = lane >> 3, lc = lane & 7;
+  const int col = col0 + 4 * lc;
+  float* o = reinterpret_cast<float*>(out);
+#pragma unroll
+  for (int it = 0; it < 8; ++it) {
+    const int r = it * 4 + lr;
+    if (row0 + r < M && col < N)
+      *reinterpret_cast<float4*>(o + static_cast<int64_t>(row0 + r) * e.ldo + col) = stg[r * 8 + (lc ^ (r & 7))];
+  }
+  __syncwarp();
+}
+
 // Epilogue of one 128 x BN accumulator: this thread owns tile row `row` and handles
 // accumulator columns [cb, ce) (gated: output columns [cb, ce) of the BN / 2 the tile
 // produces), reading the accumulator through `src`.  `part` (0 or 1) is the column half
@@ -337,7 +478,8 @@ __device__ __forceinline__ void emit_stats(const EpiParams& e, int row, int slot
 // puts its row sums in stat slot 2 n_blk + part.
 template <int BN, bool kFastRope, int FEAT, class Src>
 __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int row, int n_blk,
-                                              const Src& src, int cb, int ce, int part, int halves) {
+                                              const Src& src, int cb, int ce, int part, int halves,
+                                              float4* stg) {
   constexpr int kBN = BN;
   constexpr bool kH16 = FEAT == kFeatH16;
   // compile-time pruning of paths a feature set never takes (gemm_plan enforces it): a
@@ -349,6 +491,26 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
   float x[16], y[16];
   if (!kH16 && a.gated) {
     const int n0 = n_blk * (kBN / 2);
+    if constexpr (!kFastRope) {
+      if (stg != nullptr) {  // 32 output columns (two 16-column groups) per staged store
+#pragma unroll 1
+        for (int c = cb; c < ce; c += 32) {
+          if (n0 + c >= a.N) break;
+#pragma unroll
+          for (int half = 0; half < 2; ++half) {
+            const int cc = c + 16 * half;
+            src.load2(cc, kBN / 2 + cc, x, y);
+            apply_norm16<FEAT>(e, rn, n0 + cc, x);
+            apply_norm16<FEAT>(e, rn, a.N + n0 + cc, y);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) x[i] = e.act ? x[i] * gelu_erf_f(y[i]) : silu_f(x[i]) * y[i];
+            stage_put16_f16(stg, half, x);
+          }
+          stage_flush_f16(e, out, row - (threadIdx.x & 31), a.M, a.N, n0 + c, stg);
+        }
+        return;
+      }
+    }
     for (int c = cb; c < ce; c += 16) {
       if (n0 + c >= a.N) break;
       src.load2(c, kBN / 2 + c, x, y);
@@ -453,6 +615,12 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
     return;
   }
   if (!kNormFeat && e.kind == SGD_EPI_DELTA) {
+    if constexpr (!kH16 && !kFastRope) {  // 8-warp kernels (the 4-warp RoPE kernel has no registers to spare)
+      if (stg != nullptr) {
+        delta_staged(a, row, n0, src, cb, ce, stg);
+        return;
+      }
+    }
     // residual update: the chunk's h (and gate) loads are issued together, ahead of the
     // accumulator reads, instead of one dependent load per 8 columns
     // the residual writer (kFeatH16) serves folded-norm models, which have no AdaLN gate
@@ -505,6 +673,33 @@ __device__ __forceinline__ void epilogue_tile(const TcArgs& a, void* out, int ro
       }
     }
     return;
+  }
+  if constexpr (!kH16 && !kFastRope) {
+    if (stg != nullptr && (e.kind == SGD_EPI_F16 || e.kind == SGD_EPI_GELU || e.kind == SGD_EPI_F32)) {
+#pragma unroll 1
+      for (int c = cb; c < ce; c += 32) {
+        if (n0 + c >= a.N) break;
+        src.load2(c, c + 16, x, y);
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          float* v = half ? y : x;
+          apply_norm16<FEAT>(e, rn, n0 + c + 16 * half, v);
+          if (e.kind == SGD_EPI_GELU) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[i] = e.act ? gelu_erf_f(v[i]) : gelu_tanh_f(v[i]);
+          }
+          if (e.kind == SGD_EPI_F32)
+            stage_put16_f32(stg, half, v);
+          else
+            stage_put16_f16(stg, half, v);
+        }
+        if (e.kind == SGD_EPI_F32)
+          stage_flush_f32(e, out, row - (threadIdx.x & 31), a.M, a.N, n0 + c, stg);
+        else
+          stage_flush_f16(e, out, row - (threadIdx.x & 31), a.M, a.N, n0 + c, stg);
+      }
+      return;
+    }
   }
   float st_ss = 0.f, st_s1 = 0.f;
   for (int c = cb; c < ce; c += 32) {
@@ -698,6 +893,12 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* last_flag = reinterpret_cast<volatile int*>(tmem_slot + 2);
   volatile int* fin_flag = reinterpret_cast<volatile int*>(tmem_slot + 3);
+  // this epilogue warp's staging buffer (after the 256-byte barrier block), if the tile has one
+  float4* stg = nullptr;
+  if constexpr (C::kStaging > 0) {
+    if (threadIdx.x >= 64)
+      stg = reinterpret_cast<float4*>(tiles + kStages * kStageBytes + 256) + ((threadIdx.x >> 5) - 2) * 256;
+  }
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -831,7 +1032,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
           if (ok) {
             tc_fence_after();
             epilogue_tile<kBN, kEpiWarps == 4, FEAT>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce,
-                                                     part, kEpiWarps == 8 ? 2 : 1);
+                                                     part, kEpiWarps == 8 ? 2 : 1, stg);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -842,7 +1043,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
         if (!warp_wait(&tfull[acc], aph, abort_flag, a.status, 4)) break;
         tc_fence_after();
         epilogue_tile<kBN, kEpiWarps == 4, FEAT>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce, part,
-                                           kEpiWarps == 8 ? 2 : 1);
+                                           kEpiWarps == 8 ? 2 : 1, stg);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -855,7 +1056,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
         if (ok) {
           tc_fence_after();
           epilogue_tile<kBN, kEpiWarps == 4, FEAT>(a, out, row, n_blk, TmemSrc{tbase, a.epi.alpha}, cb, ce, part,
-                                           kEpiWarps == 8 ? 2 : 1);
+                                           kEpiWarps == 8 ? 2 : 1, stg);
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -892,7 +1093,7 @@ __global__ void __launch_bounds__(TileCfg<BK, BN, EPIW>::kThreads, 1)
       if (*last_flag != 0) {
         __threadfence();
         epilogue_tile<kBN, kEpiWarps == 4, FEAT>(a, out, row, n_blk, WsSrc<kBN>{slot0, nseg, q * 32 + lane, a.epi.alpha},
-                                           cb, ce, part, kEpiWarps == 8 ? 2 : 1);
+                                           cb, ce, part, kEpiWarps == 8 ? 2 : 1, stg);
         if (threadIdx.x == 64) a.sk_cnt[tile] = 0;
       }
       // the CTA that finished the tile (last_flag is CTA-uniform) draws its row block's ticket

@@ -223,6 +223,7 @@ struct StemParams {
 cudaError_t stem_launch(const StemParams& p, cudaStream_t s);
 
 // out[r, j] = sum_k act(x[r, k]) W[j, k] (+ add[r, j]); x fp32 or computed on the fly.
+constexpr int kGemvMaxSeg = 64;
 struct GemvParams {
   float* out;
   int ldo;
@@ -237,6 +238,12 @@ struct GemvParams {
   int n_classes;          // class ids are clamped into [0, n_classes)
   const float* add_vec;   // optional: + add_vec[j] (broadcast over rows)
   float* out_silu;        // optional: silu(out) written alongside (same layout)
+  // n_seg > 0: n_seg independent products with the same x, N, K and ldo in one launch
+  // (W = w_seg[i], out = out_seg[i]; W and out above are ignored) -- the AdaLN modulation
+  // of every block a step runs
+  int n_seg;
+  const bf16* w_seg[kGemvMaxSeg];
+  float* out_seg[kGemvMaxSeg];
 };
 cudaError_t gemv_launch(const GemvParams& p, cudaStream_t s);
 

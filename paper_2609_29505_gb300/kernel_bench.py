@@ -10,6 +10,7 @@ command that the committed ncu summaries under profiles/ were captured from.
     python -m paper_2609_29505_gb300.kernel_bench attention --batch 8 --heads 16 --tokens 256 --dh 72 --head-stride 80
     python -m paper_2609_29505_gb300.kernel_bench frozen --rows 4096 --d 4096 --caches 8
     python -m paper_2609_29505_gb300.kernel_bench norm --rows 4096 --d 4096
+    python -m paper_2609_29505_gb300.kernel_bench trajectory --config dit --budget 0.5 --reps 2
 """
 from __future__ import annotations
 
@@ -25,15 +26,42 @@ EPI = {"f16": binding.EPI_F16, "f32": binding.EPI_F32, "delta": binding.EPI_DELT
        "gated": binding.EPI_GATED, "gelu": binding.EPI_GELU, "rope": binding.EPI_ROPE}
 
 
+GRAPH = False  # --graph: replay the timed launches from one CUDA graph
+
+
 def _time(fn, iters, warmup):
-    for _ in range(warmup):
-        fn()
+    """Average launch time.  Plain: `iters` calls back to back, so a launch shorter than the
+    host's per-call work (argument checks, tensor maps, launch) is timed at the host's rate.
+    With --graph the calls are captured once into a CUDA graph (on a stream that the warm-up
+    calls also used, so the library's per-stream workspace exists before the capture) and
+    the replay is timed: device time per launch, as the step programs run them."""
+    if not GRAPH:
+        for _ in range(warmup):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(iters):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / iters
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        for _ in range(max(warmup, 1)):
+            fn()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        for _ in range(iters):
+            fn()
+    g.replay()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for _ in range(iters):
-        fn()
-    e1.record()
+    with torch.cuda.stream(s):
+        e0.record()
+        g.replay()
+        e1.record()
     torch.cuda.synchronize()
     return e0.elapsed_time(e1) / iters
 
@@ -121,9 +149,55 @@ def case_norm(a):
     return dict(case="norm", rows=a.rows, d=a.d, ms=ms, gbs=6.0 * a.rows * a.d / ms / 1e6)
 
 
+def case_trajectory(a):
+    """Whole trajectories of a synthetic model through sgd_step (its CUDA graphs), timed with
+    CUDA events: the launch sequence the step programs run, for launch lists and captures of
+    the kernels inside a step."""
+    from . import schedule, synth
+    cfg = synth.get_config(a.config)
+    T = a.T or cfg.T
+    w = synth.make_weights(cfg, "cuda")
+    inp = synth.make_inputs(cfg, "cuda")
+    sched = schedule.build_schedule(cfg, w, T, budget=a.budget)
+    model = binding.Denoiser(cfg, w)
+    model.set_schedule(T, sched["lifetimes"], sched["groups"])
+    if cfg.stem == "embed":
+        xs = [synth.token_ids_at(cfg, inp, s, T).cuda() for s in range(1, T + 1)]
+    else:
+        xs = [inp.z0.cuda()] * T
+    if cfg.head == "logits":
+        out = torch.empty(cfg.batch, cfg.n_tokens, cfg.d_out, dtype=torch.float16, device="cuda")
+    elif cfg.head == "identity":
+        out = torch.empty(cfg.batch, cfg.n_tokens, cfg.d, device="cuda")
+    else:
+        out = torch.empty(cfg.batch, cfg.n_out_tokens, cfg.out_channels, device="cuda")
+    cls = None if inp.class_ids is None else inp.class_ids.cuda()
+    ctx = None if inp.ctx is None else inp.ctx.cuda()
+    times = []
+    for _ in range(a.reps):
+        model.reset()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for s in range(1, T + 1):
+            model.step(xs[s - 1], out, synth.timestep(cfg, s, T), s, class_ids=cls, ctx=ctx)
+        e1.record()
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    model.check_device()
+    model.close()
+    ms = min(times) / T
+    return dict(case="trajectory", config=a.config, T=T, budget=a.budget, reps=a.reps, ms=ms,
+                steps_per_s=1e3 / ms)
+
+
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("case", choices=["gemm", "attention", "frozen", "norm"])
+    ap.add_argument("case", choices=["gemm", "attention", "frozen", "norm", "trajectory"])
+    ap.add_argument("--config", default="dit", help="trajectory: synthetic model config")
+    ap.add_argument("--T", type=int, default=0, help="trajectory: horizon (0: the config's)")
+    ap.add_argument("--budget", type=float, default=0.5, help="trajectory: layer-step budget")
+    ap.add_argument("--reps", type=int, default=2, help="trajectory: whole trajectories")
     ap.add_argument("--M", type=int, default=4096)
     ap.add_argument("--N", type=int, default=12288)
     ap.add_argument("--K", type=int, default=4096)
@@ -153,11 +227,16 @@ def main():
     ap.add_argument("--caches", type=int, default=8)
     ap.add_argument("--iters", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--graph", action="store_true",
+                    help="time the launches replayed from a CUDA graph (device time, no host overhead)")
     a = ap.parse_args()
+    global GRAPH
+    GRAPH = a.graph
     build.build()
     binding.lib()
     res = {"gemm": case_gemm, "attention": case_attention, "frozen": case_frozen,
-           "norm": case_norm}[a.case](a)
+           "norm": case_norm, "trajectory": case_trajectory}[a.case](a)
+    res["graph"] = a.graph
     res["status"] = binding.sgd_kernel_status()
     print(json.dumps(res))
 
