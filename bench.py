@@ -359,7 +359,8 @@ def run_native(args):
         kernels["frozen_run"]["frac_of_hbm"] = round(fz["bytes"] / (fz["ms"] / 1e3) / 1e9 / peaks["hbm"], 4)
 
     # end to end through the C ABI with host buffers (pinned): every step copies its
-    # inputs in and its whole output back; the output copy of step s overlaps step s + 1
+    # inputs in and its whole output back (pinned output buffers: the step's output kernel
+    # writes them directly over the host link)
     e2e = None
     if not args.no_e2e:
         import torch as _t
@@ -386,7 +387,7 @@ def run_native(args):
                "d2h_bytes_per_step": int(outs_h[0].numel() * outs_h[0].element_size()),
                "steps": n_e2e, "over": f"{len(plan)} whole trajectory(ies) of T={T} steps",
                "clocks": clk_e2e.summary(),
-               "api": "sgd_step_host_async + sgd_host_wait (output copy overlaps the next step)"}
+               "api": "sgd_step_host_async + sgd_host_wait (pinned host output written by the step's output kernel)"}
 
     sweep = None
     if args.sweep:

@@ -235,18 +235,19 @@ SGD_API int sgd_step_host(sgd_ctx* ctx, const void* state_in_host, void* out_hos
 
 /*
  * sgd_step_host_async — sgd_step_host without the final wait: the input copy and the
- * step are queued on `stream`, the output copy on a library-owned copy stream, so the
- * copy of step s overlaps the compute of step s + 1 (the device output is
- * double-buffered).  in_host / out_host should be pinned; in_host must stay unchanged
- * until the step's input copy has run, and out_host must not be read until
- * sgd_host_wait returns.  Output copies run in call order on the one copy stream, so a
- * later step may name the same out_host: its copy lands after the earlier one.
+ * step are queued on `stream`.  A pinned out_host (page-locked memory the runtime maps into
+ * the device's address space, e.g. from cudaHostAlloc / cudaMallocHost) is written by the
+ * step's output kernel directly, over the host link; any other out_host gets a copy on a
+ * library-owned copy stream from a double-buffered device output, overlapping the compute
+ * of step s + 1.  in_host should be pinned and must stay unchanged until the step's input
+ * copy has run; out_host must not be read until sgd_host_wait returns.  Writes and copies
+ * land in call order, so a later step may name the same out_host.
  */
 SGD_API int sgd_step_host_async(sgd_ctx* ctx, const void* state_in_host, void* out_host,
                                 float timestep, const int32_t* class_ids_host, const void* ctx_host,
                                 int step, void* stream);
 
-/* sgd_host_wait — wait until every output copy queued by sgd_step_host_async is done. */
+/* sgd_host_wait — wait until every output queued by sgd_step_host_async is in host memory. */
 SGD_API int sgd_host_wait(sgd_ctx* ctx);
 
 /* sgd_get_active_mask — the active set A_s of Sec. 3.1 / Algorithm 2 (unit u is evaluated

@@ -217,6 +217,8 @@ struct sgd_ctx {
   cudaStream_t copy_stream = nullptr;
   cudaEvent_t ev_done[2] = {nullptr, nullptr};
   cudaEvent_t ev_copied[2] = {nullptr, nullptr};
+  cudaEvent_t ev_last = nullptr;  // the last host-mapped step (sgd_host_wait)
+  bool ev_last_used = false;
   int async_slot = 0;
   // input-aware (drift) policy, App. B.1
   int policy = SGD_POLICY_STATIC;
@@ -237,6 +239,7 @@ struct sgd_ctx {
   int64_t graph_steps = 0, eager_steps = 0;
 
   ~sgd_ctx() {
+    if (ev_last_used) cudaEventSynchronize(ev_last);
     if (copy_stream) cudaStreamSynchronize(copy_stream);
     if (ev_drift) cudaEventDestroy(ev_drift);
     if (drift_host) cudaFreeHost(drift_host);
@@ -244,6 +247,7 @@ struct sgd_ctx {
       if (ev_done[i]) cudaEventDestroy(ev_done[i]);
       if (ev_copied[i]) cudaEventDestroy(ev_copied[i]);
     }
+    if (ev_last) cudaEventDestroy(ev_last);
     if (copy_stream) cudaStreamDestroy(copy_stream);
     for (auto e : execs) cudaGraphExecDestroy(e);
     for (auto g : graphs) cudaGraphDestroy(g);
@@ -606,24 +610,28 @@ int build_program(sgd_ctx* c, const std::vector<uint8_t>& active, const std::vec
     g2.n_classes = d.n_classes;
     g2.out_silu = c->cond_silu;
     make_gemv_op(ops, "cond.t2", g2);
-    // the modulation of every block with an active branch, in one launch (it depends on c
-    // only): per-block launches of a 16 MB weight each left most of the GPU idle
+    // the modulation (shift, scale, gate: rows 3 D k .. 3 D k + 3 D of W_mod) of every active
+    // branch k of every block, in one launch: it depends on c only, and per-block launches of
+    // a 16 MB weight each left most of the GPU idle
     GemvParams gm{};
     gm.ldo = 6 * D;
     gm.x = c->cond_silu;
     gm.ldx = D;
     gm.slot = c->slot;
     gm.in_silu = 0;
-    gm.N = 6 * D;
+    gm.N = 3 * D;
     gm.K = D;
     gm.rows = d.batch;
     for (int b = 0; b < d.n_blocks; ++b) {
-      bool any = false;
-      for (int k = 0; k < c->nbr; ++k) any = any || active[b * c->nbr + k];
-      if (!any) continue;  // modulation only for active blocks
-      gm.w_seg[gm.n_seg] = B16(c->blk[b].w_mod);
-      gm.out_seg[gm.n_seg] = c->mod + static_cast<size_t>(b) * d.batch * 6 * D;
-      ++gm.n_seg;
+      for (int k = 0; k < c->nbr; ++k) {
+        if (!active[b * c->nbr + k]) continue;  // modulation only for active branches
+        gm.w_seg[gm.n_seg] = B16(c->blk[b].w_mod) + static_cast<size_t>(k) * 3 * D * D;
+        gm.out_seg[gm.n_seg] = c->mod + static_cast<size_t>(b) * d.batch * 6 * D + static_cast<size_t>(k) * 3 * D;
+        if (++gm.n_seg == kGemvMaxSeg) {
+          make_gemv_op(ops, "mod", gm);
+          gm.n_seg = 0;
+        }
+      }
     }
     if (gm.n_seg > 0) make_gemv_op(ops, "mod", gm);
   }
@@ -1537,6 +1545,7 @@ int sgd_step_host_async(sgd_ctx* c, const void* in_host, void* out_host, float t
       CUDA_TRY(cudaEventCreateWithFlags(&c->ev_copied[i], cudaEventDisableTiming));
       if ((rc = c->alloc(reinterpret_cast<uint8_t**>(&c->st_out2[i]), c->out_bytes(), &c->ws_bytes))) return rc;
     }
+    CUDA_TRY(cudaEventCreateWithFlags(&c->ev_last, cudaEventDisableTiming));
     if (!c->st_in && (rc = c->alloc(reinterpret_cast<uint8_t**>(&c->st_in), c->in_bytes(), &c->ws_bytes))) return rc;
   }
   const int k = c->async_slot;
@@ -1553,6 +1562,21 @@ int sgd_step_host_async(sgd_ctx* c, const void* in_host, void* out_host, float t
   }
   if (ctx_host) cond.ctx = c->st_ctx;
   CUDA_TRY(cudaMemcpyAsync(c->st_in, in_host, c->in_bytes(), cudaMemcpyHostToDevice, s));
+  // pinned host output (device-mapped, as cudaHostAlloc memory is under unified addressing):
+  // the step's output kernel writes it directly over the host link.  A separate copy of
+  // the LLaDA-shaped step's 1 GB of logits ran at ~70 GB/s beside the step's own HBM
+  // traffic and left the GPU waiting for it every step.
+  {
+    cudaPointerAttributes pa{};
+    if (cudaPointerGetAttributes(&pa, out_host) == cudaSuccess && pa.type == cudaMemoryTypeHost &&
+        pa.devicePointer != nullptr) {
+      if ((rc = sgd_step(c, c->st_in, pa.devicePointer, t, &cond, step, stream))) return rc;
+      CUDA_TRY(cudaEventRecord(c->ev_last, s));
+      c->ev_last_used = true;
+      return SGD_OK;
+    }
+    cudaGetLastError();  // a pointer the runtime does not know (pageable memory)
+  }
   // the output buffer of slot k is free once its previous copy to the host has finished
   CUDA_TRY(cudaStreamWaitEvent(s, c->ev_copied[k], 0));
   if ((rc = sgd_step(c, c->st_in, c->st_out2[k], t, &cond, step, stream))) return rc;
@@ -1566,6 +1590,7 @@ int sgd_step_host_async(sgd_ctx* c, const void* in_host, void* out_host, float t
 
 int sgd_host_wait(sgd_ctx* c) {
   if (!c) return fail(SGD_ERR_ARG, "null context");
+  if (c->ev_last_used) CUDA_TRY(cudaEventSynchronize(c->ev_last));
   if (c->copy_stream) CUDA_TRY(cudaStreamSynchronize(c->copy_stream));
   return SGD_OK;
 }

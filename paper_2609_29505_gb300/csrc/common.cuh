@@ -82,13 +82,17 @@ __device__ __forceinline__ uint4 pack_f16x8(const float* f) {
   return u;
 }
 
-__device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
+// SiLU and tanh-GELU as x * sigmoid(.) with the fast exponential and division intrinsics:
+// 0.5 x (1 + tanh(u)) = x / (1 + e^(-2u)), which has no cancellation for negative x (the
+// libm tanhf / expf calls made the activation the longest part of the epilogue of a
+// short-K MLP projection).  An overflowing e^(.) gives x / inf = 0, the limit.
+__device__ __forceinline__ float silu_f(float x) { return __fdividef(x, 1.0f + __expf(-x)); }
 __device__ __forceinline__ float gelu_erf_f(float x) {
   return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
 }
 __device__ __forceinline__ float gelu_tanh_f(float x) {
-  const float c = 0.79788456080286536f;  // sqrt(2/pi)
-  return 0.5f * x * (1.0f + tanhf(c * (x + 0.044715f * x * x * x)));
+  const float c2 = 2.0f * 0.79788456080286536f;  // 2 sqrt(2/pi)
+  return __fdividef(x, 1.0f + __expf(-c2 * (x + 0.044715f * x * x * x)));
 }
 
 // ----------------------------------------------------------------------------

@@ -9,6 +9,7 @@
 //   stem, gemv, head_small, copy_out, pack_f16 — the always-on parts around the
 //                  scheduled units (input stage, conditioning, output head, U-ViT skip
 //                  operands), Sec. 4.2: conditioning and skip features stay current.
+#include <algorithm>
 #include <cmath>
 
 #include "common.cuh"
@@ -449,27 +450,59 @@ __global__ void stem_patch_kernel(const StemParams p) {
 }
 
 // out[r, j] = sum_k act(x[r, k]) W[j, k] for R <= RMAX rows (conditioning and AdaLN
-// modulation: a few rows against a large weight, bound by reading W once).  Each warp owns
-// 4 consecutive columns; a lane streams 16-byte chunks of the 4 weight rows and reuses
-// every x chunk (read once from shared memory per row) across the 4 columns.
+// modulation: a few rows against a large weight, bound by reading W once).  The block stages
+// x once in shared memory and then works through output items (32 consecutive columns of one
+// segment) with a grid of at most two blocks per SM.  Each warp owns 4 columns of an item; a
+// lane streams 16-byte chunks (8 k) of the 4 weight rows and reuses each x chunk across them.
+// x is staged as two planes (k % 8 < 4, k % 8 >= 4) so that the lanes' 16-byte x loads are
+// consecutive (no bank conflicts).  With 8 rows the warp's 4 x 8 partial sums are reduced by
+// a transpose reduction (31 shuffles, lane l ends with value l) instead of 32 butterflies.
 constexpr int kGemvCols = 4;
+
+// v[0..31] of every lane -> lane l returns the warp's sum of value l
+__device__ __forceinline__ float transpose_reduce32(float* v, int lane) {
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    const bool upper = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      const float a = v[i], b = v[i + o];
+      const float send = upper ? a : b;
+      v[i] = (upper ? b : a) + __shfl_xor_sync(0xffffffffu, send, o);
+    }
+  }
+  return v[0];
+}
+
+__device__ __forceinline__ void gemv_store(const GemvParams& p, float* out, int r, int j, float v) {
+  if (p.add_class) {
+    const int cls = min(max(p.slot->class_ids[r], 0), p.n_classes - 1);
+    v += __bfloat162float(p.add_class[static_cast<int64_t>(cls) * p.N + j]);
+  }
+  if (p.add_vec) v += p.add_vec[j];
+  out[static_cast<int64_t>(r) * p.ldo + j] = v;
+  if (p.out_silu) p.out_silu[static_cast<int64_t>(r) * p.ldo + j] = silu_f(v);
+}
+
 template <int RMAX>
 __global__ void __launch_bounds__(256) gemv_kernel(const GemvParams p) {
-  extern __shared__ float xs[];  // [xrows][K]
+  extern __shared__ float xs[];  // [xrows][2 planes][K / 2]
   pdl_wait_and_trigger();
   const int xrows = p.x_sinusoid ? 1 : (p.ldx == 0 ? 1 : p.rows);
+  const int K = p.K, half = K >> 1;
+  // x[r][k] lives at r * K + (k & 4 ? half : 0) + (k >> 3) * 4 + (k & 3)
   if (p.x_sinusoid) {
-    for (int k = threadIdx.x; k < p.K; k += blockDim.x) {
-      float x = sinusoid_at(p.slot->t, p.K, k);
+    for (int k = threadIdx.x; k < K; k += blockDim.x) {
+      float x = sinusoid_at(p.slot->t, K, k);
       if (p.in_silu) x = silu_f(x);
-      xs[k] = x;
+      xs[((k & 4) ? half : 0) + (k >> 3) * 4 + (k & 3)] = x;
     }
   } else {
     // float4 loads (K % 8 == 0, rows 16-byte aligned) in batches of 8 per thread, every load
     // of a batch issued before its first shared-memory store: x is a generic pointer that
     // the compiler cannot tell apart from xs, so a store in between would make each load
     // wait for the previous element's round trip
-    const int k4 = p.K >> 2, n4 = xrows * k4;
+    const int k4 = K >> 2, n4 = xrows * k4;
     constexpr int kBatch = 8;
     for (int i0 = threadIdx.x; i0 < n4; i0 += kBatch * blockDim.x) {
       float4 v[kBatch];
@@ -485,6 +518,7 @@ __global__ void __launch_bounds__(256) gemv_kernel(const GemvParams p) {
       for (int j = 0; j < kBatch; ++j) {
         const int i = i0 + j * blockDim.x;
         if (i < n4) {
+          const int r = i / k4, k = (i - r * k4) << 2;
           float4 x = v[j];
           if (p.in_silu) {
             x.x = silu_f(x.x);
@@ -492,78 +526,82 @@ __global__ void __launch_bounds__(256) gemv_kernel(const GemvParams p) {
             x.z = silu_f(x.z);
             x.w = silu_f(x.w);
           }
-          *reinterpret_cast<float4*>(xs + i * 4) = x;  // = xs[r * K + k]
+          *reinterpret_cast<float4*>(xs + r * K + ((k & 4) ? half : 0) + (k >> 3) * 4) = x;
         }
       }
     }
   }
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int j0 = (blockIdx.x * (blockDim.x >> 5) + warp) * kGemvCols;
-  if (j0 >= p.N) return;
-  const bf16* W = p.n_seg ? p.w_seg[blockIdx.y] : p.W;
-  float* out = p.n_seg ? p.out_seg[blockIdx.y] : p.out;
-  float acc[kGemvCols][RMAX];
+  constexpr int kItemCols = 8 * kGemvCols;  // 8 warps
+  const int per_seg = (p.N + kItemCols - 1) / kItemCols;
+  const int n_items = per_seg * (p.n_seg > 0 ? p.n_seg : 1);
+  for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
+    const int seg = item / per_seg;
+    const int j0 = (item - seg * per_seg) * kItemCols + warp * kGemvCols;
+    if (j0 >= p.N) continue;  // warp-uniform; no block-wide barrier follows
+    const bf16* W = p.n_seg ? p.w_seg[seg] : p.W;
+    float* out = p.n_seg ? p.out_seg[seg] : p.out;
+    float acc[kGemvCols * RMAX];
 #pragma unroll
-  for (int c = 0; c < kGemvCols; ++c)
-#pragma unroll
-    for (int r = 0; r < RMAX; ++r) acc[c][r] = 0.f;
-  // unrolled so that a warp's weight loads for several K steps are in flight together
+    for (int i = 0; i < kGemvCols * RMAX; ++i) acc[i] = 0.f;
+    // unrolled so that a warp's weight loads for several K steps are in flight together
 #pragma unroll 4
-  for (int k = lane * 8; k < p.K; k += 256) {
-    float w[kGemvCols][8];
+    for (int k = lane * 8; k < K; k += 256) {
+      float w[kGemvCols][8];
 #pragma unroll
-    for (int c = 0; c < kGemvCols; ++c) {
-      if (j0 + c < p.N)
-        unpack_bf16x8(*reinterpret_cast<const uint4*>(W + static_cast<int64_t>(j0 + c) * p.K + k), w[c]);
-      else
+      for (int c = 0; c < kGemvCols; ++c) {
+        if (j0 + c < p.N)
+          unpack_bf16x8(__ldg(reinterpret_cast<const uint4*>(W + static_cast<int64_t>(j0 + c) * K + k)), w[c]);
+        else
 #pragma unroll
-        for (int q = 0; q < 8; ++q) w[c][q] = 0.f;
-    }
+          for (int q = 0; q < 8; ++q) w[c][q] = 0.f;
+      }
+      const int xo = (k >> 3) * 4;
 #pragma unroll
-    for (int r = 0; r < RMAX; ++r) {
-      if (r < xrows) {
-        const float4 xa = *reinterpret_cast<const float4*>(xs + r * p.K + k);
-        const float4 xb = *reinterpret_cast<const float4*>(xs + r * p.K + k + 4);
-        const float xv[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
+      for (int r = 0; r < RMAX; ++r) {
+        if (r < xrows) {
+          const float4 xa = *reinterpret_cast<const float4*>(xs + r * K + xo);
+          const float4 xb = *reinterpret_cast<const float4*>(xs + r * K + half + xo);
+          const float xv[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
 #pragma unroll
-        for (int c = 0; c < kGemvCols; ++c)
+          for (int c = 0; c < kGemvCols; ++c)
 #pragma unroll
-          for (int q = 0; q < 8; ++q) acc[c][r] = fmaf(w[c][q], xv[q], acc[c][r]);
+            for (int q = 0; q < 8; ++q) acc[c * RMAX + r] = fmaf(w[c][q], xv[q], acc[c * RMAX + r]);
+        }
       }
     }
-  }
+    if constexpr (kGemvCols * RMAX == 32) {
+      // lane l: column j0 + l / RMAX, row l % RMAX
+      const float v = transpose_reduce32(acc, lane);
+      const int c = lane / RMAX, r = lane % RMAX;
+      if (r < p.rows && j0 + c < p.N) gemv_store(p, out, r, j0 + c, v);
+    } else {
 #pragma unroll
-  for (int c = 0; c < kGemvCols; ++c)
+      for (int i = 0; i < kGemvCols * RMAX; ++i) {
+        if (i % RMAX < xrows) {
 #pragma unroll
-    for (int r = 0; r < RMAX; ++r) {
-      if (r < xrows) {
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) acc[c][r] += __shfl_xor_sync(0xffffffffu, acc[c][r], o);
+          for (int o = 16; o > 0; o >>= 1) acc[i] += __shfl_xor_sync(0xffffffffu, acc[i], o);
+        }
       }
-    }
-  if (lane < kGemvCols && j0 + lane < p.N) {
-    const int j = j0 + lane;
-    // lane c stores column j0 + c; select chains keep acc in registers
-    float vals[RMAX];
+      if (lane < kGemvCols && j0 + lane < p.N) {
+        const int j = j0 + lane;
+        // lane c stores column j0 + c; select chains keep acc in registers
+        float vals[RMAX];
 #pragma unroll
-    for (int rr = 0; rr < RMAX; ++rr) {
-      float v = acc[0][rr];
+        for (int rr = 0; rr < RMAX; ++rr) {
+          float v = acc[rr];
 #pragma unroll
-      for (int c = 1; c < kGemvCols; ++c) v = (lane == c) ? acc[c][rr] : v;
-      vals[rr] = v;
-    }
-    for (int r = 0; r < p.rows; ++r) {
-      float v = vals[0];
+          for (int c = 1; c < kGemvCols; ++c) v = (lane == c) ? acc[c * RMAX + rr] : v;
+          vals[rr] = v;
+        }
+        for (int r = 0; r < p.rows; ++r) {
+          float v = vals[0];
 #pragma unroll
-      for (int rr = 1; rr < RMAX; ++rr) v = (xrows > 1 && rr == r) ? vals[rr] : v;
-      if (p.add_class) {
-        const int cls = min(max(p.slot->class_ids[r], 0), p.n_classes - 1);
-        v += __bfloat162float(p.add_class[static_cast<int64_t>(cls) * p.N + j]);
+          for (int rr = 1; rr < RMAX; ++rr) v = (xrows > 1 && rr == r) ? vals[rr] : v;
+          gemv_store(p, out, r, j, v);
+        }
       }
-      if (p.add_vec) v += p.add_vec[j];
-      out[static_cast<int64_t>(r) * p.ldo + j] = v;
-      if (p.out_silu) p.out_silu[static_cast<int64_t>(r) * p.ldo + j] = silu_f(v);
     }
   }
 }
@@ -811,8 +849,9 @@ cudaError_t gemv_launch_r(const GemvParams& p, size_t smem, cudaStream_t s) {
     if (e != cudaSuccess) return e;
   }
   const int cols_per_block = 8 * kGemvCols;
-  const dim3 grid((p.N + cols_per_block - 1) / cols_per_block, p.n_seg > 0 ? p.n_seg : 1);
-  return launch_k(gemv_kernel<RMAX>, grid, dim3(256), smem, s, p);
+  const int64_t items = static_cast<int64_t>((p.N + cols_per_block - 1) / cols_per_block) * (p.n_seg > 0 ? p.n_seg : 1);
+  const int grid = static_cast<int>(std::min<int64_t>(items, 2 * static_cast<int64_t>(num_sms())));
+  return launch_k(gemv_kernel<RMAX>, dim3(grid), dim3(256), smem, s, p);
 }
 
 cudaError_t gemv_launch(const GemvParams& p, cudaStream_t s) {

@@ -279,9 +279,11 @@ def test_mma_sync_attention_path_within_parity(B, name):
     m.close()
 
 
-def test_async_host_steps_equal_device_steps(B):
-    """Queued host-buffer steps (output copy overlapping the next step) return the same
-    bytes as device steps once sgd_host_wait has returned."""
+@pytest.mark.parametrize("pinned", [True, False], ids=["pinned-direct", "pageable-copy"])
+def test_async_host_steps_equal_device_steps(B, pinned):
+    """Queued host-buffer steps return the same bytes as device steps once sgd_host_wait
+    has returned: pinned outputs written by the step's kernels over the host link, pageable
+    ones through the double-buffered device output and the copy stream."""
     c = case("llada_small", 0.5)
     m = c.model(B)
     out_d = c.out_buffer()
@@ -290,7 +292,9 @@ def test_async_host_steps_equal_device_steps(B):
         m.step(c.ids_at(s).cuda(), out_d, otj.timestep(c.T, s), s)
         want.append(out_d.cpu().clone())
     m.reset()
-    outs = [torch.empty(out_d.shape, dtype=out_d.dtype).pin_memory() for _ in range(c.T)]
+    outs = [torch.empty(out_d.shape, dtype=out_d.dtype) for _ in range(c.T)]
+    if pinned:
+        outs = [o.pin_memory() for o in outs]
     ins = [c.ids_at(s).pin_memory() for s in range(1, c.T + 1)]
     for s in range(1, c.T + 1):
         m.step_host_async(ins[s - 1], outs[s - 1], otj.timestep(c.T, s), s)
